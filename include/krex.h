@@ -1,0 +1,296 @@
+/*
+ * krex.h — C ABI of the GB300 benchmarking-command data path.
+ *
+ * A kernel benchmarking command generates seeded inputs, runs a reference,
+ * runs the candidate once and checks it against the reference, and finally
+ * times the candidate in a loop of warm-up and timed launches, flushing L2
+ * between iterations and summarising the durations (paper Section 2.1,
+ * "Kernel agent" and "Benchmarking command"; Section 1).  Only the timed loop
+ * needs the GPU to itself; the paper brackets it with a critical region
+ * (Section 4.1, region.critical()) whose entry drains outstanding work,
+ * flushes L2 and pins the submitting thread (Section 4.2, "Region entry and
+ * exit", step 5).  This library is the data-parallel GPU work of one such
+ * command on one GPU, plus the region's single-process form.
+ *
+ * Conventions (all entry points):
+ *  - Every function returns a krex_status; nothing throws or aborts.  On
+ *    failure krex_last_error_string() (thread-local) describes the cause.
+ *  - Arguments are validated before any CUDA call; an invalid argument
+ *    returns KREX_ERR_INVALID and launches nothing.
+ *  - Device memory is owned by the caller (e.g. allocated with PyTorch).  The
+ *    library allocates no device memory.  It owns only the CUDA events of a
+ *    region, which krex_region_end / krex_region_abort release.
+ *  - Work is enqueued on the given stream (a cudaStream_t; NULL means the
+ *    legacy default stream) and is asynchronous, except where a function says
+ *    it synchronises.
+ *  - A sticky CUDA error is reported as KREX_ERR_CUDA and never hidden.
+ *  - Matrices are row-major: element (r, c) is at ptr + (r*ld + c)*elem_size.
+ */
+#ifndef KREX_H
+#define KREX_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; declared here so callers need no CUDA headers. */
+typedef struct CUstream_st *krex_stream_t;
+
+typedef enum {
+    KREX_OK = 0,
+    KREX_ERR_INVALID = 1,      /* bad argument (null pointer, bad dtype/shape, size mismatch) */
+    KREX_ERR_UNSUPPORTED = 2,  /* valid but not implemented (alignment, ld, shape class) */
+    KREX_ERR_CUDA = 3,         /* a CUDA runtime/driver call failed */
+    KREX_ERR_STATE = 4,        /* call out of order (region misuse) */
+    KREX_ERR_TIMEOUT = 5,      /* a bounded wait ran out (region drain) */
+    KREX_ERR_DEVICE = 6        /* a kernel reported an error through its status word */
+} krex_status;
+
+typedef enum { KREX_BF16 = 1, KREX_F32 = 2 } krex_dtype;
+
+typedef enum {
+    KREX_DIST_UNIFORM_PM1 = 0, /* U[-1,1] rounded to bf16 (out must be KREX_BF16) */
+    KREX_DIST_NORMAL = 1       /* N(0, sigma^2) in fp32 (out must be KREX_F32)    */
+} krex_dist;
+
+typedef enum {
+    KREX_OP_GEMM_BF16 = 0,     /* C[MxN] = A[MxK] B[KxN]; bf16 in, fp32 accumulate */
+    KREX_OP_SOFTMAX_F32 = 1    /* Y = row softmax of X, fp32                        */
+} krex_op;
+
+/* A caller-owned device matrix.  dtype is a krex_dtype; ld >= cols, in elements. */
+typedef struct {
+    void *ptr;
+    int32_t dtype;
+    int32_t reserved;
+    int64_t rows, cols, ld;
+} krex_buf;
+
+/* Result of krex_check.  max_abs_err is the largest |out - ref| (compared by
+ * IEEE bit pattern, so a NaN difference dominates; 0 for empty inputs). */
+typedef struct {
+    float max_abs_err;
+    uint32_t reserved;
+    uint64_t n_violations;
+} krex_check_result;
+
+/* Options of a critical region (paper Section 4.1 region.critical(); entry
+ * preparation of Section 4.2 step 5).
+ *   max_iters        capacity for timed iterations (1 .. KREX_MAX_ITERS)
+ *   drain_timeout_us how long region_begin may wait for the stream to drain
+ *                    (<= 0: 10 s)
+ *   flush_on_entry   nonzero: write flush_bytes of flush_scratch after the
+ *                    drain (the L2 flush of region entry)
+ *   pin_cpu          nonzero: pin the calling thread to the core it runs on
+ *                    for the region's lifetime, restored at region end
+ *   flush_scratch    device buffer of >= flush_bytes (needed if flush_on_entry)
+ */
+typedef struct {
+    int32_t max_iters;
+    int32_t flush_on_entry;
+    int32_t pin_cpu;
+    int32_t reserved;
+    int64_t drain_timeout_us;
+    void *flush_scratch;
+    size_t flush_bytes;
+} krex_region_opts;
+
+#define KREX_MAX_ITERS 100000
+
+typedef struct krex_region krex_region; /* opaque; created by begin, released by end/abort */
+
+/* ----------------------------------------------------------- inputs ------ */
+
+/* Seeded input generation (Section 2.1: a command generates its inputs before
+ * the check and the timed loop).  Element e = r*cols + c of `out` (logical
+ * row-major index) is element e of the counter-based stream
+ *   key = mix64(seed + (tensor_id+1)*G), draw j = mix64(key + (j+1)*G),
+ * G = 0x9E3779B97F4A7C15, mix64 = the SplitMix64 output mix.
+ * KREX_DIST_UNIFORM_PM1: elements 2j, 2j+1 take bits 63..40 and 31..8 of draw
+ * j; b -> (b - 2^23) 2^-23 rounded to bf16 (RNE).  KREX_DIST_NORMAL: pair j is
+ * a Box-Muller pair from draw j (u1 = (hi24+1) 2^-24, u2 = lo24 2^-24) scaled by
+ * sigma, in fp32.  Output is bit-identical for any launch shape.
+ * Errors: INVALID for a null/empty-but-nonzero buffer, dtype/dist mismatch,
+ * ld < cols, sigma not finite; UNSUPPORTED if ptr is not 16-byte aligned.
+ * Asynchronous. */
+krex_status krex_gen_inputs(uint64_t seed, uint32_t tensor_id, int32_t dist, float sigma,
+                            krex_buf out, krex_stream_t stream);
+
+/* ------------------------------------------------------- candidate ------- */
+
+/* The timed candidate (Section 2.1, Figure 1a's GEMM benchmarking command).
+ * KREX_OP_GEMM_BF16: in[0] = A (M x K, bf16), in[1] = B (K x N, bf16), out = C
+ *   (M x N, bf16, RNE from the fp32 accumulator).  tcgen05 tensor cores with
+ *   TMEM accumulators, TMA loads.  Needs K, N, lda, ldb multiples of 8 and
+ *   16-byte aligned A, B (TMA), else UNSUPPORTED.  K = 0 gives C = 0.
+ * KREX_OP_SOFTMAX_F32: in[0] = X (rows x cols, fp32), out = Y (same shape,
+ *   fp32); y = exp(x - max) / sum exp(x - max) per row, one HBM pass.
+ * Errors: INVALID for wrong n_in, dtypes or shapes; DEVICE if the kernel's
+ * bounded waits ran out (reported by a later krex_device_status call).
+ * Asynchronous. */
+krex_status krex_run_candidate(int32_t op, const krex_buf *in, int32_t n_in, krex_buf out,
+                               krex_stream_t stream);
+
+/* The reference the check compares against (Section 2.1: the command checks
+ * its result against a reference implementation).  CUDA cores only, fp32
+ * accumulation and fp32 output: GEMM ref = fp32 M x N; softmax ref = fp32,
+ * computed in three passes (max, sum, write).  Same shapes and errors as
+ * krex_run_candidate, except that ref must be KREX_F32. Asynchronous. */
+krex_status krex_run_reference(int32_t op, const krex_buf *in, int32_t n_in, krex_buf ref,
+                               krex_stream_t stream);
+
+/* ---------------------------------------------------------- L2 flush ----- */
+
+/* The L2 flush between timed iterations (Section 2.1: harnesses often flush
+ * L2 between iterations; Section 4.2 step 5: region entry flushes L2 with a
+ * write over an L2-sized buffer).  Writes `bytes` bytes of `scratch` (device,
+ * 16-byte aligned); each call writes a different value so no write can be
+ * elided.  bytes = 0 is a no-op.  Asynchronous. */
+krex_status krex_flush_l2(void *scratch, size_t bytes, krex_stream_t stream);
+
+/* Bytes of L2 on the current device (cudaDevAttrL2CacheSize). */
+krex_status krex_l2_bytes(size_t *bytes);
+
+/* ------------------------------------------------------------- check ----- */
+
+/* Bytes of device scratch krex_check needs (at least 16-byte aligned). */
+size_t krex_check_scratch_bytes(void);
+
+/* The correctness check (Section 2.1: check against the reference, return a
+ * verdict).  Per element, in IEEE fp32 without fused multiply-add:
+ *   d = |out - ref|, violation iff !(d <= atol + rtol*|ref|)  (NaN counts).
+ * out may be bf16 or fp32 (widened exactly); ref is fp32 or bf16.  Shapes must
+ * match.  dev_scratch: caller-owned device memory of >= krex_check_scratch_bytes()
+ * bytes; its contents on entry do not matter.  SYNCHRONISES `stream` and writes
+ * *host_result.  The result is bit-identical for any launch shape (max and
+ * count are exact).  Errors: INVALID for null pointers, shape/dtype mismatch,
+ * small scratch. */
+krex_status krex_check(krex_buf out, krex_buf ref, float atol, float rtol, void *dev_scratch,
+                       size_t scratch_bytes, krex_check_result *host_result,
+                       krex_stream_t stream);
+
+/* ------------------------------------------------------------ region ----- */
+
+/* Enter a critical region on `stream` (Section 4.1; Section 4.2 step 5).
+ * Drains the stream: polls cudaStreamQuery, spinning briefly and then
+ * sleeping (the spin-park policy of Section 4.3), until it is idle or
+ * drain_timeout_us passes (-> KREX_ERR_TIMEOUT; nothing is started and no
+ * region is created: a failing entry never starts measurement, Section 4.2).
+ * Then optionally flushes L2 and pins the thread.  The region owns 2*max_iters
+ * CUDA events (pooled across regions).  One region per stream at a time:
+ * begin on a stream that already has an open region returns KREX_ERR_STATE.
+ * *r is set only on success. */
+krex_status krex_region_begin(krex_region **r, krex_stream_t stream, const krex_region_opts *opts);
+
+/* Record the start / end event of the next timed iteration on the region's
+ * stream.  Must alternate begin, end; STATE on misuse; INVALID past max_iters. */
+krex_status krex_iter_begin(krex_region *r);
+krex_status krex_iter_end(krex_region *r);
+
+/* Leave the region: synchronise the last event, read each iteration's
+ * duration (cudaEventElapsedTime, ms), sort a copy and report p50 and p95 by
+ * linear interpolation between order statistics; unpin the thread; release
+ * the region.  durations_ms (may be NULL) receives min(n, cap) durations in
+ * iteration order; *n (may be NULL) the number of timed iterations; p50/p95
+ * (may be NULL) are NaN if there were none.  The region is released even when
+ * an error is returned. */
+krex_status krex_region_end(krex_region *r, float *durations_ms, int32_t cap, int32_t *n,
+                            double *p50_ms, double *p95_ms);
+
+/* Release a region without reading its timings (error paths). */
+krex_status krex_region_abort(krex_region *r);
+
+/* ------------------------------------------------ timing loop (native) --- */
+
+/* The whole timed loop of a benchmarking command in native code: region
+ * entry (drain, flush, pin), `warmup` untimed iterations and `iters` timed
+ * iterations, each = L2 flush (opts->flush_bytes of opts->flush_scratch,
+ * outside the event pair) then the candidate between a start and an end event
+ * (Section 2.1; warm-up belongs inside the region, Section 4.1), then region
+ * end.  durations_ms needs room for `iters` values. */
+krex_status krex_bench_candidate(int32_t op, const krex_buf *in, int32_t n_in, krex_buf out,
+                                 const krex_region_opts *opts, int32_t warmup, int32_t iters,
+                                 float *durations_ms, double *p50_ms, double *p95_ms,
+                                 krex_stream_t stream);
+
+/* ------------------------------------------------------- one command ----- */
+
+/* One benchmarking command (Section 2.1): inputs -> reference -> candidate
+ * once -> check -> timed loop.  */
+typedef struct {
+    int32_t op;                /* krex_op */
+    int32_t warmup;            /* untimed iterations inside the region */
+    int32_t iters;             /* timed iterations (1 .. KREX_MAX_ITERS) */
+    int32_t pin_cpu;           /* pin the thread inside the region */
+    int64_t M, N, K;           /* GEMM: A MxK, B KxN, C MxN.  softmax: rows M, cols N */
+    uint64_t seed;             /* input seed; A = tensor 0, B = tensor 1 (softmax X = 0) */
+    float sigma;               /* softmax inputs: N(0, sigma^2) */
+    float atol, rtol;          /* check tolerances */
+    int32_t reserved;
+    int64_t drain_timeout_us;
+    size_t flush_bytes;        /* L2 flush size per iteration (and at region entry) */
+} krex_command;
+
+/* Device buffers of a command, all caller-owned.  in[0], in[1] (GEMM A, B) or
+ * in[0] (softmax X); out = candidate output; ref = fp32 reference output;
+ * flush_scratch >= flush_bytes; check_scratch >= krex_check_scratch_bytes(). */
+typedef struct {
+    krex_buf in[2];
+    krex_buf out;
+    krex_buf ref;
+    void *flush_scratch;
+    void *check_scratch;
+    size_t check_scratch_bytes;
+} krex_command_bufs;
+
+typedef struct {
+    krex_check_result check;
+    int32_t passed;            /* 1 iff check.n_violations == 0 */
+    int32_t n_iters;           /* timed iterations run (0 if the check failed) */
+    double p50_ms, p95_ms;     /* of the timed iterations */
+    int32_t launches;          /* kernels this command launched */
+    int32_t reserved;
+    double phase_ms[5];        /* host wall time: inputs, reference, candidate, check, timed loop */
+} krex_command_result;
+
+/* Run one command.  host_in (may be NULL): if given, host_in[i] (pinned host
+ * memory, rows*cols contiguous elements of in[i]) is copied to the device
+ * instead of generating the inputs.  host_out (may be NULL): if given, the
+ * candidate output is copied back to it (rows*cols contiguous elements) after
+ * the timed loop.  durations_ms (may be NULL) receives the `iters` timed
+ * durations.  A failing check skips the timed loop (passed = 0, n_iters = 0)
+ * and still returns KREX_OK: the verdict is the result.  SYNCHRONISES. */
+krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *bufs,
+                             const void *const *host_in, void *host_out, float *durations_ms,
+                             krex_command_result *result, krex_stream_t stream);
+
+/* ------------------------------------------------------ host helpers ----- */
+
+/* Linear-interpolated percentile of n host floats (q in [0,1]); host only. */
+krex_status krex_percentile(const float *x, int32_t n, double q, double *out);
+
+/* Read and clear the device-side status word written by kernels whose
+ * bounded waits ran out (0 = none).  Synchronises the device. */
+krex_status krex_device_status(uint32_t *code);
+
+/* Kernels this library has launched in this process, over all entry points
+ * (host-side counter; the bench reports its change over the timed region). */
+uint64_t krex_launch_count(void);
+
+const char *krex_status_string(krex_status s);
+const char *krex_last_error_string(void);
+int32_t krex_version(void);
+
+/* Test hook: enqueue on `stream` a host callback that waits until *gate != 0
+ * (polled every 100 us, at most hold_ms milliseconds), so tests can make a
+ * stream busy from the host and exercise the region drain timeout without
+ * stalling the GPU. */
+krex_status krex_debug_hold_stream(krex_stream_t stream, volatile int32_t *gate, int32_t hold_ms);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KREX_H */

@@ -1,0 +1,58 @@
+// Internal declarations shared by the translation units of libkrex.so.
+// Not part of the public ABI (see include/krex.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "krex.h"
+
+namespace krex {
+
+// ---- device properties (cached per device) -------------------------------
+int sm_count();                 // multiprocessors of the current device
+size_t l2_bytes_current();      // L2 size of the current device
+
+// ---- kernel launchers (return the launch error, never synchronise) --------
+
+// K1: SplitMix64 -> U[-1,1] -> bf16, 16-byte stores.  `key` is the stream key.
+cudaError_t launch_fill_uniform_bf16(uint64_t key, void *out, int64_t rows, int64_t cols,
+                                     int64_t ld, cudaStream_t s);
+// K2: SplitMix64 -> Box-Muller -> N(0, sigma^2) fp32, 16-byte stores.
+cudaError_t launch_fill_normal_f32(uint64_t key, float sigma, float *out, int64_t rows,
+                                   int64_t cols, int64_t ld, cudaStream_t s);
+// K3: grid-stride writer of `bytes` bytes of `value`.
+cudaError_t launch_flush(void *p, size_t bytes, uint32_t value, cudaStream_t s);
+// K6: compare-and-reduce; result (16 bytes) lands in scratch.
+size_t check_scratch_bytes();
+cudaError_t launch_check(const void *out, int out_dtype, int64_t ldo, const void *ref,
+                         int ref_dtype, int64_t ldr, int64_t rows, int64_t cols, float atol,
+                         float rtol, void *scratch, cudaStream_t s);
+// K5: single-pass online row softmax.
+cudaError_t launch_softmax(const float *x, int64_t ldx, float *y, int64_t ldy, int64_t rows,
+                           int64_t cols, cudaStream_t s);
+// K8: three-pass reference softmax.
+cudaError_t launch_softmax_ref(const float *x, int64_t ldx, float *y, int64_t ldy,
+                               int64_t rows, int64_t cols, cudaStream_t s);
+// K7: SIMT fp32 reference GEMM (bf16 in, fp32 out).
+cudaError_t launch_gemm_ref(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb,
+                            float *c, int64_t ldc, int64_t M, int64_t N, int64_t K,
+                            cudaStream_t s);
+// K4: tcgen05 GEMM.  Returns KREX_OK or an error status with a message set.
+krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb,
+                                uint16_t *c, int64_t ldc, int64_t M, int64_t N, int64_t K,
+                                cudaStream_t s);
+// Device status word of the GEMM kernel's bounded waits (read and clear).
+cudaError_t read_and_clear_device_status(uint32_t *code);
+
+// ---- errors -----------------------------------------------------------------
+krex_status set_error(krex_status st, const char *fmt, ...);
+krex_status cuda_error(cudaError_t e, const char *what);
+
+}  // namespace krex
+
+#define KREX_CUDA_TRY(call)                                            \
+    do {                                                               \
+        cudaError_t _e = (call);                                       \
+        if (_e != cudaSuccess) return ::krex::cuda_error(_e, #call);   \
+    } while (0)

@@ -1,0 +1,290 @@
+// K3: the L2-flush writer and K6: the compare-and-reduce correctness check.
+//
+// Flush (paper Section 2.1: harnesses flush L2 between timed iterations;
+// Section 4.2 step 5: region entry flushes L2 by writing an L2-sized buffer):
+// a grid-stride loop of 16-byte stores of a per-call value.
+//
+// Check (Section 2.1: the command checks the candidate against the reference
+// and returns a verdict).  Per element, IEEE fp32 without contraction:
+//     d = |out - ref|,  violation iff !(d <= atol + rtol*|ref|)
+// max |d| is reduced over the IEEE bit pattern as unsigned (valid ordering for
+// non-negative floats; a NaN dominates and is reported as the canonical quiet
+// NaN 0x7FC00000).  Warp reduction with __reduce_max_sync/__reduce_add_sync,
+// one partial per block in scratch, one atomic ticket per block; the last
+// block to take a ticket combines the partials and re-arms the ticket.  Max
+// and count are exact, so the result does not depend on the launch shape.
+#include <cuda_bf16.h>
+
+#include "common.cuh"
+
+namespace krex {
+namespace {
+
+// ------------------------------------------------------------------ flush --
+
+__global__ void __launch_bounds__(512)
+flush_kernel(uint4 *__restrict__ p, size_t n16, uint32_t value, uint8_t *tail, size_t ntail) {
+    const uint4 v = make_uint4(value, value ^ 0x9E3779B9u, value + 1u, ~value);
+    size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const size_t stride = (size_t)gridDim.x * blockDim.x;
+    for (; i + 3 * stride < n16; i += 4 * stride) {
+        p[i] = v;
+        p[i + stride] = v;
+        p[i + 2 * stride] = v;
+        p[i + 3 * stride] = v;
+    }
+    for (; i < n16; i += stride) p[i] = v;
+    if (blockIdx.x == 0 && threadIdx.x < ntail) tail[threadIdx.x] = (uint8_t)value;
+}
+
+// ------------------------------------------------------------------ check --
+
+constexpr int kCheckThreads = 256;
+constexpr int kCheckMaxBlocks = 2048;
+constexpr uint32_t kCanonicalNaN = 0x7FC00000u;
+
+struct Partial {
+    uint32_t max_bits;
+    uint32_t pad;
+    unsigned long long count;
+};
+
+// Scratch layout (device, caller-owned).
+struct CheckScratch {
+    Partial result;          // final {max_bits, count}
+    unsigned int ticket;     // blocks that have published a partial
+    unsigned int pad[3];
+    Partial partial[kCheckMaxBlocks];
+};
+
+__device__ __forceinline__ float widen(const __nv_bfloat16 *p, int64_t i) {
+    return __uint_as_float((uint32_t)(*reinterpret_cast<const uint16_t *>(p + i)) << 16);
+}
+__device__ __forceinline__ float widen(const float *p, int64_t i) { return p[i]; }
+
+struct Acc {
+    uint32_t max_bits = 0;
+    uint32_t count = 0;
+    __device__ __forceinline__ void add(float o, float r, float atol, float rtol) {
+        float d = fabsf(__fsub_rn(o, r));
+        float thr = __fadd_rn(atol, __fmul_rn(rtol, fabsf(r)));
+        count += !(d <= thr);
+        uint32_t b = (d != d) ? kCanonicalNaN : __float_as_uint(d);
+        max_bits = max(max_bits, b);
+    }
+};
+
+__device__ __forceinline__ void bf16x8(const uint4 &u, float *f) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        f[2 * k] = __uint_as_float(w[k] << 16);
+        f[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
+    }
+}
+
+// Publish the block's partial and, in the last block, the final result.
+__device__ __forceinline__ void block_reduce_publish(Acc acc, CheckScratch *sc) {
+    __shared__ uint32_t s_max[kCheckThreads / 32];
+    __shared__ uint32_t s_cnt[kCheckThreads / 32];
+    __shared__ bool s_last;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    uint32_t m = __reduce_max_sync(0xffffffffu, acc.max_bits);
+    uint32_t c = __reduce_add_sync(0xffffffffu, acc.count);
+    if (lane == 0) {
+        s_max[warp] = m;
+        s_cnt[warp] = c;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t bm = 0;
+        unsigned long long bc = 0;
+        for (int w = 0; w < kCheckThreads / 32; ++w) {
+            bm = max(bm, s_max[w]);
+            bc += s_cnt[w];
+        }
+        sc->partial[blockIdx.x].max_bits = bm;
+        sc->partial[blockIdx.x].count = bc;
+        __threadfence();
+        unsigned int t = atomicAdd(&sc->ticket, 1u);
+        s_last = (t == gridDim.x - 1);
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    // last block: combine all partials (exact max and sum)
+    uint32_t bm = 0;
+    unsigned long long bc = 0;
+    for (int b = threadIdx.x; b < (int)gridDim.x; b += blockDim.x) {
+        volatile Partial *p = &sc->partial[b];
+        bm = max(bm, p->max_bits);
+        bc += p->count;
+    }
+    bm = __reduce_max_sync(0xffffffffu, bm);
+    for (int o = 16; o > 0; o >>= 1) bc += __shfl_xor_sync(0xffffffffu, bc, o);
+    __syncthreads();
+    __shared__ unsigned long long s_cnt64[kCheckThreads / 32];
+    if (lane == 0) {
+        s_max[warp] = bm;
+        s_cnt64[warp] = bc;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t fm = 0;
+        unsigned long long fc = 0;
+        for (int w = 0; w < kCheckThreads / 32; ++w) {
+            fm = max(fm, s_max[w]);
+            fc += s_cnt64[w];
+        }
+        sc->result.max_bits = fm;
+        sc->result.pad = 0;
+        sc->result.count = fc;
+        sc->ticket = 0;  // re-arm for the next call
+    }
+}
+
+// Contiguous fast path: bf16 out vs fp32 ref, 8 elements per step.
+__global__ void __launch_bounds__(kCheckThreads)
+check_bf16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref, int64_t n8,
+                   const __nv_bfloat16 *out_s, const float *ref_s, int64_t n, float atol,
+                   float rtol, CheckScratch *sc) {
+    Acc acc;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < n8; g += stride) {
+        uint4 o = __ldcs(out + g);
+        float4 r0 = __ldcs(ref + 2 * g);
+        float4 r1 = __ldcs(ref + 2 * g + 1);
+        float f[8];
+        bf16x8(o, f);
+        acc.add(f[0], r0.x, atol, rtol);
+        acc.add(f[1], r0.y, atol, rtol);
+        acc.add(f[2], r0.z, atol, rtol);
+        acc.add(f[3], r0.w, atol, rtol);
+        acc.add(f[4], r1.x, atol, rtol);
+        acc.add(f[5], r1.y, atol, rtol);
+        acc.add(f[6], r1.z, atol, rtol);
+        acc.add(f[7], r1.w, atol, rtol);
+    }
+    if (blockIdx.x == 0)
+        for (int64_t i = n8 * 8 + threadIdx.x; i < n; i += blockDim.x)
+            acc.add(widen(out_s, i), ref_s[i], atol, rtol);
+    block_reduce_publish(acc, sc);
+}
+
+// Contiguous fast path: fp32 out vs fp32 ref, 4 elements per step, 2 steps unrolled.
+__global__ void __launch_bounds__(kCheckThreads)
+check_f32_f32_vec(const float4 *__restrict__ out, const float4 *__restrict__ ref, int64_t n4,
+                  const float *out_s, const float *ref_s, int64_t n, float atol, float rtol,
+                  CheckScratch *sc) {
+    Acc acc;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    for (; g + stride < n4; g += 2 * stride) {
+        float4 o0 = __ldcs(out + g), r0 = __ldcs(ref + g);
+        float4 o1 = __ldcs(out + g + stride), r1 = __ldcs(ref + g + stride);
+        acc.add(o0.x, r0.x, atol, rtol);
+        acc.add(o0.y, r0.y, atol, rtol);
+        acc.add(o0.z, r0.z, atol, rtol);
+        acc.add(o0.w, r0.w, atol, rtol);
+        acc.add(o1.x, r1.x, atol, rtol);
+        acc.add(o1.y, r1.y, atol, rtol);
+        acc.add(o1.z, r1.z, atol, rtol);
+        acc.add(o1.w, r1.w, atol, rtol);
+    }
+    for (; g < n4; g += stride) {
+        float4 o0 = __ldcs(out + g), r0 = __ldcs(ref + g);
+        acc.add(o0.x, r0.x, atol, rtol);
+        acc.add(o0.y, r0.y, atol, rtol);
+        acc.add(o0.z, r0.z, atol, rtol);
+        acc.add(o0.w, r0.w, atol, rtol);
+    }
+    if (blockIdx.x == 0)
+        for (int64_t i = n4 * 4 + threadIdx.x; i < n; i += blockDim.x)
+            acc.add(out_s[i], ref_s[i], atol, rtol);
+    block_reduce_publish(acc, sc);
+}
+
+// Any layout / dtype pair: one element per step.
+template <typename TO, typename TR>
+__global__ void __launch_bounds__(kCheckThreads)
+check_generic(const TO *out, int64_t ldo, const TR *ref, int64_t ldr, int64_t rows,
+              int64_t cols, float atol, float rtol, CheckScratch *sc) {
+    Acc acc;
+    const int64_t n = rows * cols;
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
+        int64_t r = i / cols, c = i - r * cols;
+        acc.add(widen(out, r * ldo + c), widen(ref, r * ldr + c), atol, rtol);
+    }
+    block_reduce_publish(acc, sc);
+}
+
+int check_blocks(int64_t items) {
+    int64_t b = (items + kCheckThreads - 1) / kCheckThreads;
+    int64_t cap = (int64_t)sm_count() * 8;
+    if (cap > kCheckMaxBlocks) cap = kCheckMaxBlocks;
+    if (b > cap) b = cap;
+    if (b < 1) b = 1;
+    return (int)b;
+}
+
+}  // namespace
+
+size_t check_scratch_bytes() { return sizeof(CheckScratch); }
+
+cudaError_t launch_flush(void *p, size_t bytes, uint32_t value, cudaStream_t s) {
+    if (bytes == 0) return cudaSuccess;
+    size_t n16 = bytes / 16, ntail = bytes % 16;
+    int64_t blocks = (int64_t)((n16 + 511) / 512);
+    int64_t cap = (int64_t)sm_count() * 4;
+    if (blocks > cap) blocks = cap;
+    if (blocks < 1) blocks = 1;
+    flush_kernel<<<(unsigned)blocks, 512, 0, s>>>(static_cast<uint4 *>(p), n16, value,
+                                                  static_cast<uint8_t *>(p) + n16 * 16, ntail);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_check(const void *out, int out_dtype, int64_t ldo, const void *ref,
+                         int ref_dtype, int64_t ldr, int64_t rows, int64_t cols, float atol,
+                         float rtol, void *scratch, cudaStream_t s) {
+    CheckScratch *sc = static_cast<CheckScratch *>(scratch);
+    // zero the result and the ticket: the scratch contents on entry do not matter
+    cudaError_t e = cudaMemsetAsync(sc, 0, offsetof(CheckScratch, partial), s);
+    if (e != cudaSuccess) return e;
+    const int64_t n = rows * cols;
+    const bool contiguous = (ldo == cols && ldr == cols) || rows <= 1;
+    const bool a16 = ((reinterpret_cast<uintptr_t>(out) | reinterpret_cast<uintptr_t>(ref)) & 15u) == 0;
+    if (contiguous && a16 && out_dtype == KREX_BF16 && ref_dtype == KREX_F32) {
+        int64_t n8 = n / 8;
+        check_bf16_f32_vec<<<check_blocks(n8), kCheckThreads, 0, s>>>(
+            static_cast<const uint4 *>(out), static_cast<const float4 *>(ref), n8,
+            static_cast<const __nv_bfloat16 *>(out), static_cast<const float *>(ref), n, atol,
+            rtol, sc);
+    } else if (contiguous && a16 && out_dtype == KREX_F32 && ref_dtype == KREX_F32) {
+        int64_t n4 = n / 4;
+        check_f32_f32_vec<<<check_blocks(n4 / 2), kCheckThreads, 0, s>>>(
+            static_cast<const float4 *>(out), static_cast<const float4 *>(ref), n4,
+            static_cast<const float *>(out), static_cast<const float *>(ref), n, atol, rtol, sc);
+    } else {
+        int blocks = check_blocks(n);
+        if (out_dtype == KREX_BF16 && ref_dtype == KREX_F32)
+            check_generic<__nv_bfloat16, float><<<blocks, kCheckThreads, 0, s>>>(
+                static_cast<const __nv_bfloat16 *>(out), ldo, static_cast<const float *>(ref), ldr,
+                rows, cols, atol, rtol, sc);
+        else if (out_dtype == KREX_F32 && ref_dtype == KREX_F32)
+            check_generic<float, float><<<blocks, kCheckThreads, 0, s>>>(
+                static_cast<const float *>(out), ldo, static_cast<const float *>(ref), ldr, rows,
+                cols, atol, rtol, sc);
+        else if (out_dtype == KREX_BF16 && ref_dtype == KREX_BF16)
+            check_generic<__nv_bfloat16, __nv_bfloat16><<<blocks, kCheckThreads, 0, s>>>(
+                static_cast<const __nv_bfloat16 *>(out), ldo,
+                static_cast<const __nv_bfloat16 *>(ref), ldr, rows, cols, atol, rtol, sc);
+        else
+            check_generic<float, __nv_bfloat16><<<blocks, kCheckThreads, 0, s>>>(
+                static_cast<const float *>(out), ldo, static_cast<const __nv_bfloat16 *>(ref), ldr,
+                rows, cols, atol, rtol, sc);
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace krex

@@ -1,0 +1,493 @@
+// K4: the timed GEMM candidate, C = A B with bf16 operands, fp32 accumulation
+// in tensor memory and bf16 output (paper Section 2.1 and Figure 1a: the GEMM
+// benchmarking command whose timed loop is 8.5% of the command).
+//
+// Blackwell design (sm_103a), one persistent CTA per SM:
+//   warp 0      TMA producer: cp.async.bulk.tensor loads of A (K-major, 128B
+//               swizzle) and B (N-major, 128B swizzle) into a STAGES-deep ring
+//               of shared-memory stages, completion tracked by mbarrier
+//               transaction counts.
+//   warp 1      MMA issuer: one thread issues tcgen05.mma.cta_group::1.kind::f16
+//               (M=128, N=256, K=16) into a TMEM accumulator and releases each
+//               stage with tcgen05.commit.
+//   warp 2      allocates / frees the 512 TMEM columns (two 128x256 fp32
+//               accumulators, so the epilogue of tile i overlaps the MMAs of
+//               tile i+1).
+//   warps 4-7   epilogue: tcgen05.ld 32x32b (each warp owns 32 TMEM lanes = 32
+//               rows), fp32 -> bf16 RNE, 16-byte global stores.
+// Tiles are visited in groups of GROUP_M row blocks so concurrently running
+// CTAs share A and B panels in L2.
+//
+// Every mbarrier wait is bounded (globaltimer); a wait that runs out sets a
+// shared abort flag and the device status word, every role drains what it
+// has in flight (bounded), TMEM is freed and the kernel returns.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+#include <unordered_map>
+
+#include "common.cuh"
+
+namespace krex {
+
+__device__ uint32_t g_gemm_status;  // 0 = ok; else 0x1000 | role << 4 | site
+
+namespace {
+
+constexpr int BM = 128, BN = 256, BK = 64;
+constexpr int STAGES = 4;
+constexpr int A_STAGE_BYTES = BM * BK * 2;          // 16 KiB
+constexpr int B_BOX_N = 64;                         // 64 bf16 = 128-byte swizzle span
+constexpr int B_BOXES = BN / B_BOX_N;               // 4 boxes per stage
+constexpr int B_BOX_BYTES = BK * B_BOX_N * 2;       // 8 KiB
+constexpr int B_STAGE_BYTES = BK * BN * 2;          // 32 KiB
+constexpr int TMEM_COLS = 2 * BN;                   // 512
+constexpr int THREADS = 256;
+constexpr int GROUP_M = 16;
+constexpr int EPI_THREADS = 128;
+constexpr int NUM_BARS = 2 * STAGES + 4 + 1;        // full, empty, tmem_full[2], tmem_empty[2], mma_done
+constexpr size_t SMEM_BYTES = 1024 /*align slack*/ + (size_t)STAGES * (A_STAGE_BYTES + B_STAGE_BYTES) +
+                              NUM_BARS * 8 + 16;
+
+// Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (bits 7-9 =
+// 1), B bf16 (bits 10-12 = 1), A K-major (bit 15 = 0), B MN-major (bit 16 = 1),
+// N >> 3 in bits 17-22, M >> 4 in bits 24-28.
+constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | (1u << 16) |
+                           ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
+
+// Shared-memory matrix descriptor: start >> 4 (bits 0-13), leading byte
+// offset >> 4 (16-29), stride byte offset >> 4 (32-45), version 1 (46-47),
+// base offset 0, swizzle mode 2 = 128B (61-63).
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) | (2ull << 61);
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ uint64_t globaltimer() {
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for the phase with parity `parity` of `bar` to complete.  Returns false
+// if the CTA is aborting (unless `drain`) or `timeout_ns` passed (then it
+// starts the abort).  Drain waits ignore the abort flag: they let work that is
+// already in flight finish before shared memory or TMEM is released.
+__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
+                                       uint64_t timeout_ns, uint32_t site, bool drain = false) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = globaltimer();
+    for (uint32_t spin = 1;; ++spin) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((spin & 63u) == 0) {
+            if (!drain && *abort_flag) return false;
+            if (globaltimer() - t0 > timeout_ns) {
+                *abort_flag = 1u;
+                atomicCAS(&g_gemm_status, 0u, 0x1000u | site);
+                return false;
+            }
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar,
+                                            int32_t c0, int32_t c1) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(IDESC), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+
+// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (thread t <-> lane base+t).
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+          "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
+          "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
+          "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, int &mb, int &nb) {
+    const int per_group = GROUP_M * tiles_n;
+    const int g = tile / per_group;
+    const int first_m = g * GROUP_M;
+    const int gsize = min(tiles_m - first_m, GROUP_M);
+    const int in_g = tile - g * per_group;
+    mb = first_m + in_g % gsize;
+    nb = in_g / gsize;
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+gemm_bf16_tcgen05(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                  uint16_t *__restrict__ C, int64_t ldc, int M, int N, int K, int tiles_m,
+                  int tiles_n, int c_vec, uint64_t timeout_ns) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~uintptr_t(1023));
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + STAGES * A_STAGE_BYTES;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + STAGES * B_STAGE_BYTES);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + NUM_BARS);
+    volatile uint32_t *abort_flag = tmem_slot + 1;
+
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+    auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
+    auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
+    const uint32_t mma_done_bar = bar0 + 8u * (2 * STAGES + 4);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int num_tiles = tiles_m * tiles_n;
+    const int num_kb = (K + BK - 1) / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(full_bar(s), 1);
+            mbar_init(empty_bar(s), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(tfull_bar(a), 1);
+            mbar_init(tempty_bar(a), EPI_THREADS);
+        }
+        mbar_init(mma_done_bar, 1);
+        *abort_flag = 0u;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+    }
+    if (warp == 2) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(TMEM_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        // ------------------------------------------------------ TMA producer
+        int stage = 0;
+        uint32_t phase = 0;
+        int filled = 0;  // total stage fills issued
+        bool ok = true;
+        for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x) {
+            int mb, nb;
+            tile_coords(tile, tiles_m, tiles_n, mb, nb);
+            const int n0 = nb * BN;
+            const int nbox = min(B_BOXES, (N - n0 + B_BOX_N - 1) / B_BOX_N);  // boxes inside N
+            const uint32_t bytes = A_STAGE_BYTES + nbox * B_BOX_BYTES;
+            for (int kb = 0; kb < num_kb; ++kb) {
+                if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, timeout_ns, 0x01)) {
+                    ok = false;
+                    break;
+                }
+                mbar_expect_tx(full_bar(stage), bytes);
+                tma_load_2d(smem_u32(sA + stage * A_STAGE_BYTES), &tmA, full_bar(stage), kb * BK,
+                            mb * BM);
+                for (int j = 0; j < nbox; ++j)
+                    tma_load_2d(smem_u32(sB + stage * B_STAGE_BYTES + j * B_BOX_BYTES), &tmB,
+                                full_bar(stage), n0 + j * B_BOX_N, kb * BK);
+                ++filled;
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+        }
+        if (!ok) {
+            // let the loads already issued land before shared memory is released
+            const int last = filled < STAGES ? filled : STAGES;
+            for (int i = 1; i <= last; ++i) {
+                const int f = filled - i;
+                mbar_wait(full_bar(f % STAGES), (uint32_t)((f / STAGES) & 1), abort_flag,
+                          10000000ull, 0x02, true);
+            }
+        }
+    } else if (warp == 1 && lane == 0) {
+        // --------------------------------------------------------- MMA issuer
+        int stage = 0;
+        uint32_t phase = 0;
+        bool ok = true;
+        int local = 0;
+        for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x, ++local) {
+            const int acc = local & 1;
+            const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
+            if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, timeout_ns, 0x11)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+            for (int kb = 0; kb < num_kb; ++kb) {
+                if (!mbar_wait(full_bar(stage), phase, abort_flag, timeout_ns, 0x12)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint64_t adesc = sdesc_sw128(smem_u32(sA + stage * A_STAGE_BYTES), 16, 1024);
+                const uint64_t bdesc =
+                    sdesc_sw128(smem_u32(sB + stage * B_STAGE_BYTES), B_BOX_BYTES, 1024);
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k) {
+                    // A: +32 bytes along K inside the 128B swizzle row; B: +2 core
+                    // groups of 8 K-rows (2 x 1024 bytes) per K=16 step.
+                    mma_bf16(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(128 * k),
+                             (kb | k) != 0 ? 1u : 0u);
+                }
+                mma_commit(empty_bar(stage));
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (ok) mma_commit(tfull_bar(acc));
+        }
+        // all MMAs issued by this thread complete before TMEM can be freed
+        mma_commit(mma_done_bar);
+        mbar_wait(mma_done_bar, 0u, abort_flag, 10000000ull, 0x13, true);
+    } else if (warp >= 4) {
+        // ----------------------------------------------------------- epilogue
+        const int ew = warp - 4;  // TMEM lanes [32*ew, 32*ew+32)
+        int local = 0;
+        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
+            int mb, nb;
+            tile_coords(tile, tiles_m, tiles_n, mb, nb);
+            const int acc = local & 1;
+            const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
+            // every lane waits; the vote keeps the warp converged (all lanes load
+            // or none) for the .sync.aligned TMEM loads even if a wait runs out
+            const bool waited = mbar_wait(tfull_bar(acc), acc_phase, abort_flag, timeout_ns, 0x21);
+            if (!__all_sync(0xffffffffu, waited)) break;
+            tc_fence_after();
+            const int row = mb * BM + ew * 32 + lane;
+            const int n0 = nb * BN;
+            uint16_t *crow = C + (int64_t)row * ldc;
+#pragma unroll 1
+            for (int c = 0; c < BN / 32; ++c) {
+                const int col0 = n0 + c * 32;
+                if (col0 >= N) break;  // warp-uniform
+                uint32_t v[32];
+                tmem_ld32(tmem_base + ((uint32_t)(ew * 32) << 16) + (uint32_t)(acc * BN + c * 32), v);
+                if (row < M) {
+                    uint32_t p[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        __nv_bfloat162 h =
+                            __floats2bfloat162_rn(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+                        p[i] = *reinterpret_cast<uint32_t *>(&h);
+                    }
+                    if (c_vec && col0 + 32 <= N) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(crow + col0);
+                        dst[0] = make_uint4(p[0], p[1], p[2], p[3]);
+                        dst[1] = make_uint4(p[4], p[5], p[6], p[7]);
+                        dst[2] = make_uint4(p[8], p[9], p[10], p[11]);
+                        dst[3] = make_uint4(p[12], p[13], p[14], p[15]);
+                    } else {
+                        for (int i = 0; i < 32 && col0 + i < N; ++i)
+                            crow[col0 + i] = (uint16_t)((i & 1) ? (p[i >> 1] >> 16) : (p[i >> 1] & 0xFFFFu));
+                    }
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(tempty_bar(acc));
+        }
+    }
+
+    // ---------------------------------------------------------------- teardown
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
+                     "r"(TMEM_COLS)
+                     : "memory");
+    }
+}
+
+// ---------------------------------------------------------------- host side
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+struct MapKey {
+    const void *ptr;
+    uint64_t inner, outer, stride_bytes;
+    uint32_t box_inner, box_outer;
+    bool operator==(const MapKey &o) const {
+        return ptr == o.ptr && inner == o.inner && outer == o.outer &&
+               stride_bytes == o.stride_bytes && box_inner == o.box_inner && box_outer == o.box_outer;
+    }
+};
+struct MapKeyHash {
+    size_t operator()(const MapKey &k) const {
+        size_t h = std::hash<const void *>()(k.ptr);
+        h ^= std::hash<uint64_t>()(k.inner * 0x9E3779B97F4A7C15ull + k.outer) + (h << 6) + (h >> 2);
+        h ^= std::hash<uint64_t>()(k.stride_bytes ^ ((uint64_t)k.box_inner << 32 | k.box_outer)) + (h << 6);
+        return h;
+    }
+};
+
+// 2-D bf16 tensor map: inner dimension contiguous, 128-byte swizzle, OOB -> 0.
+// Encoded maps are cached (a map is a pure function of its key).
+krex_status make_map(const void *ptr, uint64_t inner, uint64_t outer, uint64_t ld_elems,
+                     uint32_t box_inner, uint32_t box_outer, CUtensorMap *out) {
+    static std::mutex mu;
+    static std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
+    MapKey key{ptr, inner, outer, ld_elems * 2, box_inner, box_outer};
+    {
+        std::lock_guard<std::mutex> lk(mu);
+        auto it = cache.find(key);
+        if (it != cache.end()) {
+            *out = it->second;
+            return KREX_OK;
+        }
+    }
+    auto enc = get_encode_fn();
+    if (!enc) return set_error(KREX_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {ld_elems * 2};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides,
+                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return set_error(KREX_ERR_CUDA, "cuTensorMapEncodeTiled failed (CUresult %d)", (int)r);
+    std::lock_guard<std::mutex> lk(mu);
+    if (cache.size() > 4096) cache.clear();
+    cache.emplace(key, *out);
+    return KREX_OK;
+}
+
+uint64_t wait_timeout_ns() {
+    static uint64_t t = [] {
+        const char *e = getenv("KREX_WAIT_TIMEOUT_MS");
+        long ms = e ? atol(e) : 0;
+        if (ms <= 0) ms = 2000;
+        return (uint64_t)ms * 1000000ull;
+    }();
+    return t;
+}
+
+}  // namespace
+
+krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb,
+                                uint16_t *c, int64_t ldc, int64_t M, int64_t N, int64_t K,
+                                cudaStream_t s) {
+    if (M == 0 || N == 0) return KREX_OK;
+    if (K == 0) {
+        KREX_CUDA_TRY(cudaMemset2DAsync(c, (size_t)ldc * 2, 0, (size_t)N * 2, (size_t)M, s));
+        return KREX_OK;
+    }
+    if (M > (1ll << 31) - BM || N > (1ll << 31) - BN || K > (1ll << 31) - BK)
+        return set_error(KREX_ERR_UNSUPPORTED, "GEMM dimension too large for the tcgen05 path");
+    CUtensorMap ma, mb;
+    krex_status st = make_map(a, (uint64_t)K, (uint64_t)M, (uint64_t)lda, BK, BM, &ma);
+    if (st != KREX_OK) return st;
+    st = make_map(b, (uint64_t)N, (uint64_t)K, (uint64_t)ldb, B_BOX_N, BK, &mb);
+    if (st != KREX_OK) return st;
+
+    static thread_local int attr_dev = -1;
+    int dev = 0;
+    KREX_CUDA_TRY(cudaGetDevice(&dev));
+    if (attr_dev != dev) {
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)SMEM_BYTES));
+        attr_dev = dev;
+    }
+    const int tiles_m = (int)((M + BM - 1) / BM), tiles_n = (int)((N + BN - 1) / BN);
+    const int64_t tiles = (int64_t)tiles_m * tiles_n;
+    const int grid = (int)(tiles < sm_count() ? tiles : sm_count());
+    const int c_vec = ((reinterpret_cast<uintptr_t>(c) & 15u) == 0) && (ldc % 8 == 0);
+    gemm_bf16_tcgen05<<<grid, THREADS, SMEM_BYTES, s>>>(ma, mb, c, ldc, (int)M, (int)N, (int)K, tiles_m,
+                                                        tiles_n, c_vec, wait_timeout_ns());
+    KREX_CUDA_TRY(cudaGetLastError());
+    return KREX_OK;
+}
+
+cudaError_t read_and_clear_device_status(uint32_t *code) {
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return e;
+    e = cudaMemcpyFromSymbol(code, g_gemm_status, sizeof(uint32_t));
+    if (e != cudaSuccess) return e;
+    const uint32_t zero = 0;
+    return cudaMemcpyToSymbol(g_gemm_status, &zero, sizeof(uint32_t));
+}
+
+}  // namespace krex

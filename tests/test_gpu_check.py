@@ -1,0 +1,98 @@
+"""GPU parity: the compare-and-reduce check returns exactly the oracle's
+{max_abs_err, n_violations} on the same (host-generated) inputs, for every
+dtype pair, layout, edge case and at the full output sizes."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_30057_gb300 as krex
+import inputs
+from gpu_util import Guarded, to_bf16_tensor
+from oracle import gen, ref
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def scratch():
+    krex.build()
+    return torch.empty(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
+
+
+def _f32_of(bits_or_f32):
+    a = np.asarray(bits_or_f32)
+    return gen.bf16_to_f32(a) if a.dtype == np.uint16 else a.astype(np.float32)
+
+
+def _dev(a):
+    a = np.asarray(a)
+    return to_bf16_tensor(a) if a.dtype == np.uint16 else torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _run(out_h, ref_h, atol, rtol, scratch):
+    got = krex.krex_check(_dev(out_h), _dev(ref_h), atol, rtol, scratch)
+    want = ref.check_f32(_f32_of(out_h), _f32_of(ref_h), atol, rtol)
+    assert got[1] == want[1]
+    assert ref.check_bits(got[0]) == ref.check_bits(want[0])
+    return got
+
+
+@pytest.mark.parametrize("n", [1, 7, 8, 9, 1000, 4097, 100003])
+@pytest.mark.parametrize("pair", ["bf16_f32", "f32_f32", "bf16_bf16", "f32_bf16"])
+def test_check_matches_oracle(n, pair, scratch):
+    r32 = inputs.normal_f32(n, (1, n))
+    o32 = inputs.perturbed(r32, n + 1, 0.3, 0.05)
+    o = inputs.bf16_bits_from_f32(o32) if pair.startswith("bf16") else o32
+    r = inputs.bf16_bits_from_f32(r32) if pair.endswith("bf16") else r32
+    for atol, rtol in ((1e-2, 1e-2), (2.0 ** -12 * 64, 2.0 ** -7), (0.0, 0.0), (1.0, 0.0)):
+        _run(o, r, atol, rtol, scratch)
+
+
+def test_check_strided_layout(scratch):
+    rows, cols, ld = 37, 50, 64
+    r32 = inputs.normal_f32(1, (rows, cols))
+    o32 = inputs.perturbed(r32, 2, 0.2, 0.1)
+    go = Guarded(rows, cols, torch.float32, ld=ld)
+    go.view.copy_(torch.from_numpy(o32))
+    gr = Guarded(rows, cols, torch.float32, ld=ld + 8)
+    gr.view.copy_(torch.from_numpy(r32))
+    got = krex.krex_check(go.view, gr.view, 1e-2, 1e-2, scratch)
+    want = ref.check_f32(o32, r32, 1e-2, 1e-2)
+    assert got[1] == want[1] and ref.check_bits(got[0]) == ref.check_bits(want[0])
+
+
+def test_check_edges(scratch):
+    # exact threshold passes, one ulp above fails; NaN counts and dominates; signed zeros
+    r = np.array([1.0, 1.0, 2.0, 0.0, 3.0, 5.0], dtype=np.float32)
+    o = np.array([1.5, np.nextafter(np.float32(1.5), np.float32(2)), np.nan, -0.0, 3.0, np.inf], dtype=np.float32)
+    mx, nv = _run(o, r, 0.5, 0.0, scratch)
+    assert nv == 3 and math.isnan(mx)
+    _run(r, r, 0.0, 0.0, scratch)
+    # empty inputs
+    e = torch.empty(0, 4, dtype=torch.float32, device="cuda")
+    assert krex.krex_check(e, e, 0.0, 0.0, scratch) == (0.0, 0)
+
+
+def test_check_twice_is_deterministic(scratch):
+    r32 = inputs.normal_f32(5, (512, 512))
+    o32 = inputs.perturbed(r32, 6, 0.5, 1e-3)
+    a, b = _dev(o32), _dev(r32)
+    first = krex.krex_check(a, b, 1e-4, 1e-3, scratch)
+    second = krex.krex_check(a, b, 1e-4, 1e-3, scratch)
+    assert first[1] == second[1] and ref.check_bits(first[0]) == ref.check_bits(second[0])
+
+
+@pytest.mark.parametrize("shape,pair", [((4096, 4096), "bf16_f32"), ((16384, 16384), "bf16_f32"),
+                                         ((65536, 8192), "f32_f32")])
+def test_check_full_size(shape, pair, scratch):
+    # full output sizes of the workloads, planted violations at seeded positions
+    r32 = inputs.normal_f32(17, shape, 4.0)
+    o32 = r32.copy()
+    g = inputs.rng(18)
+    idx = g.integers(0, r32.size, 5000)
+    o32.ravel()[idx] += g.standard_normal(idx.size).astype(np.float32) * 0.5
+    o = inputs.bf16_bits_from_f32(o32) if pair == "bf16_f32" else o32
+    atol, rtol = (2.0 ** -12 * math.sqrt(shape[0]), 2.0 ** -7) if pair == "bf16_f32" else (1e-6, 0.0)
+    _run(o, r32, atol, rtol, scratch)

@@ -1,0 +1,147 @@
+"""GPU parity: the tcgen05 GEMM candidate (and the SIMT reference) against the
+oracle's fp64 GEMM: exact on identity / permutation / small-integer inputs,
+within |d| <= 2^-7 |ref| + 2^-12 sqrt(K) element by element on seeded inputs
+(ragged tails, several tiles and waves), on seeded samples at the large sizes."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_30057_gb300 as krex
+from gpu_util import Guarded, bits16, to_bf16_tensor
+import inputs
+from oracle import gen, ref
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    krex.build()
+
+
+def _gen(seed, M, N, K):
+    a = torch.empty(M, K, dtype=torch.bfloat16, device="cuda")
+    b = torch.empty(K, N, dtype=torch.bfloat16, device="cuda")
+    krex.krex_gen_inputs(seed, 0, krex.KREX_DIST_UNIFORM_PM1, 0.0, a)
+    krex.krex_gen_inputs(seed, 1, krex.KREX_DIST_UNIFORM_PM1, 0.0, b)
+    return a, b
+
+
+def _candidate(a, b, guard=True):
+    M, N = a.shape[0], b.shape[1]
+    c = Guarded(M, N, torch.bfloat16) if guard else None
+    out = c.view if guard else torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [a, b], out)
+    torch.cuda.synchronize()
+    assert krex.krex_device_status() == 0
+    if guard:
+        assert c.canaries_intact()
+    return out
+
+
+def _within_tol(got_bits, want64, K):
+    got = gen.bf16_to_f32(got_bits).astype(np.float64)
+    err = np.abs(got - want64)
+    tol = ref.gemm_tolerance(want64, K)
+    return np.all(err <= tol), float(np.max(err / tol))
+
+
+def test_identity_is_exact():
+    n = 256
+    a, _ = _gen(1, 256, n, 384)
+    eye = to_bf16_tensor(inputs.bf16_bits_from_f32(inputs.identity(384)))
+    c = _candidate(a, eye)
+    assert np.array_equal(bits16(c), bits16(a))
+
+
+def test_permutation_is_exact():
+    a, _ = _gen(2, 128, 512, 512)
+    p, perm = inputs.permutation_matrix(512, 9)
+    c = _candidate(a, to_bf16_tensor(inputs.bf16_bits_from_f32(p)))
+    assert np.array_equal(bits16(c), bits16(a)[:, perm])
+
+
+def test_small_integers_are_exact():
+    # integer operands in [-4, 4]: every partial sum is an integer < 2^8 * K,
+    # exact in fp32; outputs below 256 are exact in bf16
+    M, N, K = 256, 512, 64
+    g = inputs.rng(4)
+    a = g.integers(-4, 5, (M, K)).astype(np.float32)
+    b = g.integers(-4, 5, (K, N)).astype(np.float32)
+    ab, bb = inputs.bf16_bits_from_f32(a), inputs.bf16_bits_from_f32(b)
+    c = _candidate(to_bf16_tensor(ab), to_bf16_tensor(bb))
+    want = ref.gemm_f64(ab, bb)
+    assert np.max(np.abs(want)) < 256
+    assert np.array_equal(gen.bf16_to_f32(bits16(c)).astype(np.float64), want)
+
+
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (128, 256, 128), (256, 512, 256), (100, 72, 40),
+                                   (129, 264, 136), (1, 8, 8), (300, 1000, 520), (1024, 2048, 512),
+                                   (2048, 4096, 1024), (640, 384, 4104)])
+def test_seeded_gemm_within_tolerance(M, N, K):
+    seed = 1000 + M + N + K
+    a, b = _gen(seed, M, N, K)
+    c = _candidate(a, b)
+    want = ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N))
+    ok, worst = _within_tol(bits16(c), want, K)
+    assert ok, worst
+
+
+def test_k_zero_gives_zero_and_empty_is_noop():
+    a = torch.empty(64, 0, dtype=torch.bfloat16, device="cuda")
+    b = torch.empty(0, 32, dtype=torch.bfloat16, device="cuda")
+    c = torch.full((64, 32), 3.0, dtype=torch.bfloat16, device="cuda")
+    krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [a, b], c)
+    torch.cuda.synchronize()
+    assert torch.count_nonzero(c).item() == 0
+    e = torch.empty(0, 16, dtype=torch.bfloat16, device="cuda")
+    krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [e, torch.empty(16, 8, dtype=torch.bfloat16, device="cuda")],
+                            torch.empty(0, 8, dtype=torch.bfloat16, device="cuda"))
+
+
+def test_unsupported_shapes_are_rejected():
+    a = torch.zeros(16, 12, dtype=torch.bfloat16, device="cuda")
+    b = torch.zeros(12, 16, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(krex.KrexError, match="UNSUPPORTED"):
+        krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [a, b], torch.empty(16, 16, dtype=torch.bfloat16,
+                                                                               device="cuda"))
+
+
+@pytest.mark.parametrize("M,N,K", [(256, 256, 256), (300, 1000, 520), (1024, 2048, 512)])
+def test_reference_gemm_within_fp32_bound(M, N, K):
+    seed = 77 + M
+    a, b = _gen(seed, M, N, K)
+    r = Guarded(M, N, torch.float32)
+    krex.krex_run_reference(krex.KREX_OP_GEMM_BF16, [a, b], r.view)
+    torch.cuda.synchronize()
+    assert r.canaries_intact()
+    ah, bh = gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N)
+    want = ref.gemm_f64(ah, bh)
+    absab = np.abs(gen.bf16_to_f32(ah).astype(np.float64)) @ np.abs(gen.bf16_to_f32(bh).astype(np.float64))
+    # fp32 recursive summation bound: |err| <= K u sum|ab| (u = 2^-24), plus output rounding
+    assert np.all(np.abs(r.view.cpu().numpy() - want) <= (K + 2) * 2.0 ** -24 * absab + 1e-30)
+
+
+def test_gemm_4096_full_output():
+    M = N = K = 4096
+    a, b = _gen(2, M, N, K)
+    c = _candidate(a, b, guard=False)
+    want = ref.gemm_f64(gen.uniform_bf16(2, 0, M, K), gen.uniform_bf16(2, 1, K, N))
+    ok, worst = _within_tol(bits16(c), want, K)
+    assert ok, worst
+
+
+@pytest.mark.parametrize("n,seed", [(8192, 4), (16384, 5)])
+def test_gemm_large_sampled(n, seed):
+    a, b = _gen(seed, n, n, n)
+    c = _candidate(a, b, guard=False)
+    i, j = ref.sample_indices(seed, 2, 4096, n, n)
+    got = bits16(c[torch.from_numpy(i).cuda(), torch.from_numpy(j).cuda()])
+    want = ref.gemm_sampled_f64(seed, n, n, n, i, j)
+    ok, worst = _within_tol(got, want, n)
+    assert ok, worst
+    # property at any size: the whole output is finite and bounded by K
+    assert torch.isfinite(c.float()).all().item()
+    assert c.float().abs().max().item() <= n

@@ -1,0 +1,98 @@
+"""GPU parity: seeded input generation is bit-identical to the oracle
+(uniform bf16 and Box-Muller fp32), on ragged, strided and full-size shapes."""
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_30057_gb300 as krex
+from gpu_util import Guarded, bits16
+from oracle import gen, ref
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    krex.build()
+
+
+SHAPES = [(1, 1), (1, 7), (3, 5), (8, 8), (7, 13), (256, 256), (33, 1000), (1000, 1001), (2, 4099)]
+
+
+@pytest.mark.parametrize("rows,cols", SHAPES)
+def test_uniform_bitexact_contiguous(rows, cols):
+    g = Guarded(rows, cols, torch.bfloat16)
+    krex.krex_gen_inputs(7, 1, krex.KREX_DIST_UNIFORM_PM1, 0.0, g.view)
+    torch.cuda.synchronize()
+    assert np.array_equal(bits16(g.view), gen.uniform_bf16(7, 1, rows, cols))
+    assert g.canaries_intact()
+
+
+@pytest.mark.parametrize("rows,cols,ld", [(5, 16, 24), (9, 40, 48), (4, 13, 16), (6, 7, 9)])
+def test_uniform_bitexact_strided(rows, cols, ld):
+    g = Guarded(rows, cols, torch.bfloat16, ld=ld)
+    krex.krex_gen_inputs(11, 0, krex.KREX_DIST_UNIFORM_PM1, 0.0, g.view)
+    torch.cuda.synchronize()
+    assert np.array_equal(bits16(g.view), gen.uniform_bf16(11, 0, rows, cols))
+    assert g.canaries_intact()
+
+
+@pytest.mark.parametrize("rows,cols", SHAPES)
+def test_normal_bitexact_contiguous(rows, cols):
+    g = Guarded(rows, cols, torch.float32)
+    krex.krex_gen_inputs(3, 0, krex.KREX_DIST_NORMAL, 2.0, g.view)
+    torch.cuda.synchronize()
+    got = g.view.cpu().numpy()
+    assert np.array_equal(got.view(np.uint32), gen.normal_f32(3, 0, rows, cols, 2.0).view(np.uint32))
+    assert g.canaries_intact()
+
+
+@pytest.mark.parametrize("rows,cols,ld", [(5, 16, 20), (4, 13, 16), (6, 7, 9)])
+def test_normal_bitexact_strided(rows, cols, ld):
+    g = Guarded(rows, cols, torch.float32, ld=ld)
+    krex.krex_gen_inputs(5, 2, krex.KREX_DIST_NORMAL, 0.75, g.view)
+    torch.cuda.synchronize()
+    assert np.array_equal(g.view.cpu().numpy().view(np.uint32),
+                          gen.normal_f32(5, 2, rows, cols, 0.75).view(np.uint32))
+    assert g.canaries_intact()
+
+
+def test_normal_exhaustive_ln_and_sincos_inputs():
+    # 2^22 pairs cover a large share of the 24-bit u1 and u2 inputs
+    n = 1 << 23
+    t = torch.empty(1, n, dtype=torch.float32, device="cuda")
+    krex.krex_gen_inputs(99, 4, krex.KREX_DIST_NORMAL, 2.0, t)
+    torch.cuda.synchronize()
+    assert np.array_equal(t.cpu().numpy().view(np.uint32), gen.normal_f32(99, 4, 1, n, 2.0).view(np.uint32))
+
+
+@pytest.mark.parametrize("seed,n", [(2, 4096), (4, 8192)])
+def test_uniform_full_size_bitexact(seed, n):
+    for tid, (r, c) in enumerate(((n, n), (n, n))):
+        t = torch.empty(r, c, dtype=torch.bfloat16, device="cuda")
+        krex.krex_gen_inputs(seed, tid, krex.KREX_DIST_UNIFORM_PM1, 0.0, t)
+        torch.cuda.synchronize()
+        assert np.array_equal(bits16(t), gen.uniform_bf16(seed, tid, r, c))
+        del t
+
+
+def test_uniform_16384_sampled_bitexact():
+    n = 16384
+    t = torch.empty(n, n, dtype=torch.bfloat16, device="cuda")
+    krex.krex_gen_inputs(5, 1, krex.KREX_DIST_UNIFORM_PM1, 0.0, t)
+    torch.cuda.synchronize()
+    host = bits16(t).ravel()
+    i, j = ref.sample_indices(5, 7, 1 << 20, n * n, 1)
+    idx = np.concatenate([i, np.arange(4096), np.arange(n * n - 4096, n * n)])
+    assert np.array_equal(host[idx], gen.uniform_bf16_at(5, 1, idx))
+
+
+def test_normal_softmax_input_sampled_bitexact():
+    rows, cols = 65536, 8192
+    t = torch.empty(rows, cols, dtype=torch.float32, device="cuda")
+    krex.krex_gen_inputs(3, 0, krex.KREX_DIST_NORMAL, 2.0, t)
+    torch.cuda.synchronize()
+    host = t.cpu().numpy().ravel()
+    i, _ = ref.sample_indices(3, 9, 1 << 20, rows * cols, 1)
+    idx = np.concatenate([i, np.arange(cols), np.arange(rows * cols - cols, rows * cols)])
+    assert np.array_equal(host[idx].view(np.uint32), gen.normal_f32_at(3, 0, idx, 2.0).view(np.uint32))
