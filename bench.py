@@ -256,6 +256,10 @@ def main():
     ap.add_argument("--no-kernels", action="store_true", help="skip the per-kernel table")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--kernel-only", default=None,
+                    choices=["gemm", "gemm_ref", "fill_uniform", "fill_normal", "flush", "check", "softmax"],
+                    help="launch one kernel of the workload --launches times and exit (for ncu captures)")
+    ap.add_argument("--launches", type=int, default=3)
     args = ap.parse_args()
 
     rank = int(os.environ.get("RANK", "0"))
@@ -264,6 +268,8 @@ def main():
 
     if args.impl == "reference":
         return reference_arm(args, rank, world)
+    if args.kernel_only:
+        return kernel_only(args)
 
     import torch
     import paper_2609_30057_gb300 as krex
@@ -399,6 +405,46 @@ def main():
     print(json.dumps(line))
     if dist is not None:
         dist.destroy_process_group()
+
+
+def kernel_only(args):
+    """Set up the workload (or the softmax workload for softmax / fill_normal),
+    then launch one kernel --launches times; used for ncu captures."""
+    import torch
+    import paper_2609_30057_gb300 as krex
+    from paper_2609_30057_gb300.command import WORKLOADS, Workspace
+    krex.build()
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream()
+    name = SOFTMAX_WORKLOAD if args.kernel_only in ("softmax", "fill_normal") else args.workload
+    w = WORKLOADS[name]
+    ws = Workspace(w)
+    k = args.kernel_only
+    # minimal set-up: inputs, and for the check the two outputs it compares
+    if w.op == 0:
+        krex.krex_gen_inputs(w.seed, 0, 0, 0.0, ws.inputs[0], stream)
+        krex.krex_gen_inputs(w.seed, 1, 0, 0.0, ws.inputs[1], stream)
+    else:
+        krex.krex_gen_inputs(w.seed, 0, 1, w.sigma, ws.inputs[0], stream)
+    if k == "check":
+        krex.krex_run_reference(w.op, ws.inputs, ws.ref, stream)
+        krex.krex_run_candidate(w.op, ws.inputs, ws.out, stream)
+    fn = {
+        "gemm": lambda: krex.krex_run_candidate(0, ws.inputs, ws.out, stream),
+        "gemm_ref": lambda: krex.krex_run_reference(0, ws.inputs, ws.ref, stream),
+        "fill_uniform": lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, ws.inputs[0], stream),
+        "fill_normal": lambda: krex.krex_gen_inputs(w.seed, 0, 1, w.sigma, ws.inputs[0], stream),
+        "flush": lambda: krex.krex_flush_l2(ws.flush, stream=stream),
+        "check": lambda: krex.krex_check(ws.out, ws.ref, w.atol, w.rtol, ws.check_scratch, stream),
+        "softmax": lambda: krex.krex_run_candidate(1, ws.inputs, ws.out, stream),
+    }[k]
+    for _ in range(args.launches):
+        if k != "flush":
+            krex.krex_flush_l2(ws.flush, stream=stream)
+        fn()
+    torch.cuda.synchronize()
+    assert krex.krex_device_status() == 0
+    print(json.dumps({"kernel_only": k, "workload": w.name, "launches": args.launches}))
 
 
 def reference_arm(args, rank, world):
