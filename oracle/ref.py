@@ -104,7 +104,10 @@ def check_f32(out_f32: np.ndarray, ref_f32: np.ndarray, atol: float, rtol: float
       thr = atol + rtol·|ref|
       violation iff not (d ≤ thr)      (a NaN anywhere counts)
     max_abs_err = maximum of d ordered by bit pattern as unsigned, so any NaN
-    dominates; 0 for no elements.  Returns (max_abs_err as float32, n_violations).
+    dominates, and a NaN maximum is reported as the canonical quiet NaN
+    0x7FC00000 (IEEE 754 leaves NaN payloads unspecified, and x86, Arm and the
+    GPU produce different ones); 0 for no elements.
+    Returns (max_abs_err as float32, n_violations).
     """
     o = np.asarray(out_f32, dtype=np.float32).ravel()
     r = np.asarray(ref_f32, dtype=np.float32).ravel()
@@ -114,7 +117,8 @@ def check_f32(out_f32: np.ndarray, ref_f32: np.ndarray, atol: float, rtol: float
         d = np.abs(o - r)
         thr = np.float32(atol) + np.float32(rtol) * np.abs(r)
         viol = ~(d <= thr)
-    mx = d.view(np.uint32).max()
+    bits = np.where(np.isnan(d), np.uint32(0x7FC00000), d.view(np.uint32))
+    mx = bits.max()
     return np.array([mx], dtype=np.uint32).view(np.float32)[0], int(viol.sum())
 
 

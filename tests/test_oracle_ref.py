@@ -158,7 +158,7 @@ def _check_brute(out, ref_, atol, rtol):
         thr = _f32(_f32(atol) + _f32(_f32(rtol) * abs(r)))
         if not (d <= thr):
             nv += 1
-        bits = struct.unpack("I", struct.pack("f", d))[0]
+        bits = 0x7FC00000 if d != d else struct.unpack("I", struct.pack("f", d))[0]
         mx_bits = max(mx_bits, bits)
     return mx_bits, nv
 
@@ -183,6 +183,10 @@ def test_check_nan_counts_and_dominates():
     out = np.array([1.0, np.nan, 3.0], dtype=np.float32)
     mx, nv = ref.check_f32(out, ref_, 1.0, 1.0)
     assert nv == 1 and np.isnan(mx)
+    # any NaN payload, either sign, is reported as the canonical quiet NaN
+    odd_nan = np.array([0xFFC01234], dtype=np.uint32).view(np.float32)
+    mx, nv = ref.check_f32(np.concatenate([out, odd_nan]), np.append(ref_, 1.0), 1.0, 1.0)
+    assert nv == 2 and ref.check_bits(mx) == 0x7FC00000
     mx, nv = ref.check_f32(np.array([np.inf], np.float32), np.array([np.inf], np.float32), 1.0, 0.0)
     assert nv == 1 and np.isnan(mx)                  # inf - inf = NaN
 
