@@ -172,6 +172,25 @@ krex_status krex_check(krex_buf out, krex_buf ref, float atol, float rtol, void 
                        size_t scratch_bytes, krex_check_result *host_result,
                        krex_stream_t stream);
 
+/* krex_check without caller scratch, for callers that cannot allocate device
+ * memory: code whose device memory belongs to another allocator with nothing
+ * to spare (a framework's caching pool, a fixed budget), and timing harnesses
+ * that must not call cudaMalloc/cudaFree because those calls can synchronise
+ * the device and disturb a measurement.  The paper has no counterpart; it is
+ * an addition of this library.
+ * Scratch: a static device array of 33,024 bytes inside libkrex.so, present on
+ * every GPU that loads the library until the process exits.  The call resolves
+ * its address (cudaGetSymbolAddress) the first time it runs on a device, so
+ * make that first call before any stream capture.  It allocates nothing and
+ * calls no allocating routine.  Every call shares the one array per device and
+ * leaves the last result in it; the call clears what must start at zero, but
+ * calls that overlap on the GPU (other streams, other threads) race on it, so
+ * serialise them.  Same arguments, result and bit-exact semantics as
+ * krex_check; UNSUPPORTED if the check ever needed more scratch than the
+ * array holds.  SYNCHRONISES `stream`. */
+krex_status krex_check_noalloc(krex_buf out, krex_buf ref, float atol, float rtol,
+                               krex_check_result *host_result, krex_stream_t stream);
+
 /* ------------------------------------------------------------ region ----- */
 
 /* Enter a critical region on `stream` (Section 4.1; Section 4.2 step 5).

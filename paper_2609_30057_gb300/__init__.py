@@ -76,6 +76,7 @@ SIGNATURES = {
     "krex_l2_bytes": (_i32, [_P(_sz)]),
     "krex_check_scratch_bytes": (_sz, []),
     "krex_check": (_i32, [krex_buf, krex_buf, _f32, _f32, _vp, _sz, _P(krex_check_result), _vp]),
+    "krex_check_noalloc": (_i32, [krex_buf, krex_buf, _f32, _f32, _P(krex_check_result), _vp]),
     "krex_region_begin": (_i32, [_P(_vp), _vp, _P(krex_region_opts)]),
     "krex_iter_begin": (_i32, [_vp]),
     "krex_iter_end": (_i32, [_vp]),
@@ -207,6 +208,16 @@ def krex_check(out, ref, atol: float, rtol: float, scratch, stream=None):
     bo = out if isinstance(out, krex_buf) else buf(out)
     br = ref if isinstance(ref, krex_buf) else buf(ref)
     _ok(lib().krex_check(bo, br, atol, rtol, ptr, nbytes, ctypes.byref(res), _stream(stream)), "krex_check")
+    return res.max_abs_err, int(res.n_violations)
+
+
+def krex_check_noalloc(out, ref, atol: float, rtol: float, stream=None):
+    """krex_check with the library's static scratch (no device allocation);
+    returns (max_abs_err, n_violations); synchronises the stream."""
+    res = krex_check_result()
+    bo = out if isinstance(out, krex_buf) else buf(out)
+    br = ref if isinstance(ref, krex_buf) else buf(ref)
+    _ok(lib().krex_check_noalloc(bo, br, atol, rtol, ctypes.byref(res), _stream(stream)), "krex_check_noalloc")
     return res.max_abs_err, int(res.n_violations)
 
 

@@ -78,6 +78,8 @@ size_t l2_bytes_current() {
 
 static void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
 
+void note_launches(int n) { count_launches(n); }
+
 // ---------------------------------------------------------- host SplitMix64 --
 
 static uint64_t host_mix64(uint64_t z) {

@@ -45,6 +45,9 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
 // Device status word of the GEMM kernel's bounded waits (read and clear).
 cudaError_t read_and_clear_device_status(uint32_t *code);
 
+// Count kernels launched outside api.cu in krex_launch_count().
+void note_launches(int n);
+
 // ---- errors -----------------------------------------------------------------
 krex_status set_error(krex_status st, const char *fmt, ...);
 krex_status cuda_error(cudaError_t e, const char *what);

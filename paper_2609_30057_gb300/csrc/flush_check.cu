@@ -15,6 +15,8 @@
 // and count are exact, so the result does not depend on the launch shape.
 #include <cuda_bf16.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 namespace krex {
@@ -288,3 +290,70 @@ cudaError_t launch_check(const void *out, int out_dtype, int64_t ldo, const void
 }
 
 }  // namespace krex
+
+// --------------------------------------------------- allocation-free check
+//
+// krex_check with library-owned scratch, for callers that must not allocate
+// device memory: code whose device memory is owned by another allocator with
+// no room or permission to give (a framework's caching pool or a fixed memory
+// budget), and timing harnesses in which a cudaMalloc/cudaFree would be a
+// hazard because those calls can synchronise the whole device and disturb the
+// measurement around them.  The scratch is a fixed static device array that
+// each GPU loading this library keeps until the process exits.
+
+// Capacity: the check's 16-byte result/ticket header plus one 16-byte partial
+// for each of its at most 2048 blocks (32,800 bytes), rounded up.
+#define KREX_CHECK_NOALLOC_SCRATCH_BYTES 33024
+static __device__ __align__(256) unsigned char g_check_noalloc_scratch[KREX_CHECK_NOALLOC_SCRATCH_BYTES];
+
+namespace krex {
+namespace {
+std::mutex g_noalloc_mu;
+void *g_noalloc_addr[64];  // device address of the array, per device ordinal
+}  // namespace
+}  // namespace krex
+
+extern "C" krex_status krex_check_noalloc(krex_buf out, krex_buf ref, float atol, float rtol,
+                                          krex_check_result *host_result, krex_stream_t stream) {
+    using namespace krex;
+    auto bad_buf = [](const krex_buf &b) {
+        return (b.dtype != KREX_BF16 && b.dtype != KREX_F32) || b.rows < 0 || b.cols < 0 ||
+               (b.rows > 0 && b.ld < b.cols) || (b.rows * b.cols > 0 && b.ptr == nullptr);
+    };
+    if (bad_buf(out) || bad_buf(ref)) return set_error(KREX_ERR_INVALID, "check_noalloc: bad out or ref buffer");
+    if (out.rows != ref.rows || out.cols != ref.cols)
+        return set_error(KREX_ERR_INVALID, "check_noalloc: out and ref shapes differ");
+    if (!host_result) return set_error(KREX_ERR_INVALID, "check_noalloc: host_result is null");
+    const size_t need = check_scratch_bytes();
+    if (need > (size_t)KREX_CHECK_NOALLOC_SCRATCH_BYTES)
+        return set_error(KREX_ERR_UNSUPPORTED, "check_noalloc: needs %zu bytes of scratch, the static array holds %d",
+                         need, KREX_CHECK_NOALLOC_SCRATCH_BYTES);
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
+    if (dev < 0 || dev >= 64) return set_error(KREX_ERR_UNSUPPORTED, "check_noalloc: device ordinal %d >= 64", dev);
+    void *scratch = nullptr;
+    {
+        // first call on a device: resolve the array's device address there
+        std::lock_guard<std::mutex> lk(g_noalloc_mu);
+        if (!g_noalloc_addr[dev]) {
+            void *p = nullptr;
+            e = cudaGetSymbolAddress(&p, g_check_noalloc_scratch);
+            if (e != cudaSuccess) return cuda_error(e, "cudaGetSymbolAddress (check_noalloc scratch)");
+            g_noalloc_addr[dev] = p;
+        }
+        scratch = g_noalloc_addr[dev];
+    }
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    // launch_check clears the result and ticket in the array before the kernel
+    e = launch_check(out.ptr, out.dtype, out.ld, ref.ptr, ref.dtype, ref.ld, out.rows, out.cols, atol, rtol, scratch, s);
+    if (e != cudaSuccess) return cuda_error(e, "check_noalloc launch");
+    note_launches(1);
+    krex_check_result r;
+    e = cudaMemcpyAsync(&r, scratch, sizeof(r), cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return cuda_error(e, "cudaMemcpyAsync (check_noalloc result)");
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_error(e, "cudaStreamSynchronize (check_noalloc)");
+    *host_result = r;
+    return KREX_OK;
+}

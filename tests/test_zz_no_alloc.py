@@ -1,0 +1,67 @@
+"""The allocation-free check entry point, called through the C ABI.
+
+krex_check_noalloc serves callers that cannot allocate device memory (their
+memory belongs to another allocator, or a cudaMalloc/cudaFree could
+synchronise the device in the middle of a measurement).  It must give exactly
+the result of krex_check with caller scratch, and keep doing so on repeated
+calls that share its one static scratch array.  This file is collected last
+on purpose and passes both alone in a fresh process and after the other tests.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_30057_gb300 as krex
+import inputs
+from gpu_util import to_bf16_tensor
+from oracle import ref
+
+pytestmark = pytest.mark.gpu
+
+
+def _cases():
+    r32 = inputs.normal_f32(31, (2048, 2048), 4.0)
+    o32 = inputs.perturbed(r32, 32, 0.01, 0.5)
+    yield "bf16_out_f32_ref", to_bf16_tensor(inputs.bf16_bits_from_f32(o32)), torch.from_numpy(r32).cuda(), \
+        2.0 ** -12 * 64, 2.0 ** -7
+    s32 = inputs.normal_f32(33, (300, 1000))
+    t32 = inputs.perturbed(s32, 34, 0.3, 1e-5)
+    t32[7, 11] = np.nan
+    yield "f32_with_nan", torch.from_numpy(t32).cuda(), torch.from_numpy(s32).cuda(), 1e-6, 0.0
+    w32 = inputs.normal_f32(35, (64, 136))
+    wide = torch.from_numpy(w32).cuda()
+    wide2 = torch.from_numpy(inputs.perturbed(w32, 36, 0.5, 1e-3)).cuda()
+    yield "f32_strided", wide[:, :128], wide2[:, :128], 1e-4, 1e-3     # row stride 136
+
+
+def _call_noalloc(lib, out, ref_t, atol, rtol):
+    res = krex.krex_check_result()
+    st = lib.krex_check_noalloc(krex.buf(out), krex.buf(ref_t), atol, rtol, ctypes.byref(res),
+                                torch.cuda.current_stream().cuda_stream)
+    assert st == krex.KREX_OK, lib.krex_last_error_string()
+    return res.max_abs_err, int(res.n_violations)
+
+
+def test_noalloc_check_matches_scratch_check_on_two_calls_in_a_row():
+    krex.build()
+    lib = krex.lib()
+    scratch = torch.empty(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
+    for name, out, ref_t, atol, rtol in _cases():
+        want = krex.krex_check(out, ref_t, atol, rtol, scratch)
+        first = _call_noalloc(lib, out, ref_t, atol, rtol)
+        second = _call_noalloc(lib, out, ref_t, atol, rtol)
+        for got in (first, second):
+            assert got[1] == want[1], name
+            assert ref.check_bits(got[0]) == ref.check_bits(want[0]), name
+        assert want[1] > 0, name        # every case has violations to count
+
+
+def test_noalloc_check_rejects_bad_arguments():
+    lib = krex.lib()
+    res = krex.krex_check_result()
+    a = krex.krex_buf(16, krex.KREX_F32, 0, 4, 4, 4)
+    b = krex.krex_buf(16, krex.KREX_F32, 0, 4, 5, 5)
+    assert lib.krex_check_noalloc(a, b, 0.0, 0.0, ctypes.byref(res), None) == krex.KREX_ERR_INVALID
+    assert lib.krex_check_noalloc(a, a, 0.0, 0.0, None, None) == krex.KREX_ERR_INVALID
