@@ -369,6 +369,323 @@ gemm_bf16_tcgen05(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     }
 }
 
+// ===================================================== 2-SM (cta_group::2) form
+//
+// A cluster of two CTAs on a TPC computes a 256 x 256 tile with
+// tcgen05.mma.cta_group::2 (M = 256): CTA r holds rows [128r, 128r+128) of the
+// A tile and columns [128r, 128r+128) of the B tile in its own shared memory,
+// and its own TMEM holds its 128 rows of the 256-column accumulator.  Per SM
+// a stage is 32 KiB (A 128x64 + half of B 64x128), so six stages fit and the
+// L2 -> SM traffic per flop is two thirds of the 1-SM form.
+//   - both CTAs' TMA loads complete on the leader CTA's (rank 0) full barrier
+//     (.cta_group::2 lets the barrier live in the peer CTA);
+//   - the leader's MMA thread releases a stage in both CTAs and publishes an
+//     accumulator to both epilogues with multicast tcgen05.commit;
+//   - each epilogue warp of either CTA tells the leader its accumulator half
+//     is drained with a remote mbarrier arrive.
+
+namespace v2 {
+constexpr int BM = 128;                          // rows per CTA (256 per pair)
+constexpr int BN = 256;                          // widest pair tile (the kernel takes bn <= BN)
+constexpr int BK = 64;
+constexpr int STAGES = 7;
+constexpr int A_STAGE_BYTES = BM * BK * 2;       // 16 KiB
+constexpr int B_HALF = BN / 2;                   // 128 columns per CTA
+constexpr int B_BOX_N = 64;
+constexpr int B_BOXES = B_HALF / B_BOX_N;        // 2
+constexpr int B_BOX_BYTES = BK * B_BOX_N * 2;    // 8 KiB
+constexpr int B_STAGE_BYTES = BK * B_HALF * 2;   // 16 KiB
+constexpr int B_PAD_BYTES = 0;
+constexpr int TMEM_COLS = 2 * BN;                // two 128-lane x 256-column accumulators
+constexpr int GROUP_M = 8;                       // pair-tile rows per raster group
+constexpr int EPI_WARPS = 4;
+constexpr int NUM_BARS = 2 * STAGES + 4 + 1;
+constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * (A_STAGE_BYTES + B_STAGE_BYTES) + B_PAD_BYTES +
+                              NUM_BARS * 8 + 16;
+// kind::f16, D fp32, A/B bf16, A K-major, B MN-major, M = 256 (pair); N is
+// added at run time in bits 17-22
+constexpr uint32_t IDESC_NO_N = (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | (1u << 16) |
+                                ((uint32_t)(256 >> 4) << 24);
+}  // namespace v2
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// shared::cluster address of the same shared variable in CTA `rank`
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+                 : "memory");
+}
+
+// TMA load into this CTA's shared memory, completing on an mbarrier that may
+// live in the peer CTA of the pair (the leader's full barrier).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap *map, uint32_t bar_cluster,
+                                                 int32_t c0, int32_t c1) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(c0), "r"(c1)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                              uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+// Arrive on the barrier at this shared offset in both CTAs of the pair once
+// all MMAs issued so far by this thread have completed.
+__device__ __forceinline__ void mma_commit_pair(uint32_t bar) {
+    const uint16_t mask = 0x3;
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+        " [%0], %1;" ::"r"(bar), "h"(mask)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit_local_pair(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tile_coords_pair(int tile, int tiles_m, int tiles_n, int &mb, int &nb) {
+    const int per_group = v2::GROUP_M * tiles_n;
+    const int g = tile / per_group;
+    const int first_m = g * v2::GROUP_M;
+    const int gsize = min(tiles_m - first_m, v2::GROUP_M);
+    const int in_g = tile - g * per_group;
+    mb = first_m + in_g % gsize;
+    nb = in_g / gsize;
+}
+
+__device__ __forceinline__ void spin_ns(uint64_t ns) {
+    const uint64_t t0 = globaltimer();
+    while (globaltimer() - t0 < ns) {
+    }
+}
+
+// Pair tiles are 256 x bn (bn a multiple of 32, 128 <= bn <= 256); tiles_m,
+// tiles_n count them.  The host picks bn so the tiles fill whole waves.
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                      uint16_t *__restrict__ C, int64_t ldc, int M, int N, int K, int bn, int tiles_m,
+                      int tiles_n, int c_vec, uint64_t timeout_ns) {
+    // this kernel's tile constants shadow the 1-SM ones
+    constexpr int BM = v2::BM, BN = v2::BN, BK = v2::BK, STAGES = v2::STAGES;
+    constexpr int A_STAGE_BYTES = v2::A_STAGE_BYTES, B_STAGE_BYTES = v2::B_STAGE_BYTES;
+    constexpr int B_BOX_N = v2::B_BOX_N;
+    const int B_HALF = bn >> 1;                              // B columns per CTA
+    const int B_BOXES = (B_HALF + B_BOX_N - 1) / B_BOX_N;    // TMA boxes per CTA and stage
+    const uint32_t idesc = v2::IDESC_NO_N | ((uint32_t)(bn >> 3) << 17);
+    constexpr int B_BOX_BYTES = v2::B_BOX_BYTES, B_PAD_BYTES = v2::B_PAD_BYTES;
+    constexpr int TMEM_COLS = v2::TMEM_COLS, NUM_BARS = v2::NUM_BARS, EPI_WARPS = v2::EPI_WARPS;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                ~uintptr_t(1023));
+    uint8_t *sA = smem;
+    uint8_t *sB = smem + STAGES * A_STAGE_BYTES;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + STAGES * B_STAGE_BYTES + B_PAD_BYTES);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + NUM_BARS);
+    volatile uint32_t *abort_flag = tmem_slot + 1;
+
+    const uint32_t bar0 = smem_u32(bars);
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+    auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
+    auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
+    const uint32_t mma_done_bar = bar0 + 8u * (2 * STAGES + 4);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const bool leader = rank == 0;
+    const int cluster_id = blockIdx.x >> 1, nclusters = gridDim.x >> 1;
+    const int num_tiles = tiles_m * tiles_n;
+    const int num_kb = (K + BK - 1) / BK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(full_bar(s), 1);
+            mbar_init(empty_bar(s), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(tfull_bar(a), 1);
+            mbar_init(tempty_bar(a), 2 * EPI_WARPS);  // one arrive per epilogue warp of both CTAs
+        }
+        mbar_init(mma_done_bar, 1);
+        *abort_flag = 0u;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
+    }
+    if (warp == 2) {
+        // one warp of each CTA of the pair allocates collectively
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(TMEM_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncwarp();    // .aligned cluster barrier: every warp converged
+    cluster_sync();  // barriers of both CTAs initialised, TMEM allocated
+    tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0 && lane == 0) {
+        // ------------------------------------------------------ TMA producer
+        int stage = 0;
+        uint32_t phase = 0;
+        bool ok = true;
+        for (int tile = cluster_id; ok && tile < num_tiles; tile += nclusters) {
+            int mb, nb;
+            tile_coords_pair(tile, tiles_m, tiles_n, mb, nb);
+            // what each CTA of the pair loads (boxes wholly outside the matrix are skipped)
+            int a_ok[2], nbox[2];
+            for (int r = 0; r < 2; ++r) {
+                a_ok[r] = (mb * 2 * BM + r * BM) < M;
+                const int n0r = nb * bn + r * B_HALF;
+                nbox[r] = n0r < N ? min(B_BOXES, (N - n0r + B_BOX_N - 1) / B_BOX_N) : 0;
+            }
+            const uint32_t pair_bytes = (uint32_t)((a_ok[0] + a_ok[1]) * A_STAGE_BYTES +
+                                                   (nbox[0] + nbox[1]) * B_BOX_BYTES);
+            const int m0 = mb * 2 * BM + (int)rank * BM;
+            const int n0 = nb * bn + (int)rank * B_HALF;
+            for (int kb = 0; kb < num_kb; ++kb) {
+                if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, timeout_ns, 0x31)) {
+                    ok = false;
+                    break;
+                }
+                if (leader) mbar_expect_tx(full_bar(stage), pair_bytes);
+                const uint32_t fb = mapa_shared(full_bar(stage), 0);
+                if (a_ok[rank])
+                    tma_load_2d_pair(smem_u32(sA + stage * A_STAGE_BYTES), &tmA, fb, kb * BK, m0);
+                for (int j = 0; j < nbox[rank]; ++j)
+                    tma_load_2d_pair(smem_u32(sB + stage * B_STAGE_BYTES + j * B_BOX_BYTES), &tmB, fb,
+                                     n0 + j * B_BOX_N, kb * BK);
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+        }
+        if (!ok) spin_ns(200000);  // let loads already issued land before shared memory is released
+    } else if (warp == 1 && lane == 0 && leader) {
+        // ------------------------------------------------ MMA issuer (leader)
+        int stage = 0;
+        uint32_t phase = 0;
+        bool ok = true;
+        int local = 0;
+        for (int tile = cluster_id; ok && tile < num_tiles; tile += nclusters, ++local) {
+            const int acc = local & 1;
+            const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
+            if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, timeout_ns, 0x41)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+            for (int kb = 0; kb < num_kb; ++kb) {
+                if (!mbar_wait(full_bar(stage), phase, abort_flag, timeout_ns, 0x42)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint64_t adesc = sdesc_sw128(smem_u32(sA + stage * A_STAGE_BYTES), 16, 1024);
+                const uint64_t bdesc = sdesc_sw128(smem_u32(sB + stage * B_STAGE_BYTES), B_BOX_BYTES, 1024);
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k)
+                    mma_bf16_pair(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(128 * k), idesc,
+                                  (kb | k) != 0 ? 1u : 0u);
+                mma_commit_pair(empty_bar(stage));
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (ok) mma_commit_pair(tfull_bar(acc));
+        }
+        mma_commit_local_pair(mma_done_bar);
+        mbar_wait(mma_done_bar, 0u, abort_flag, 10000000ull, 0x43, true);
+    } else if (warp >= 4) {
+        // ------------------------------------------------ epilogue (both CTAs)
+        const int ew = warp - 4;
+        const uint32_t tempty_leader0 = mapa_shared(tempty_bar(0), 0);
+        const uint32_t tempty_leader1 = mapa_shared(tempty_bar(1), 0);
+        int local = 0;
+        for (int tile = cluster_id; tile < num_tiles; tile += nclusters, ++local) {
+            int mb, nb;
+            tile_coords_pair(tile, tiles_m, tiles_n, mb, nb);
+            const int acc = local & 1;
+            const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
+            const bool waited = mbar_wait(tfull_bar(acc), acc_phase, abort_flag, timeout_ns, 0x51);
+            if (!__all_sync(0xffffffffu, waited)) break;
+            tc_fence_after();
+            const int row = mb * 2 * BM + (int)rank * BM + ew * 32 + lane;
+            const int n0 = nb * bn;
+            uint16_t *crow = C + (int64_t)row * ldc;
+#pragma unroll 1
+            for (int c = 0; c < bn / 32; ++c) {
+                const int col0 = n0 + c * 32;
+                if (col0 >= N) break;  // warp-uniform
+                uint32_t v[32];
+                tmem_ld32(tmem_base + ((uint32_t)(ew * 32) << 16) + (uint32_t)(acc * BN + c * 32), v);
+                if (row < M) {
+                    uint32_t p[16];
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        __nv_bfloat162 h =
+                            __floats2bfloat162_rn(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+                        p[i] = *reinterpret_cast<uint32_t *>(&h);
+                    }
+                    if (c_vec && col0 + 32 <= N) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(crow + col0);
+                        dst[0] = make_uint4(p[0], p[1], p[2], p[3]);
+                        dst[1] = make_uint4(p[4], p[5], p[6], p[7]);
+                        dst[2] = make_uint4(p[8], p[9], p[10], p[11]);
+                        dst[3] = make_uint4(p[12], p[13], p[14], p[15]);
+                    } else {
+                        for (int i = 0; i < 32 && col0 + i < N; ++i)
+                            crow[col0 + i] = (uint16_t)((i & 1) ? (p[i >> 1] >> 16) : (p[i >> 1] & 0xFFFFu));
+                    }
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_remote(acc ? tempty_leader1 : tempty_leader0);
+        }
+    }
+
+    // ---------------------------------------------------------------- teardown
+    tc_fence_before();
+    __syncwarp();
+    cluster_sync();  // the leader's MMAs into both CTAs' TMEM are complete
+    if (warp == 2) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem_base), "r"(TMEM_COLS)
+                     : "memory");
+    }
+}
+
 // ---------------------------------------------------------------- host side
 
 PFN_cuTensorMapEncodeTiled_v12000 get_encode_fn() {
@@ -435,6 +752,26 @@ krex_status make_map(const void *ptr, uint64_t inner, uint64_t outer, uint64_t l
     return KREX_OK;
 }
 
+// Pair-tile width for the 2-SM kernel.  Measured on GB300, a tcgen05.mma of
+// N = 224 or 192 costs about as much time as N = 256, so narrower tiles only
+// add waves: 256 everywhere.  KREX_GEMM_BN (a multiple of 32 in [128, 256])
+// overrides it for experiments and tests.
+int pick_pair_tile_n() {
+    const char *e = getenv("KREX_GEMM_BN");
+    if (e) {
+        int v = atoi(e);
+        if (v >= 128 && v <= 256 && v % 32 == 0) return v;
+    }
+    return 256;
+}
+
+// 2 = the 2-SM (cta_group::2) kernel, 1 = the 1-SM kernel; KREX_GEMM_SM picks
+// one (read on every call so a process can compare both).
+int gemm_variant() {
+    const char *e = getenv("KREX_GEMM_SM");
+    return (e && e[0] == '1') ? 1 : 2;
+}
+
 uint64_t wait_timeout_ns() {
     static uint64_t t = [] {
         const char *e = getenv("KREX_WAIT_TIMEOUT_MS");
@@ -464,19 +801,43 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
     if (st != KREX_OK) return st;
 
     static thread_local int attr_dev = -1;
+    static thread_local int max_clusters = 0;
     int dev = 0;
     KREX_CUDA_TRY(cudaGetDevice(&dev));
     if (attr_dev != dev) {
         KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05_2sm, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)v2::SMEM_BYTES));
+        // co-resident CTA pairs; a persistent grid larger than this would only queue
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(2 * (unsigned)(sm_count() / 2), 1, 1);
+        cfg.blockDim = dim3(THREADS, 1, 1);
+        cfg.dynamicSmemBytes = v2::SMEM_BYTES;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, gemm_bf16_tcgen05_2sm, &cfg) != cudaSuccess || n <= 0) {
+            cudaGetLastError();
+            n = sm_count() / 2;
+        }
+        max_clusters = n;
         attr_dev = dev;
     }
-    const int tiles_m = (int)((M + BM - 1) / BM), tiles_n = (int)((N + BN - 1) / BN);
-    const int64_t tiles = (int64_t)tiles_m * tiles_n;
-    const int grid = (int)(tiles < sm_count() ? tiles : sm_count());
     const int c_vec = ((reinterpret_cast<uintptr_t>(c) & 15u) == 0) && (ldc % 8 == 0);
-    gemm_bf16_tcgen05<<<grid, THREADS, SMEM_BYTES, s>>>(ma, mb, c, ldc, (int)M, (int)N, (int)K, tiles_m,
-                                                        tiles_n, c_vec, wait_timeout_ns());
+    if (gemm_variant() == 2) {
+        const int tiles_m = (int)((M + 2 * v2::BM - 1) / (2 * v2::BM));
+        const int bn = pick_pair_tile_n();
+        const int tiles_n = (int)((N + bn - 1) / bn);
+        const int64_t tiles = (int64_t)tiles_m * tiles_n;
+        const int clusters = (int)(tiles < max_clusters ? tiles : max_clusters);
+        gemm_bf16_tcgen05_2sm<<<2 * clusters, THREADS, v2::SMEM_BYTES, s>>>(
+            ma, mb, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, c_vec, wait_timeout_ns());
+    } else {
+        const int tiles_m = (int)((M + BM - 1) / BM), tiles_n = (int)((N + BN - 1) / BN);
+        const int64_t tiles = (int64_t)tiles_m * tiles_n;
+        const int grid = (int)(tiles < sm_count() ? tiles : sm_count());
+        gemm_bf16_tcgen05<<<grid, THREADS, SMEM_BYTES, s>>>(ma, mb, c, ldc, (int)M, (int)N, (int)K, tiles_m,
+                                                            tiles_n, c_vec, wait_timeout_ns());
+    }
     KREX_CUDA_TRY(cudaGetLastError());
     return KREX_OK;
 }

@@ -21,6 +21,13 @@ def built():
     krex.build()
 
 
+@pytest.fixture(params=["1", "2"], ids=["1sm", "2sm"])
+def variant(request, monkeypatch):
+    """Both tcgen05 kernels: 1-SM (cta_group::1) and 2-SM (cta_group::2)."""
+    monkeypatch.setenv("KREX_GEMM_SM", request.param)
+    return request.param
+
+
 def _gen(seed, M, N, K):
     a = torch.empty(M, K, dtype=torch.bfloat16, device="cuda")
     b = torch.empty(K, N, dtype=torch.bfloat16, device="cuda")
@@ -48,7 +55,7 @@ def _within_tol(got_bits, want64, K):
     return np.all(err <= tol), float(np.max(err / tol))
 
 
-def test_identity_is_exact():
+def test_identity_is_exact(variant):
     n = 256
     a, _ = _gen(1, 256, n, 384)
     eye = to_bf16_tensor(inputs.bf16_bits_from_f32(inputs.identity(384)))
@@ -56,14 +63,14 @@ def test_identity_is_exact():
     assert np.array_equal(bits16(c), bits16(a))
 
 
-def test_permutation_is_exact():
+def test_permutation_is_exact(variant):
     a, _ = _gen(2, 128, 512, 512)
     p, perm = inputs.permutation_matrix(512, 9)
     c = _candidate(a, to_bf16_tensor(inputs.bf16_bits_from_f32(p)))
     assert np.array_equal(bits16(c), bits16(a)[:, perm])
 
 
-def test_small_integers_are_exact():
+def test_small_integers_are_exact(variant):
     # integer operands in [-4, 4]: every partial sum is an integer < 2^8 * K,
     # exact in fp32; outputs below 256 are exact in bf16
     M, N, K = 256, 512, 64
@@ -80,7 +87,7 @@ def test_small_integers_are_exact():
 @pytest.mark.parametrize("M,N,K", [(128, 256, 64), (128, 256, 128), (256, 512, 256), (100, 72, 40),
                                    (129, 264, 136), (1, 8, 8), (300, 1000, 520), (1024, 2048, 512),
                                    (2048, 4096, 1024), (640, 384, 4104)])
-def test_seeded_gemm_within_tolerance(M, N, K):
+def test_seeded_gemm_within_tolerance(M, N, K, variant):
     seed = 1000 + M + N + K
     a, b = _gen(seed, M, N, K)
     c = _candidate(a, b)
@@ -89,7 +96,20 @@ def test_seeded_gemm_within_tolerance(M, N, K):
     assert ok, worst
 
 
-def test_k_zero_gives_zero_and_empty_is_noop():
+@pytest.mark.parametrize("bn", [128, 160, 192, 224, 256])
+@pytest.mark.parametrize("M,N,K", [(300, 1000, 520), (512, 1792, 256), (256, 224, 64)])
+def test_2sm_every_pair_tile_width(M, N, K, bn, monkeypatch):
+    monkeypatch.setenv("KREX_GEMM_SM", "2")
+    monkeypatch.setenv("KREX_GEMM_BN", str(bn))
+    seed = 3000 + M + N + K
+    a, b = _gen(seed, M, N, K)
+    c = _candidate(a, b)
+    want = ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N))
+    ok, worst = _within_tol(bits16(c), want, K)
+    assert ok, worst
+
+
+def test_k_zero_gives_zero_and_empty_is_noop(variant):
     a = torch.empty(64, 0, dtype=torch.bfloat16, device="cuda")
     b = torch.empty(0, 32, dtype=torch.bfloat16, device="cuda")
     c = torch.full((64, 32), 3.0, dtype=torch.bfloat16, device="cuda")
@@ -124,7 +144,7 @@ def test_reference_gemm_within_fp32_bound(M, N, K):
     assert np.all(np.abs(r.view.cpu().numpy() - want) <= (K + 2) * 2.0 ** -24 * absab + 1e-30)
 
 
-def test_gemm_4096_full_output():
+def test_gemm_4096_full_output(variant):
     M = N = K = 4096
     a, b = _gen(2, M, N, K)
     c = _candidate(a, b, guard=False)
