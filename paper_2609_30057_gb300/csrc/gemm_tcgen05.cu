@@ -388,7 +388,7 @@ namespace v2 {
 constexpr int BM = 128;                          // rows per CTA (256 per pair)
 constexpr int BN = 256;                          // widest pair tile (the kernel takes bn <= BN)
 constexpr int BK = 64;
-constexpr int STAGES = 7;
+constexpr int STAGES = 6;
 constexpr int A_STAGE_BYTES = BM * BK * 2;       // 16 KiB
 constexpr int B_HALF = BN / 2;                   // 128 columns per CTA
 constexpr int B_BOX_N = 64;
@@ -396,12 +396,15 @@ constexpr int B_BOXES = B_HALF / B_BOX_N;        // 2
 constexpr int B_BOX_BYTES = BK * B_BOX_N * 2;    // 8 KiB
 constexpr int B_STAGE_BYTES = BK * B_HALF * 2;   // 16 KiB
 constexpr int B_PAD_BYTES = 0;
+constexpr int EPI_BOX_COLS = 64;                 // TMA-store box: 64 columns x 32 rows (4 KiB)
+constexpr int EPI_BUF_BYTES = 32 * EPI_BOX_COLS * 2;
+constexpr int EPI_BYTES = 4 * 2 * EPI_BUF_BYTES; // 4 epilogue warps x 2 buffers
 constexpr int TMEM_COLS = 2 * BN;                // two 128-lane x 256-column accumulators
 constexpr int GROUP_M = 8;                       // pair-tile rows per raster group
 constexpr int EPI_WARPS = 4;
 constexpr int NUM_BARS = 2 * STAGES + 4 + 1;
 constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * (A_STAGE_BYTES + B_STAGE_BYTES) + B_PAD_BYTES +
-                              NUM_BARS * 8 + 16;
+                              EPI_BYTES + NUM_BARS * 8 + 16;
 // kind::f16, D fp32, A/B bf16, A K-major, B MN-major, M = 256 (pair); N is
 // added at run time in bits 17-22
 constexpr uint32_t IDESC_NO_N = (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | (1u << 16) |
@@ -442,6 +445,24 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
         : "memory");
 }
 
+// TMA store of one box from this CTA's shared memory (bulk-group completion).
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, uint32_t src, int32_t c0, int32_t c1) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(src), "r"(c0), "r"(c1)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit_group() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+// wait until at most N committed bulk groups still read shared memory
+template <int N>
+__device__ __forceinline__ void bulk_wait_group_read() {
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void bulk_wait_group_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 __device__ __forceinline__ void mma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                               uint32_t accumulate) {
     asm volatile(
@@ -468,11 +489,12 @@ __device__ __forceinline__ void mma_commit_local_pair(uint32_t bar) {
         : "memory");
 }
 
-__device__ __forceinline__ void tile_coords_pair(int tile, int tiles_m, int tiles_n, int &mb, int &nb) {
-    const int per_group = v2::GROUP_M * tiles_n;
+__device__ __forceinline__ void tile_coords_pair(int tile, int tiles_m, int tiles_n, int group_m, int &mb,
+                                                 int &nb) {
+    const int per_group = group_m * tiles_n;
     const int g = tile / per_group;
-    const int first_m = g * v2::GROUP_M;
-    const int gsize = min(tiles_m - first_m, v2::GROUP_M);
+    const int first_m = g * group_m;
+    const int gsize = min(tiles_m - first_m, group_m);
     const int in_g = tile - g * per_group;
     mb = first_m + in_g % gsize;
     nb = in_g / gsize;
@@ -484,12 +506,13 @@ __device__ __forceinline__ void spin_ns(uint64_t ns) {
     }
 }
 
-// Pair tiles are 256 x bn (bn a multiple of 32, 128 <= bn <= 256); tiles_m,
+// Pair tiles are 256 x bn (bn a multiple of 64, 128 <= bn <= 256); tiles_m,
 // tiles_n count them.  The host picks bn so the tiles fill whole waves.
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                      uint16_t *__restrict__ C, int64_t ldc, int M, int N, int K, int bn, int tiles_m,
-                      int tiles_n, int c_vec, uint64_t timeout_ns) {
+                      const __grid_constant__ CUtensorMap tmC, uint16_t *__restrict__ C, int64_t ldc, int M,
+                      int N, int K, int bn, int tiles_m, int tiles_n, int group_m, int c_vec, int c_tma,
+                      int stages, uint64_t timeout_ns) {
     // this kernel's tile constants shadow the 1-SM ones
     constexpr int BM = v2::BM, BN = v2::BN, BK = v2::BK, STAGES = v2::STAGES;
     constexpr int A_STAGE_BYTES = v2::A_STAGE_BYTES, B_STAGE_BYTES = v2::B_STAGE_BYTES;
@@ -504,7 +527,8 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                                                 ~uintptr_t(1023));
     uint8_t *sA = smem;
     uint8_t *sB = smem + STAGES * A_STAGE_BYTES;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + STAGES * B_STAGE_BYTES + B_PAD_BYTES);
+    uint8_t *sEpi = sB + STAGES * B_STAGE_BYTES + B_PAD_BYTES;  // 1024-aligned staging buffers
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sEpi + v2::EPI_BYTES);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + NUM_BARS);
     volatile uint32_t *abort_flag = tmem_slot + 1;
 
@@ -558,7 +582,7 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
         bool ok = true;
         for (int tile = cluster_id; ok && tile < num_tiles; tile += nclusters) {
             int mb, nb;
-            tile_coords_pair(tile, tiles_m, tiles_n, mb, nb);
+            tile_coords_pair(tile, tiles_m, tiles_n, group_m, mb, nb);
             // what each CTA of the pair loads (boxes wholly outside the matrix are skipped)
             int a_ok[2], nbox[2];
             for (int r = 0; r < 2; ++r) {
@@ -582,7 +606,7 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                 for (int j = 0; j < nbox[rank]; ++j)
                     tma_load_2d_pair(smem_u32(sB + stage * B_STAGE_BYTES + j * B_BOX_BYTES), &tmB, fb,
                                      n0 + j * B_BOX_N, kb * BK);
-                if (++stage == STAGES) {
+                if (++stage == stages) {
                     stage = 0;
                     phase ^= 1u;
                 }
@@ -617,7 +641,7 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                     mma_bf16_pair(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(128 * k), idesc,
                                   (kb | k) != 0 ? 1u : 0u);
                 mma_commit_pair(empty_bar(stage));
-                if (++stage == STAGES) {
+                if (++stage == stages) {
                     stage = 0;
                     phase ^= 1u;
                 }
@@ -631,41 +655,85 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
         const int ew = warp - 4;
         const uint32_t tempty_leader0 = mapa_shared(tempty_bar(0), 0);
         const uint32_t tempty_leader1 = mapa_shared(tempty_bar(1), 0);
+        uint32_t epi_buf = 0;  // staging buffers used so far by this warp
         int local = 0;
         for (int tile = cluster_id; tile < num_tiles; tile += nclusters, ++local) {
             int mb, nb;
-            tile_coords_pair(tile, tiles_m, tiles_n, mb, nb);
+            tile_coords_pair(tile, tiles_m, tiles_n, group_m, mb, nb);
             const int acc = local & 1;
             const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
             const bool waited = mbar_wait(tfull_bar(acc), acc_phase, abort_flag, timeout_ns, 0x51);
             if (!__all_sync(0xffffffffu, waited)) break;
             tc_fence_after();
-            const int row = mb * 2 * BM + (int)rank * BM + ew * 32 + lane;
+            const int row0 = mb * 2 * BM + (int)rank * BM + ew * 32;  // this warp's 32 rows
+            const int row = row0 + lane;
             const int n0 = nb * bn;
-            uint16_t *crow = C + (int64_t)row * ldc;
+            const uint32_t tbase = tmem_base + ((uint32_t)(ew * 32) << 16) + (uint32_t)(acc * BN);
+            if (c_tma) {
+                // 64-column chunks: TMEM -> registers -> bf16 -> 128B-swizzled staging
+                // buffer (row = lane, 16-byte chunk j at j ^ (lane % 8)) -> one TMA store of
+                // the 32 x 64 box; two buffers per warp alternate.
+                if (row0 < M) {
 #pragma unroll 1
-            for (int c = 0; c < bn / 32; ++c) {
-                const int col0 = n0 + c * 32;
-                if (col0 >= N) break;  // warp-uniform
-                uint32_t v[32];
-                tmem_ld32(tmem_base + ((uint32_t)(ew * 32) << 16) + (uint32_t)(acc * BN + c * 32), v);
-                if (row < M) {
-                    uint32_t p[16];
+                    for (int c = 0; c < bn / v2::EPI_BOX_COLS; ++c) {
+                        const int col0 = n0 + c * v2::EPI_BOX_COLS;
+                        if (col0 >= N) break;  // warp-uniform
+                        uint8_t *buf = sEpi + (ew * 2 + (epi_buf & 1)) * v2::EPI_BUF_BYTES;
+                        if (lane == 0) bulk_wait_group_read<1>();  // the store that used `buf` has read it
+                        __syncwarp();
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        __nv_bfloat162 h =
-                            __floats2bfloat162_rn(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
-                        p[i] = *reinterpret_cast<uint32_t *>(&h);
+                        for (int h = 0; h < 2; ++h) {
+                            uint32_t v[32];
+                            tmem_ld32(tbase + (uint32_t)(c * v2::EPI_BOX_COLS + h * 32), v);
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) {
+                                uint32_t w[4];
+#pragma unroll
+                                for (int i = 0; i < 4; ++i) {
+                                    __nv_bfloat162 hv = __floats2bfloat162_rn(__uint_as_float(v[8 * q + 2 * i]),
+                                                                              __uint_as_float(v[8 * q + 2 * i + 1]));
+                                    w[i] = *reinterpret_cast<uint32_t *>(&hv);
+                                }
+                                const int j = h * 4 + q;  // 16-byte chunk of the 128-byte row
+                                *reinterpret_cast<uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                                    make_uint4(w[0], w[1], w[2], w[3]);
+                            }
+                        }
+                        fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0) {
+                            tma_store_2d(&tmC, smem_u32(buf), col0, row0);
+                            bulk_commit_group();
+                        }
+                        ++epi_buf;
                     }
-                    if (c_vec && col0 + 32 <= N) {
-                        uint4 *dst = reinterpret_cast<uint4 *>(crow + col0);
-                        dst[0] = make_uint4(p[0], p[1], p[2], p[3]);
-                        dst[1] = make_uint4(p[4], p[5], p[6], p[7]);
-                        dst[2] = make_uint4(p[8], p[9], p[10], p[11]);
-                        dst[3] = make_uint4(p[12], p[13], p[14], p[15]);
-                    } else {
-                        for (int i = 0; i < 32 && col0 + i < N; ++i)
-                            crow[col0 + i] = (uint16_t)((i & 1) ? (p[i >> 1] >> 16) : (p[i >> 1] & 0xFFFFu));
+                }
+            } else {
+                uint16_t *crow = C + (int64_t)row * ldc;
+#pragma unroll 1
+                for (int c = 0; c < bn / 32; ++c) {
+                    const int col0 = n0 + c * 32;
+                    if (col0 >= N) break;  // warp-uniform
+                    uint32_t v[32];
+                    tmem_ld32(tbase + (uint32_t)(c * 32), v);
+                    if (row < M) {
+                        uint32_t p[16];
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            __nv_bfloat162 h =
+                                __floats2bfloat162_rn(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
+                            p[i] = *reinterpret_cast<uint32_t *>(&h);
+                        }
+                        if (c_vec && col0 + 32 <= N) {
+                            uint4 *dst = reinterpret_cast<uint4 *>(crow + col0);
+                            dst[0] = make_uint4(p[0], p[1], p[2], p[3]);
+                            dst[1] = make_uint4(p[4], p[5], p[6], p[7]);
+                            dst[2] = make_uint4(p[8], p[9], p[10], p[11]);
+                            dst[3] = make_uint4(p[12], p[13], p[14], p[15]);
+                        } else {
+                            for (int i = 0; i < 32 && col0 + i < N; ++i)
+                                crow[col0 + i] = (uint16_t)((i & 1) ? (p[i >> 1] >> 16) : (p[i >> 1] & 0xFFFFu));
+                        }
                     }
                 }
             }
@@ -673,6 +741,8 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
             __syncwarp();
             if (lane == 0) mbar_arrive_remote(acc ? tempty_leader1 : tempty_leader0);
         }
+        if (lane == 0) bulk_wait_group_all();  // stores complete before shared memory goes away
+        __syncwarp();
     }
 
     // ---------------------------------------------------------------- teardown
@@ -754,15 +824,36 @@ krex_status make_map(const void *ptr, uint64_t inner, uint64_t outer, uint64_t l
 
 // Pair-tile width for the 2-SM kernel.  Measured on GB300, a tcgen05.mma of
 // N = 224 or 192 costs about as much time as N = 256, so narrower tiles only
-// add waves: 256 everywhere.  KREX_GEMM_BN (a multiple of 32 in [128, 256])
-// overrides it for experiments and tests.
+// add waves: 256 everywhere.  KREX_GEMM_BN (128, 192 or 256: the epilogue
+// stores 64-column boxes) overrides it for experiments and tests.
 int pick_pair_tile_n() {
     const char *e = getenv("KREX_GEMM_BN");
     if (e) {
         int v = atoi(e);
-        if (v >= 128 && v <= 256 && v % 32 == 0) return v;
+        if (v >= 128 && v <= 256 && v % 64 == 0) return v;
     }
     return 256;
+}
+
+// Pair-tile rows per raster group of the 2-SM kernel; KREX_GEMM_GROUP overrides.
+int raster_group() {
+    const char *e = getenv("KREX_GEMM_GROUP");
+    if (e) {
+        int v = atoi(e);
+        if (v >= 1 && v <= 64) return v;
+    }
+    return v2::GROUP_M;
+}
+
+// Stages of the 2-SM kernel's shared-memory ring in use (at most v2::STAGES);
+// KREX_GEMM_STAGES overrides.
+int ring_stages() {
+    const char *e = getenv("KREX_GEMM_STAGES");
+    if (e) {
+        int v = atoi(e);
+        if (v >= 2 && v <= v2::STAGES) return v;
+    }
+    return v2::STAGES;
 }
 
 // 2 = the 2-SM (cta_group::2) kernel, 1 = the 1-SM kernel; KREX_GEMM_SM picks
@@ -824,13 +915,23 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
     }
     const int c_vec = ((reinterpret_cast<uintptr_t>(c) & 15u) == 0) && (ldc % 8 == 0);
     if (gemm_variant() == 2) {
+        // TMA-store epilogue when C rows start on 16 bytes; else direct stores
+        CUtensorMap mc;
+        int c_tma = c_vec;
+        if (c_tma) {
+            st = make_map(c, (uint64_t)N, (uint64_t)M, (uint64_t)ldc, v2::EPI_BOX_COLS, 32, &mc);
+            if (st != KREX_OK) return st;
+        } else {
+            mc = ma;  // unused
+        }
         const int tiles_m = (int)((M + 2 * v2::BM - 1) / (2 * v2::BM));
         const int bn = pick_pair_tile_n();
         const int tiles_n = (int)((N + bn - 1) / bn);
         const int64_t tiles = (int64_t)tiles_m * tiles_n;
         const int clusters = (int)(tiles < max_clusters ? tiles : max_clusters);
         gemm_bf16_tcgen05_2sm<<<2 * clusters, THREADS, v2::SMEM_BYTES, s>>>(
-            ma, mb, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, c_vec, wait_timeout_ns());
+            ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, raster_group(), c_vec, c_tma,
+            ring_stages(), wait_timeout_ns());
     } else {
         const int tiles_m = (int)((M + BM - 1) / BM), tiles_n = (int)((N + BN - 1) / BN);
         const int64_t tiles = (int64_t)tiles_m * tiles_n;
