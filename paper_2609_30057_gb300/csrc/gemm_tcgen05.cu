@@ -500,6 +500,28 @@ __device__ __forceinline__ void tile_coords_pair(int tile, int tiles_m, int tile
     nb = in_g / gsize;
 }
 
+// Work item w of the 2-SM kernel -> pair tile (mb, nb), its first column and
+// its width.  Items below full_items are whole pair tiles (width bn); the rest
+// are halves (width bn/2) of the last tiles, so a final partial wave keeps
+// twice as many SM pairs busy.
+__device__ __forceinline__ void work_item(int w, int full_items, int tiles_m, int tiles_n, int group_m, int bn,
+                                          int &mb, int &nb, int &col0, int &width) {
+    int tile = w, half = -1;
+    if (w >= full_items) {
+        const int u = w - full_items;
+        tile = full_items + (u >> 1);
+        half = u & 1;
+    }
+    tile_coords_pair(tile, tiles_m, tiles_n, group_m, mb, nb);
+    if (half < 0) {
+        col0 = nb * bn;
+        width = bn;
+    } else {
+        width = bn >> 1;
+        col0 = nb * bn + half * width;
+    }
+}
+
 __device__ __forceinline__ void spin_ns(uint64_t ns) {
     const uint64_t t0 = globaltimer();
     while (globaltimer() - t0 < ns) {
@@ -511,15 +533,12 @@ __device__ __forceinline__ void spin_ns(uint64_t ns) {
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ CUtensorMap tmC, uint16_t *__restrict__ C, int64_t ldc, int M,
-                      int N, int K, int bn, int tiles_m, int tiles_n, int group_m, int c_vec, int c_tma,
-                      int stages, uint64_t timeout_ns) {
+                      int N, int K, int bn, int tiles_m, int tiles_n, int full_items, int num_items,
+                      int group_m, int c_vec, int c_tma, int stages, uint64_t timeout_ns) {
     // this kernel's tile constants shadow the 1-SM ones
     constexpr int BM = v2::BM, BN = v2::BN, BK = v2::BK, STAGES = v2::STAGES;
     constexpr int A_STAGE_BYTES = v2::A_STAGE_BYTES, B_STAGE_BYTES = v2::B_STAGE_BYTES;
     constexpr int B_BOX_N = v2::B_BOX_N;
-    const int B_HALF = bn >> 1;                              // B columns per CTA
-    const int B_BOXES = (B_HALF + B_BOX_N - 1) / B_BOX_N;    // TMA boxes per CTA and stage
-    const uint32_t idesc = v2::IDESC_NO_N | ((uint32_t)(bn >> 3) << 17);
     constexpr int B_BOX_BYTES = v2::B_BOX_BYTES, B_PAD_BYTES = v2::B_PAD_BYTES;
     constexpr int TMEM_COLS = v2::TMEM_COLS, NUM_BARS = v2::NUM_BARS, EPI_WARPS = v2::EPI_WARPS;
     extern __shared__ uint8_t smem_raw[];
@@ -543,7 +562,6 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
     const uint32_t rank = cluster_ctarank();
     const bool leader = rank == 0;
     const int cluster_id = blockIdx.x >> 1, nclusters = gridDim.x >> 1;
-    const int num_tiles = tiles_m * tiles_n;
     const int num_kb = (K + BK - 1) / BK;
 
     if (threadIdx.x == 0) {
@@ -580,20 +598,22 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
         int stage = 0;
         uint32_t phase = 0;
         bool ok = true;
-        for (int tile = cluster_id; ok && tile < num_tiles; tile += nclusters) {
-            int mb, nb;
-            tile_coords_pair(tile, tiles_m, tiles_n, group_m, mb, nb);
+        for (int w = cluster_id; ok && w < num_items; w += nclusters) {
+            int mb, nb, col0, width;
+            work_item(w, full_items, tiles_m, tiles_n, group_m, bn, mb, nb, col0, width);
+            const int b_half = width >> 1;                            // B columns per CTA
+            const int b_boxes = (b_half + B_BOX_N - 1) / B_BOX_N;     // TMA boxes per CTA and stage
             // what each CTA of the pair loads (boxes wholly outside the matrix are skipped)
             int a_ok[2], nbox[2];
             for (int r = 0; r < 2; ++r) {
                 a_ok[r] = (mb * 2 * BM + r * BM) < M;
-                const int n0r = nb * bn + r * B_HALF;
-                nbox[r] = n0r < N ? min(B_BOXES, (N - n0r + B_BOX_N - 1) / B_BOX_N) : 0;
+                const int n0r = col0 + r * b_half;
+                nbox[r] = n0r < N ? min(b_boxes, (N - n0r + B_BOX_N - 1) / B_BOX_N) : 0;
             }
             const uint32_t pair_bytes = (uint32_t)((a_ok[0] + a_ok[1]) * A_STAGE_BYTES +
                                                    (nbox[0] + nbox[1]) * B_BOX_BYTES);
             const int m0 = mb * 2 * BM + (int)rank * BM;
-            const int n0 = nb * bn + (int)rank * B_HALF;
+            const int n0 = col0 + (int)rank * b_half;
             for (int kb = 0; kb < num_kb; ++kb) {
                 if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, timeout_ns, 0x31)) {
                     ok = false;
@@ -619,7 +639,10 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
         uint32_t phase = 0;
         bool ok = true;
         int local = 0;
-        for (int tile = cluster_id; ok && tile < num_tiles; tile += nclusters, ++local) {
+        for (int w = cluster_id; ok && w < num_items; w += nclusters, ++local) {
+            int mb, nb, col0, width;
+            work_item(w, full_items, tiles_m, tiles_n, group_m, bn, mb, nb, col0, width);
+            const uint32_t idesc = v2::IDESC_NO_N | ((uint32_t)(width >> 3) << 17);
             const int acc = local & 1;
             const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
             if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, timeout_ns, 0x41)) {
@@ -657,9 +680,9 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
         const uint32_t tempty_leader1 = mapa_shared(tempty_bar(1), 0);
         uint32_t epi_buf = 0;  // staging buffers used so far by this warp
         int local = 0;
-        for (int tile = cluster_id; tile < num_tiles; tile += nclusters, ++local) {
-            int mb, nb;
-            tile_coords_pair(tile, tiles_m, tiles_n, group_m, mb, nb);
+        for (int w = cluster_id; w < num_items; w += nclusters, ++local) {
+            int mb, nb, col0, width;
+            work_item(w, full_items, tiles_m, tiles_n, group_m, bn, mb, nb, col0, width);
             const int acc = local & 1;
             const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
             const bool waited = mbar_wait(tfull_bar(acc), acc_phase, abort_flag, timeout_ns, 0x51);
@@ -667,7 +690,7 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
             tc_fence_after();
             const int row0 = mb * 2 * BM + (int)rank * BM + ew * 32;  // this warp's 32 rows
             const int row = row0 + lane;
-            const int n0 = nb * bn;
+            const int n0 = col0;
             const uint32_t tbase = tmem_base + ((uint32_t)(ew * 32) << 16) + (uint32_t)(acc * BN);
             if (c_tma) {
                 // 64-column chunks: TMEM -> registers -> bf16 -> 128B-swizzled staging
@@ -675,7 +698,7 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                 // the 32 x 64 box; two buffers per warp alternate.
                 if (row0 < M) {
 #pragma unroll 1
-                    for (int c = 0; c < bn / v2::EPI_BOX_COLS; ++c) {
+                    for (int c = 0; c < width / v2::EPI_BOX_COLS; ++c) {
                         const int col0 = n0 + c * v2::EPI_BOX_COLS;
                         if (col0 >= N) break;  // warp-uniform
                         uint8_t *buf = sEpi + (ew * 2 + (epi_buf & 1)) * v2::EPI_BUF_BYTES;
@@ -711,7 +734,7 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
             } else {
                 uint16_t *crow = C + (int64_t)row * ldc;
 #pragma unroll 1
-                for (int c = 0; c < bn / 32; ++c) {
+                for (int c = 0; c < width / 32; ++c) {
                     const int col0 = n0 + c * 32;
                     if (col0 >= N) break;  // warp-uniform
                     uint32_t v[32];
@@ -845,6 +868,12 @@ int raster_group() {
     return v2::GROUP_M;
 }
 
+// Column-half split of a final partial wave (on unless KREX_GEMM_TAIL_SPLIT=0).
+bool tail_split_enabled() {
+    const char *e = getenv("KREX_GEMM_TAIL_SPLIT");
+    return !(e && e[0] == '0');
+}
+
 // Stages of the 2-SM kernel's shared-memory ring in use (at most v2::STAGES);
 // KREX_GEMM_STAGES overrides.
 int ring_stages() {
@@ -928,10 +957,17 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         const int bn = pick_pair_tile_n();
         const int tiles_n = (int)((N + bn - 1) / bn);
         const int64_t tiles = (int64_t)tiles_m * tiles_n;
-        const int clusters = (int)(tiles < max_clusters ? tiles : max_clusters);
+        // Split the tiles of a final partial wave into column halves when that
+        // at most fills the co-resident pairs (4096^2: 256 tiles on 76 pairs ->
+        // 228 whole tiles + 56 halves instead of a last wave of 28 tiles).
+        const int64_t rem = tiles % max_clusters;
+        const bool split = bn == 256 && rem > 0 && 2 * rem <= max_clusters && tail_split_enabled();
+        const int64_t full_items = split ? tiles - rem : tiles;
+        const int64_t items = split ? tiles + rem : tiles;
+        const int clusters = (int)(items < max_clusters ? items : max_clusters);
         gemm_bf16_tcgen05_2sm<<<2 * clusters, THREADS, v2::SMEM_BYTES, s>>>(
-            ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, raster_group(), c_vec, c_tma,
-            ring_stages(), wait_timeout_ns());
+            ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, (int)full_items, (int)items,
+            raster_group(), c_vec, c_tma, ring_stages(), wait_timeout_ns());
     } else {
         const int tiles_m = (int)((M + BM - 1) / BM), tiles_n = (int)((N + BN - 1) / BN);
         const int64_t tiles = (int64_t)tiles_m * tiles_n;

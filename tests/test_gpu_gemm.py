@@ -126,6 +126,20 @@ def test_output_row_stride(ldc_pad, variant):
     assert ok, worst
 
 
+@pytest.mark.parametrize("split", ["0", "1"])
+@pytest.mark.parametrize("M,N,K", [(1024, 2048, 512), (4096, 1024, 256), (256, 256, 4096)])
+def test_2sm_tail_split_on_and_off(M, N, K, split, monkeypatch):
+    # a final partial wave of pair tiles is split into column halves (or not)
+    monkeypatch.setenv("KREX_GEMM_SM", "2")
+    monkeypatch.setenv("KREX_GEMM_TAIL_SPLIT", split)
+    seed = 5000 + M + N + K
+    a, b = _gen(seed, M, N, K)
+    c = _candidate(a, b)
+    want = ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N))
+    ok, worst = _within_tol(bits16(c), want, K)
+    assert ok, worst
+
+
 def test_k_zero_gives_zero_and_empty_is_noop(variant):
     a = torch.empty(64, 0, dtype=torch.bfloat16, device="cuda")
     b = torch.empty(0, 32, dtype=torch.bfloat16, device="cuda")
