@@ -100,13 +100,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Wait for the phase with parity `parity` of `bar` to complete.  Returns false
-// if the CTA is aborting (unless `drain`) or `timeout_ns` passed (then it
-// starts the abort).  Drain waits ignore the abort flag: they let work that is
-// already in flight finish before shared memory or TMEM is released.
-__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
-                                       uint64_t timeout_ns, uint32_t site, bool drain = false) {
-    if (mbar_try_wait(bar, parity)) return true;
+// Non-blocking probe of a phase (no suspend): the fast path of every wait.
+__device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Slow path of mbar_wait: bounded polling with try_wait.
+__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
+                                            uint64_t timeout_ns, uint32_t site, bool drain) {
     const uint64_t t0 = globaltimer();
     for (uint32_t spin = 1;; ++spin) {
         if (mbar_try_wait(bar, parity)) return true;
@@ -119,6 +128,18 @@ __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile u
             }
         }
     }
+}
+
+// Wait for the phase with parity `parity` of `bar` to complete.  Returns false
+// if the CTA is aborting (unless `drain`) or `timeout_ns` passed (then it
+// starts the abort).  Drain waits ignore the abort flag: they let work that is
+// already in flight finish before shared memory or TMEM is released.  The
+// common case (phase already complete) costs one inlined test_wait: the MMA
+// issuer's waits sit on the tensor pipe's critical path.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
+                                          uint64_t timeout_ns, uint32_t site, bool drain = false) {
+    if (mbar_test_wait(bar, parity)) return true;
+    return mbar_wait_slow(bar, parity, abort_flag, timeout_ns, site, drain);
 }
 
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar,
