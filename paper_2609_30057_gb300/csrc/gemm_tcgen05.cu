@@ -408,24 +408,30 @@ gemm_bf16_tcgen05(const __grid_constant__ CUtensorMap tmA, const __grid_constant
 namespace v2 {
 constexpr int BM = 128;                          // rows per CTA (256 per pair)
 constexpr int BN = 256;                          // widest pair tile (the kernel takes bn <= BN)
-constexpr int BK = 64;
-constexpr int STAGES = 6;
-constexpr int A_STAGE_BYTES = BM * BK * 2;       // 16 KiB
+constexpr int BK = 64;                           // K per TMA box / swizzle atom ("sub-block")
+constexpr int A_SUB_BYTES = BM * BK * 2;         // 16 KiB
 constexpr int B_HALF = BN / 2;                   // 128 columns per CTA
 constexpr int B_BOX_N = 64;
-constexpr int B_BOXES = B_HALF / B_BOX_N;        // 2
 constexpr int B_BOX_BYTES = BK * B_BOX_N * 2;    // 8 KiB
-constexpr int B_STAGE_BYTES = BK * B_HALF * 2;   // 16 KiB
-constexpr int B_PAD_BYTES = 0;
+constexpr int B_SUB_BYTES = BK * B_HALF * 2;     // 16 KiB
+constexpr int RING_BYTES = 6 * (A_SUB_BYTES + B_SUB_BYTES);  // 192 KiB of stages per CTA
 constexpr int EPI_BOX_COLS = 64;                 // TMA-store box: 64 columns x 32 rows (4 KiB)
 constexpr int EPI_BUF_BYTES = 32 * EPI_BOX_COLS * 2;
 constexpr int EPI_BYTES = 4 * 2 * EPI_BUF_BYTES; // 4 epilogue warps x 2 buffers
 constexpr int TMEM_COLS = 2 * BN;                // two 128-lane x 256-column accumulators
 constexpr int GROUP_M = 8;                       // pair-tile rows per raster group
 constexpr int EPI_WARPS = 4;
-constexpr int NUM_BARS = 2 * STAGES + 4 + 1;
-constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * (A_STAGE_BYTES + B_STAGE_BYTES) + B_PAD_BYTES +
-                              EPI_BYTES + NUM_BARS * 8 + 16;
+// A stage holds KSUB K sub-blocks (KSUB x 64 of K): 6 stages of 32 KiB or 3
+// of 64 KiB.  Fewer, deeper stages issue 8 MMAs per barrier wait and commit
+// instead of 4 (each commit costs the tensor pipe a few percent).
+template <int KSUB>
+struct Cfg {
+    static constexpr int STAGES = 6 / KSUB;
+    static constexpr int A_STAGE_BYTES = KSUB * A_SUB_BYTES;
+    static constexpr int B_STAGE_BYTES = KSUB * B_SUB_BYTES;
+    static constexpr int NUM_BARS = 2 * STAGES + 4 + 1;
+    static constexpr size_t SMEM_BYTES = 1024 + (size_t)RING_BYTES + EPI_BYTES + NUM_BARS * 8 + 16;
+};
 // kind::f16, D fp32, A/B bf16, A K-major, B MN-major, M = 256 (pair); N is
 // added at run time in bits 17-22
 constexpr uint32_t IDESC_NO_N = (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | (1u << 16) |
@@ -551,23 +557,25 @@ __device__ __forceinline__ void spin_ns(uint64_t ns) {
 
 // Pair tiles are 256 x bn (bn a multiple of 64, 128 <= bn <= 256); tiles_m,
 // tiles_n count them.  The host picks bn so the tiles fill whole waves.
+template <int KSUB>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ CUtensorMap tmC, uint16_t *__restrict__ C, int64_t ldc, int M,
                       int N, int K, int bn, int tiles_m, int tiles_n, int full_items, int num_items,
                       int group_m, int c_vec, int c_tma, int stages, uint64_t timeout_ns) {
     // this kernel's tile constants shadow the 1-SM ones
-    constexpr int BM = v2::BM, BN = v2::BN, BK = v2::BK, STAGES = v2::STAGES;
-    constexpr int A_STAGE_BYTES = v2::A_STAGE_BYTES, B_STAGE_BYTES = v2::B_STAGE_BYTES;
-    constexpr int B_BOX_N = v2::B_BOX_N;
-    constexpr int B_BOX_BYTES = v2::B_BOX_BYTES, B_PAD_BYTES = v2::B_PAD_BYTES;
-    constexpr int TMEM_COLS = v2::TMEM_COLS, NUM_BARS = v2::NUM_BARS, EPI_WARPS = v2::EPI_WARPS;
+    using CF = v2::Cfg<KSUB>;
+    constexpr int BM = v2::BM, BN = v2::BN, BK = v2::BK, STAGES = CF::STAGES;
+    constexpr int A_STAGE_BYTES = CF::A_STAGE_BYTES, B_STAGE_BYTES = CF::B_STAGE_BYTES;
+    constexpr int A_SUB_BYTES = v2::A_SUB_BYTES, B_SUB_BYTES = v2::B_SUB_BYTES;
+    constexpr int B_BOX_N = v2::B_BOX_N, B_BOX_BYTES = v2::B_BOX_BYTES;
+    constexpr int TMEM_COLS = v2::TMEM_COLS, NUM_BARS = CF::NUM_BARS, EPI_WARPS = v2::EPI_WARPS;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                 ~uintptr_t(1023));
     uint8_t *sA = smem;
     uint8_t *sB = smem + STAGES * A_STAGE_BYTES;
-    uint8_t *sEpi = sB + STAGES * B_STAGE_BYTES + B_PAD_BYTES;  // 1024-aligned staging buffers
+    uint8_t *sEpi = sB + STAGES * B_STAGE_BYTES;  // 1024-aligned staging buffers
     uint64_t *bars = reinterpret_cast<uint64_t *>(sEpi + v2::EPI_BYTES);
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + NUM_BARS);
     volatile uint32_t *abort_flag = tmem_slot + 1;
@@ -583,7 +591,8 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
     const uint32_t rank = cluster_ctarank();
     const bool leader = rank == 0;
     const int cluster_id = blockIdx.x >> 1, nclusters = gridDim.x >> 1;
-    const int num_kb = (K + BK - 1) / BK;
+    const int num_ksub = (K + BK - 1) / BK;               // 64-deep K sub-blocks
+    const int num_kb = (num_ksub + KSUB - 1) / KSUB;      // ring stages per tile
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -631,8 +640,8 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                 const int n0r = col0 + r * b_half;
                 nbox[r] = n0r < N ? min(b_boxes, (N - n0r + B_BOX_N - 1) / B_BOX_N) : 0;
             }
-            const uint32_t pair_bytes = (uint32_t)((a_ok[0] + a_ok[1]) * A_STAGE_BYTES +
-                                                   (nbox[0] + nbox[1]) * B_BOX_BYTES);
+            const uint32_t sub_bytes = (uint32_t)((a_ok[0] + a_ok[1]) * A_SUB_BYTES +
+                                                  (nbox[0] + nbox[1]) * B_BOX_BYTES);  // per K sub-block
             const int m0 = mb * 2 * BM + (int)rank * BM;
             const int n0 = col0 + (int)rank * b_half;
             for (int kb = 0; kb < num_kb; ++kb) {
@@ -640,13 +649,17 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                     ok = false;
                     break;
                 }
-                if (leader) mbar_expect_tx(full_bar(stage), pair_bytes);
+                const int nsub = min(KSUB, num_ksub - kb * KSUB);  // sub-blocks inside K
+                if (leader) mbar_expect_tx(full_bar(stage), sub_bytes * (uint32_t)nsub);
                 const uint32_t fb = mapa_shared(full_bar(stage), 0);
-                if (a_ok[rank])
-                    tma_load_2d_pair(smem_u32(sA + stage * A_STAGE_BYTES), &tmA, fb, kb * BK, m0);
-                for (int j = 0; j < nbox[rank]; ++j)
-                    tma_load_2d_pair(smem_u32(sB + stage * B_STAGE_BYTES + j * B_BOX_BYTES), &tmB, fb,
-                                     n0 + j * B_BOX_N, kb * BK);
+                for (int h = 0; h < nsub; ++h) {
+                    const int k0 = (kb * KSUB + h) * BK;
+                    if (a_ok[rank])
+                        tma_load_2d_pair(smem_u32(sA + stage * A_STAGE_BYTES + h * A_SUB_BYTES), &tmA, fb, k0, m0);
+                    for (int j = 0; j < nbox[rank]; ++j)
+                        tma_load_2d_pair(smem_u32(sB + stage * B_STAGE_BYTES + h * B_SUB_BYTES + j * B_BOX_BYTES),
+                                         &tmB, fb, n0 + j * B_BOX_N, k0);
+                }
                 if (++stage == stages) {
                     stage = 0;
                     phase ^= 1u;
@@ -678,12 +691,20 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                     break;
                 }
                 tc_fence_after();
-                const uint64_t adesc = sdesc_sw128(smem_u32(sA + stage * A_STAGE_BYTES), 16, 1024);
-                const uint64_t bdesc = sdesc_sw128(smem_u32(sB + stage * B_STAGE_BYTES), B_BOX_BYTES, 1024);
+                const int nsub = min(KSUB, num_ksub - kb * KSUB);
 #pragma unroll
-                for (int k = 0; k < BK / 16; ++k)
-                    mma_bf16_pair(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(128 * k), idesc,
-                                  (kb | k) != 0 ? 1u : 0u);
+                for (int h = 0; h < KSUB; ++h) {
+                    if (h < nsub) {
+                        const uint64_t adesc =
+                            sdesc_sw128(smem_u32(sA + stage * A_STAGE_BYTES + h * A_SUB_BYTES), 16, 1024);
+                        const uint64_t bdesc =
+                            sdesc_sw128(smem_u32(sB + stage * B_STAGE_BYTES + h * B_SUB_BYTES), B_BOX_BYTES, 1024);
+#pragma unroll
+                        for (int k = 0; k < BK / 16; ++k)
+                            mma_bf16_pair(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(128 * k), idesc,
+                                          (kb | h | k) != 0 ? 1u : 0u);
+                    }
+                }
                 mma_commit_pair(empty_bar(stage));
                 if (++stage == stages) {
                     stage = 0;
@@ -895,15 +916,23 @@ bool tail_split_enabled() {
     return !(e && e[0] == '0');
 }
 
-// Stages of the 2-SM kernel's shared-memory ring in use (at most v2::STAGES);
+// Stages of the 2-SM kernel's shared-memory ring in use (at most `max_stages`);
 // KREX_GEMM_STAGES overrides.
-int ring_stages() {
+int ring_stages(int max_stages) {
     const char *e = getenv("KREX_GEMM_STAGES");
     if (e) {
         int v = atoi(e);
-        if (v >= 2 && v <= v2::STAGES) return v;
+        if (v >= 2 && v <= max_stages) return v;
     }
-    return v2::STAGES;
+    return max_stages;
+}
+
+// K sub-blocks (of 64) per ring stage of the 2-SM kernel: 2 = three 64 KiB
+// stages, 1 = six 32 KiB stages; KREX_GEMM_KSUB overrides.
+int stage_ksub() {
+    const char *e = getenv("KREX_GEMM_KSUB");
+    if (e && (e[0] == '1' || e[0] == '2')) return e[0] - '0';
+    return 2;
 }
 
 // 2 = the 2-SM (cta_group::2) kernel, 1 = the 1-SM kernel; KREX_GEMM_SM picks
@@ -948,15 +977,17 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
     if (attr_dev != dev) {
         KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)SMEM_BYTES));
-        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05_2sm, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)v2::SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05_2sm<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)v2::Cfg<1>::SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05_2sm<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)v2::Cfg<2>::SMEM_BYTES));
         // co-resident CTA pairs; a persistent grid larger than this would only queue
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * (unsigned)(sm_count() / 2), 1, 1);
         cfg.blockDim = dim3(THREADS, 1, 1);
-        cfg.dynamicSmemBytes = v2::SMEM_BYTES;
+        cfg.dynamicSmemBytes = v2::Cfg<2>::SMEM_BYTES;
         int n = 0;
-        if (cudaOccupancyMaxActiveClusters(&n, gemm_bf16_tcgen05_2sm, &cfg) != cudaSuccess || n <= 0) {
+        if (cudaOccupancyMaxActiveClusters(&n, gemm_bf16_tcgen05_2sm<2>, &cfg) != cudaSuccess || n <= 0) {
             cudaGetLastError();
             n = sm_count() / 2;
         }
@@ -986,9 +1017,14 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         const int64_t full_items = split ? tiles - rem : tiles;
         const int64_t items = split ? tiles + rem : tiles;
         const int clusters = (int)(items < max_clusters ? items : max_clusters);
-        gemm_bf16_tcgen05_2sm<<<2 * clusters, THREADS, v2::SMEM_BYTES, s>>>(
-            ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, (int)full_items, (int)items,
-            raster_group(), c_vec, c_tma, ring_stages(), wait_timeout_ns());
+        if (stage_ksub() == 2)
+            gemm_bf16_tcgen05_2sm<2><<<2 * clusters, THREADS, v2::Cfg<2>::SMEM_BYTES, s>>>(
+                ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, (int)full_items, (int)items,
+                raster_group(), c_vec, c_tma, ring_stages(v2::Cfg<2>::STAGES), wait_timeout_ns());
+        else
+            gemm_bf16_tcgen05_2sm<1><<<2 * clusters, THREADS, v2::Cfg<1>::SMEM_BYTES, s>>>(
+                ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, (int)full_items, (int)items,
+                raster_group(), c_vec, c_tma, ring_stages(v2::Cfg<1>::STAGES), wait_timeout_ns());
     } else {
         const int tiles_m = (int)((M + BM - 1) / BM), tiles_n = (int)((N + BN - 1) / BN);
         const int64_t tiles = (int64_t)tiles_m * tiles_n;

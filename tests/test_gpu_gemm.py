@@ -21,10 +21,12 @@ def built():
     krex.build()
 
 
-@pytest.fixture(params=["1", "2"], ids=["1sm", "2sm"])
+@pytest.fixture(params=["1", "2", "2k1"], ids=["1sm", "2sm", "2sm_ksub1"])
 def variant(request, monkeypatch):
-    """Both tcgen05 kernels: 1-SM (cta_group::1) and 2-SM (cta_group::2)."""
-    monkeypatch.setenv("KREX_GEMM_SM", request.param)
+    """The tcgen05 kernels: 1-SM (cta_group::1), 2-SM (cta_group::2) with
+    128-deep stages (default) and with 64-deep stages."""
+    monkeypatch.setenv("KREX_GEMM_SM", request.param[0])
+    monkeypatch.setenv("KREX_GEMM_KSUB", "1" if request.param == "2k1" else "2")
     return request.param
 
 
@@ -84,7 +86,7 @@ def test_small_integers_are_exact(variant):
     assert np.array_equal(gen.bf16_to_f32(bits16(c)).astype(np.float64), want)
 
 
-@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (128, 256, 128), (256, 512, 256), (100, 72, 40),
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (128, 256, 128), (256, 512, 256), (100, 72, 40), (512, 512, 192),
                                    (129, 264, 136), (1, 8, 8), (300, 1000, 520), (1024, 2048, 512),
                                    (2048, 4096, 1024), (640, 384, 4104)])
 def test_seeded_gemm_within_tolerance(M, N, K, variant):
