@@ -177,7 +177,7 @@ def kernel_table(ws, w, peaks, stream):
     rec("gemm_ref_simt", lambda: krex.krex_run_reference(0, ws.inputs, ws.ref, stream), flops=w.flops, n=3)
     rec("gemm_tcgen05", lambda: krex.krex_run_candidate(0, ws.inputs, ws.out, stream), flops=w.flops)
     scratch = ws.check_scratch
-    rec("check_bf16_f32", lambda: krex.krex_check(ws.out, ws.ref, w.atol, w.rtol, scratch, stream),
+    rec("check_bf16_f32", lambda: krex.krex_check_launch(ws.out, ws.ref, w.atol, w.rtol, scratch, stream),
         nbytes=ws.out.numel() * 6, n=10)
     # the bandwidth-bound candidate at its own workload size
     sw = WORKLOADS[SOFTMAX_WORKLOAD]
@@ -186,7 +186,7 @@ def kernel_table(ws, w, peaks, stream):
     rec("fill_normal_f32", lambda: krex.krex_gen_inputs(sw.seed, 0, 1, sw.sigma, x, stream), nbytes=x.numel() * 4,
         n=10)
     rec("softmax_f32", lambda: krex.krex_run_candidate(1, [x], y, stream), nbytes=x.numel() * 8, n=10)
-    rec("check_f32_f32", lambda: krex.krex_check(y, x, 1e-6, 0.0, scratch, stream), nbytes=x.numel() * 8, n=5)
+    rec("check_f32_f32", lambda: krex.krex_check_launch(y, x, 1e-6, 0.0, scratch, stream), nbytes=x.numel() * 8, n=5)
     del x, y
     torch.cuda.empty_cache()
     return out

@@ -172,6 +172,16 @@ krex_status krex_check(krex_buf out, krex_buf ref, float atol, float rtol, void 
                        size_t scratch_bytes, krex_check_result *host_result,
                        krex_stream_t stream);
 
+/* The check in two halves, for callers that overlap it with other work:
+ * krex_check_launch enqueues the compare-and-reduce on `stream` and leaves the
+ * 16-byte krex_check_result at the start of dev_scratch (asynchronous; same
+ * arguments and errors as krex_check); krex_check_fetch copies that result to
+ * *host_result and SYNCHRONISES `stream`.  krex_check = launch + fetch. */
+krex_status krex_check_launch(krex_buf out, krex_buf ref, float atol, float rtol, void *dev_scratch,
+                              size_t scratch_bytes, krex_stream_t stream);
+krex_status krex_check_fetch(const void *dev_scratch, krex_check_result *host_result,
+                             krex_stream_t stream);
+
 /* krex_check without caller scratch, for callers that cannot allocate device
  * memory: code whose device memory belongs to another allocator with nothing
  * to spare (a framework's caching pool, a fixed budget), and timing harnesses

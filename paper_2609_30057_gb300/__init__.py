@@ -76,6 +76,8 @@ SIGNATURES = {
     "krex_l2_bytes": (_i32, [_P(_sz)]),
     "krex_check_scratch_bytes": (_sz, []),
     "krex_check": (_i32, [krex_buf, krex_buf, _f32, _f32, _vp, _sz, _P(krex_check_result), _vp]),
+    "krex_check_launch": (_i32, [krex_buf, krex_buf, _f32, _f32, _vp, _sz, _vp]),
+    "krex_check_fetch": (_i32, [_vp, _P(krex_check_result), _vp]),
     "krex_check_noalloc": (_i32, [krex_buf, krex_buf, _f32, _f32, _P(krex_check_result), _vp]),
     "krex_region_begin": (_i32, [_P(_vp), _vp, _P(krex_region_opts)]),
     "krex_iter_begin": (_i32, [_vp]),
@@ -208,6 +210,23 @@ def krex_check(out, ref, atol: float, rtol: float, scratch, stream=None):
     bo = out if isinstance(out, krex_buf) else buf(out)
     br = ref if isinstance(ref, krex_buf) else buf(ref)
     _ok(lib().krex_check(bo, br, atol, rtol, ptr, nbytes, ctypes.byref(res), _stream(stream)), "krex_check")
+    return res.max_abs_err, int(res.n_violations)
+
+
+def krex_check_launch(out, ref, atol: float, rtol: float, scratch, stream=None):
+    """Asynchronous check kernel; the result stays in `scratch` (see krex_check_fetch)."""
+    ptr = scratch if isinstance(scratch, int) else scratch.data_ptr()
+    nbytes = krex_check_scratch_bytes() if isinstance(scratch, int) else scratch.numel() * scratch.element_size()
+    bo = out if isinstance(out, krex_buf) else buf(out)
+    br = ref if isinstance(ref, krex_buf) else buf(ref)
+    _ok(lib().krex_check_launch(bo, br, atol, rtol, ptr, nbytes, _stream(stream)), "krex_check_launch")
+
+
+def krex_check_fetch(scratch, stream=None):
+    """(max_abs_err, n_violations) left by krex_check_launch; synchronises the stream."""
+    res = krex_check_result()
+    ptr = scratch if isinstance(scratch, int) else scratch.data_ptr()
+    _ok(lib().krex_check_fetch(ptr, ctypes.byref(res), _stream(stream)), "krex_check_fetch")
     return res.max_abs_err, int(res.n_violations)
 
 

@@ -363,24 +363,36 @@ krex_status krex_l2_bytes(size_t *bytes) {
 
 size_t krex_check_scratch_bytes(void) { return check_scratch_bytes(); }
 
-krex_status krex_check(krex_buf out, krex_buf ref, float atol, float rtol, void *dev_scratch, size_t scratch_bytes,
-                       krex_check_result *host_result, krex_stream_t stream) {
+krex_status krex_check_launch(krex_buf out, krex_buf ref, float atol, float rtol, void *dev_scratch,
+                              size_t scratch_bytes, krex_stream_t stream) {
     krex_status st;
     if ((st = check_buf(out, "out")) || (st = check_buf(ref, "ref"))) return st;
     if (out.rows != ref.rows || out.cols != ref.cols) return set_error(KREX_ERR_INVALID, "out and ref shapes differ");
-    if (!host_result) return set_error(KREX_ERR_INVALID, "host_result is null");
     if (!dev_scratch || scratch_bytes < check_scratch_bytes())
         return set_error(KREX_ERR_INVALID, "check scratch needs %zu bytes", check_scratch_bytes());
     if (!aligned16(dev_scratch)) return set_error(KREX_ERR_UNSUPPORTED, "check scratch must be 16-byte aligned");
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     KREX_CUDA_TRY(launch_check(out.ptr, out.dtype, out.ld, ref.ptr, ref.dtype, ref.ld, out.rows, out.cols, atol, rtol,
-                               dev_scratch, s));
+                               dev_scratch, reinterpret_cast<cudaStream_t>(stream)));
     count_launches(1);
+    return ok();
+}
+
+krex_status krex_check_fetch(const void *dev_scratch, krex_check_result *host_result, krex_stream_t stream) {
+    if (!dev_scratch || !host_result) return set_error(KREX_ERR_INVALID, "check_fetch: null argument");
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     krex_check_result r;
     KREX_CUDA_TRY(cudaMemcpyAsync(&r, dev_scratch, sizeof(r), cudaMemcpyDeviceToHost, s));
     KREX_CUDA_TRY(cudaStreamSynchronize(s));
     *host_result = r;
     return ok();
+}
+
+krex_status krex_check(krex_buf out, krex_buf ref, float atol, float rtol, void *dev_scratch, size_t scratch_bytes,
+                       krex_check_result *host_result, krex_stream_t stream) {
+    if (!host_result) return set_error(KREX_ERR_INVALID, "host_result is null");
+    krex_status st = krex_check_launch(out, ref, atol, rtol, dev_scratch, scratch_bytes, stream);
+    if (st) return st;
+    return krex_check_fetch(dev_scratch, host_result, stream);
 }
 
 krex_status krex_region_begin(krex_region **r, krex_stream_t stream, const krex_region_opts *opts) {

@@ -75,6 +75,16 @@ def test_check_edges(scratch):
     assert krex.krex_check(e, e, 0.0, 0.0, scratch) == (0.0, 0)
 
 
+def test_check_launch_then_fetch_equals_check(scratch):
+    r32 = inputs.normal_f32(7, (300, 700))
+    o32 = inputs.perturbed(r32, 8, 0.2, 1e-3)
+    a, b = _dev(o32), _dev(r32)
+    krex.krex_check_launch(a, b, 1e-4, 1e-3, scratch)
+    got = krex.krex_check_fetch(scratch)
+    want = ref.check_f32(o32, r32, 1e-4, 1e-3)
+    assert got[1] == want[1] and ref.check_bits(got[0]) == ref.check_bits(want[0])
+
+
 def test_check_twice_is_deterministic(scratch):
     r32 = inputs.normal_f32(5, (512, 512))
     o32 = inputs.perturbed(r32, 6, 0.5, 1e-3)
