@@ -262,9 +262,8 @@ def main():
     ap.add_argument("--launches", type=int, default=3)
     args = ap.parse_args()
 
-    rank = int(os.environ.get("RANK", "0"))
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    from paper_2609_30057_gb300 import replicas
+    rank, world, local_rank = replicas.rank_world()
 
     if args.impl == "reference":
         return reference_arm(args, rank, world)
@@ -291,8 +290,7 @@ def main():
     stream = torch.cuda.current_stream()
 
     def barrier():
-        if dist is not None:
-            dist.barrier()
+        replicas.barrier(dist)
 
     for _ in range(args.warmup):
         r = ws.run()
@@ -321,13 +319,9 @@ def main():
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
     barrier()
-    launches = krex.krex_launch_count() - launches0
-    elapsed_ms = ev0.elapsed_time(ev1)
-    t_max = torch.tensor([elapsed_ms], device="cuda")
-    if dist is not None:
-        dist.all_reduce(t_max, op=dist.ReduceOp.MAX)
-    elapsed_ms = t_max.item()
-    value = world * args.steps / (elapsed_ms / 1e3)
+    launches = int(replicas.sum_over_ranks(dist, krex.krex_launch_count() - launches0, device="cuda"))
+    elapsed_ms = replicas.max_over_ranks(dist, ev0.elapsed_time(ev1), device="cuda")
+    value = replicas.aggregate_throughput(args.steps, world, elapsed_ms / 1e3)
 
     # ------------------------------------------------ e2e (host buffers)
     e2e = None
@@ -350,10 +344,8 @@ def main():
         e1.record(stream)
         torch.cuda.synchronize()
         barrier()
-        te = torch.tensor([e0.elapsed_time(e1)], device="cuda")
-        if dist is not None:
-            dist.all_reduce(te, op=dist.ReduceOp.MAX)
-        e2e = {"value": world * args.steps / (te.item() / 1e3), "unit": "cmds/s",
+        te_ms = replicas.max_over_ranks(dist, e0.elapsed_time(e1), device="cuda")
+        e2e = {"value": replicas.aggregate_throughput(args.steps, world, te_ms / 1e3), "unit": "cmds/s",
                "h2d_bytes_per_step": sum(h.numel() * h.element_size() for h in host_in),
                "d2h_bytes_per_step": host_out.numel() * host_out.element_size() + 16}
 
