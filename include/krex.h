@@ -87,7 +87,12 @@ typedef struct {
  *   pin_cpu          nonzero: pin the calling thread to the core it runs on
  *                    for the region's lifetime, restored at region end
  *   flush_scratch    device buffer of >= flush_bytes (needed if flush_on_entry)
+ *   gate, tenant     optional (gate may be NULL): region entry first enters the
+ *                    gate as holder `tenant` (sibling tenants drained and
+ *                    blocked, see krex_gate_enter); region end/abort exits it
  */
+typedef struct krex_gate krex_gate; /* opaque; see the gate section below */
+
 typedef struct {
     int32_t max_iters;
     int32_t flush_on_entry;
@@ -96,6 +101,9 @@ typedef struct {
     int64_t drain_timeout_us;
     void *flush_scratch;
     size_t flush_bytes;
+    krex_gate *gate;           /* optional: enter this gate as `tenant` before the drain */
+    int32_t tenant;
+    int32_t reserved2;
 } krex_region_opts;
 
 #define KREX_MAX_ITERS 100000
@@ -231,6 +239,51 @@ krex_status krex_region_end(krex_region *r, float *durations_ms, int32_t cap, in
 
 /* Release a region without reading its timings (error paths). */
 krex_status krex_region_abort(krex_region *r);
+
+/* -------------------------------------------------- in-region gate ----- */
+
+/* The in-process form of the paper's in-region GPU exclusivity (Section 4.2,
+ * "GPU exclusivity", steps 1-3 and 8).  Tenants are submitting threads, each
+ * with the stream its GPU work goes to.  Host-side only: a tenant brackets
+ * every submission with submit_begin/submit_end; a holder's gate_enter blocks
+ * new sibling submissions and drains the outstanding ones before returning.
+ * Timeouts are in microseconds (<= 0: 10 s).  Thread-safe. */
+
+/* Create / destroy a gate with up to max_tenants tenants (1..4096).  Destroy
+ * fails with STATE while a holder is inside. */
+krex_status krex_gate_create(krex_gate **gate, int32_t max_tenants);
+krex_status krex_gate_destroy(krex_gate *gate);
+
+/* Register a tenant whose work goes to `stream` (NULL: nothing to synchronise
+ * in the drain).  Registration is serialised with gate closure: while a holder
+ * is inside, it waits for the gate to reopen (TIMEOUT after timeout_us). */
+krex_status krex_gate_register(krex_gate *gate, krex_stream_t stream, int64_t timeout_us,
+                               int32_t *tenant);
+/* STATE if the tenant holds the gate or has a submission open. */
+krex_status krex_gate_unregister(krex_gate *gate, int32_t tenant);
+
+/* Counter-and-gate (Section 4.2): increment the tenant's in-flight counter,
+ * then check the gate; if another tenant holds it, retract the increment and
+ * park until it reopens (TIMEOUT after timeout_us).  On OK the caller issues
+ * its GPU work, then calls submit_end, also when the work failed. */
+krex_status krex_gate_submit_begin(krex_gate *gate, int32_t tenant, int64_t timeout_us);
+krex_status krex_gate_submit_end(krex_gate *gate, int32_t tenant);
+
+/* Enter as holder (steps 1-3): take the region lock, claim the gate with a new
+ * epoch (*epoch), then for every sibling wait for its in-flight counter to
+ * reach zero, synchronise its stream and acknowledge the epoch.  Returns only
+ * when every sibling acknowledged this epoch with a zero counter.  On TIMEOUT
+ * or a CUDA error the gate is reopened and the lock released: a failing entry
+ * never starts measurement.  STATE if the caller already holds the gate. */
+krex_status krex_gate_enter(krex_gate *gate, int32_t holder, int64_t timeout_us, uint64_t *epoch);
+
+/* Exit (step 8), bound to the holder and the epoch of its entry: wait for the
+ * holder's own submissions to finish host-side, reopen the gate (parked
+ * tenants resume), release the region lock.  STATE for a stale holder/epoch. */
+krex_status krex_gate_exit(krex_gate *gate, int32_t holder, uint64_t epoch);
+
+/* Current holder (-1 = open), last epoch, and number of parked submitters. */
+krex_status krex_gate_state(krex_gate *gate, int32_t *holder, uint64_t *epoch, int32_t *parked);
 
 /* ------------------------------------------------ timing loop (native) --- */
 

@@ -39,7 +39,8 @@ class krex_region_opts(ctypes.Structure):
     _fields_ = [("max_iters", ctypes.c_int32), ("flush_on_entry", ctypes.c_int32),
                 ("pin_cpu", ctypes.c_int32), ("reserved", ctypes.c_int32),
                 ("drain_timeout_us", ctypes.c_int64), ("flush_scratch", ctypes.c_void_p),
-                ("flush_bytes", ctypes.c_size_t)]
+                ("flush_bytes", ctypes.c_size_t), ("gate", ctypes.c_void_p), ("tenant", ctypes.c_int32),
+                ("reserved2", ctypes.c_int32)]
 
 
 class krex_command(ctypes.Structure):
@@ -95,6 +96,15 @@ SIGNATURES = {
     "krex_last_error_string": (ctypes.c_char_p, []),
     "krex_version": (_i32, []),
     "krex_debug_hold_stream": (_i32, [_vp, _P(_i32), _i32]),
+    "krex_gate_create": (_i32, [_P(_vp), _i32]),
+    "krex_gate_destroy": (_i32, [_vp]),
+    "krex_gate_register": (_i32, [_vp, _vp, _i64, _P(_i32)]),
+    "krex_gate_unregister": (_i32, [_vp, _i32]),
+    "krex_gate_submit_begin": (_i32, [_vp, _i32, _i64]),
+    "krex_gate_submit_end": (_i32, [_vp, _i32]),
+    "krex_gate_enter": (_i32, [_vp, _i32, _i64, _P(_u64)]),
+    "krex_gate_exit": (_i32, [_vp, _i32, _u64]),
+    "krex_gate_state": (_i32, [_vp, _P(_i32), _P(_u64), _P(_i32)]),
 }
 
 _lib = None
@@ -241,11 +251,12 @@ def krex_check_noalloc(out, ref, atol: float, rtol: float, stream=None):
 
 
 def krex_region_begin(stream=None, max_iters: int = 100, flush_scratch=None, flush_bytes: int = 0,
-                      flush_on_entry: bool = True, pin_cpu: bool = False, drain_timeout_us: int = 0) -> int:
+                      flush_on_entry: bool = True, pin_cpu: bool = False, drain_timeout_us: int = 0,
+                      gate=None, tenant: int = 0) -> int:
     o = krex_region_opts(max_iters, int(bool(flush_on_entry and flush_bytes)), int(pin_cpu), 0, drain_timeout_us,
                          None if flush_scratch is None else
                          (flush_scratch if isinstance(flush_scratch, int) else flush_scratch.data_ptr()),
-                         flush_bytes)
+                         flush_bytes, None if gate is None else gate.handle, tenant, 0)
     h = _vp()
     _ok(lib().krex_region_begin(ctypes.byref(h), _stream(stream), ctypes.byref(o)), "krex_region_begin")
     return h.value
@@ -290,11 +301,13 @@ class Region:
 
 @contextlib.contextmanager
 def region(stream=None, max_iters: int = 100, flush_scratch=None, flush_bytes: int = 0, pin_cpu: bool = False,
-           drain_timeout_us: int = 0):
-    """Critical region (the paper's ``region.critical()``, Section 4.1): drains the
-    stream, flushes L2, optionally pins the thread; ``r.iteration()`` brackets a
-    timed iteration; after the block ``r.durations_ms``, ``r.p50_ms``, ``r.p95_ms``."""
-    h = krex_region_begin(stream, max_iters, flush_scratch, flush_bytes, True, pin_cpu, drain_timeout_us)
+           drain_timeout_us: int = 0, gate=None, tenant: int = 0):
+    """Critical region (the paper's ``region.critical()``, Section 4.1): enters the
+    gate if one is given (sibling tenants blocked and drained), drains the stream,
+    flushes L2, optionally pins the thread; ``r.iteration()`` brackets a timed
+    iteration; after the block ``r.durations_ms``, ``r.p50_ms``, ``r.p95_ms``."""
+    h = krex_region_begin(stream, max_iters, flush_scratch, flush_bytes, True, pin_cpu, drain_timeout_us, gate,
+                          tenant)
     r = Region(h)
     try:
         yield r
@@ -305,12 +318,13 @@ def region(stream=None, max_iters: int = 100, flush_scratch=None, flush_bytes: i
 
 
 def krex_bench_candidate(op: int, inputs, out, warmup: int, iters: int, flush_scratch=None, flush_bytes: int = 0,
-                         pin_cpu: bool = False, drain_timeout_us: int = 0, stream=None):
-    """Native timing loop; returns (durations_ms, p50_ms, p95_ms)."""
+                         pin_cpu: bool = False, drain_timeout_us: int = 0, stream=None, gate=None, tenant: int = 0):
+    """Native timing loop (optionally gated); returns (durations_ms, p50_ms, p95_ms)."""
     arr, n = _bufs(inputs)
     bo = out if isinstance(out, krex_buf) else buf(out)
     fs = None if flush_scratch is None else (flush_scratch if isinstance(flush_scratch, int) else flush_scratch.data_ptr())
-    o = krex_region_opts(max(iters, 1), int(flush_bytes > 0), int(pin_cpu), 0, drain_timeout_us, fs, flush_bytes)
+    o = krex_region_opts(max(iters, 1), int(flush_bytes > 0), int(pin_cpu), 0, drain_timeout_us, fs, flush_bytes,
+                         None if gate is None else gate.handle, tenant, 0)
     d = (_f32 * max(iters, 1))()
     p50, p95 = _f64(math.nan), _f64(math.nan)
     _ok(lib().krex_bench_candidate(op, arr, n, bo, ctypes.byref(o), warmup, iters, d, ctypes.byref(p50),
@@ -352,3 +366,57 @@ def krex_launch_count() -> int:
 def krex_debug_hold_stream(gate, hold_ms: int, stream=None):
     """Test hook: block `stream` on the host until gate.value != 0 (or hold_ms)."""
     _ok(lib().krex_debug_hold_stream(_stream(stream), ctypes.byref(gate), hold_ms), "krex_debug_hold_stream")
+
+
+# ------------------------------------------------------------------ gate --
+
+class Gate:
+    """The in-region gate (paper Section 4.2, in-process form): tenants bracket
+    submissions with ``submission(t)``; a holder's ``enter``/``exit`` (or a
+    ``region(..., gate=g, tenant=t)``) blocks and drains sibling tenants."""
+
+    def __init__(self, max_tenants: int = 64):
+        h = _vp()
+        _ok(lib().krex_gate_create(ctypes.byref(h), max_tenants), "krex_gate_create")
+        self.handle = h.value
+
+    def close(self):
+        if self.handle:
+            _ok(lib().krex_gate_destroy(self.handle), "krex_gate_destroy")
+            self.handle = None
+
+    def register(self, stream=None, timeout_us: int = 0) -> int:
+        t = _i32(-1)
+        s = None if stream is None else _stream(stream)
+        _ok(lib().krex_gate_register(self.handle, s, timeout_us, ctypes.byref(t)), "krex_gate_register")
+        return t.value
+
+    def unregister(self, tenant: int):
+        _ok(lib().krex_gate_unregister(self.handle, tenant), "krex_gate_unregister")
+
+    def submit_begin(self, tenant: int, timeout_us: int = 0):
+        _ok(lib().krex_gate_submit_begin(self.handle, tenant, timeout_us), "krex_gate_submit_begin")
+
+    def submit_end(self, tenant: int):
+        _ok(lib().krex_gate_submit_end(self.handle, tenant), "krex_gate_submit_end")
+
+    @contextlib.contextmanager
+    def submission(self, tenant: int, timeout_us: int = 0):
+        self.submit_begin(tenant, timeout_us)
+        try:
+            yield
+        finally:
+            self.submit_end(tenant)
+
+    def enter(self, holder: int, timeout_us: int = 0) -> int:
+        e = _u64(0)
+        _ok(lib().krex_gate_enter(self.handle, holder, timeout_us, ctypes.byref(e)), "krex_gate_enter")
+        return e.value
+
+    def exit(self, holder: int, epoch: int):
+        _ok(lib().krex_gate_exit(self.handle, holder, epoch), "krex_gate_exit")
+
+    def state(self):
+        h, e, p = _i32(0), _u64(0), _i32(0)
+        _ok(lib().krex_gate_state(self.handle, ctypes.byref(h), ctypes.byref(e), ctypes.byref(p)), "krex_gate_state")
+        return h.value, e.value, p.value

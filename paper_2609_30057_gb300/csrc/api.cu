@@ -269,6 +269,9 @@ krex_status drain_stream(cudaStream_t s, int64_t timeout_us) {
 
 struct krex_region {
     cudaStream_t stream;
+    krex_gate *gate;
+    int32_t tenant;
+    uint64_t epoch;
     int device;
     int32_t max_iters;
     int32_t n_begun;
@@ -281,6 +284,7 @@ struct krex_region {
 using namespace krex;
 
 static void region_release(krex_region *r) {
+    if (r->gate) krex_gate_exit(r->gate, r->tenant, r->epoch);  // reopen the gate (step 8)
     if (r->pinned) pthread_setaffinity_np(pthread_self(), sizeof(cpu_set_t), &r->old_mask);
     event_pool().give(r->device, r->ev);
     {
@@ -411,14 +415,27 @@ krex_status krex_region_begin(krex_region **r, krex_stream_t stream, const krex_
         std::lock_guard<std::mutex> lk(g_open_mu);
         open_streams().erase(s);
     };
+    // 0) optional gate: block and drain sibling tenants (Section 4.2 steps 1-3)
+    uint64_t epoch = 0;
+    if (opts->gate) {
+        krex_status gst = krex_gate_enter(opts->gate, opts->tenant, opts->drain_timeout_us, &epoch);
+        if (gst) {
+            unmark();
+            return gst;
+        }
+    }
     // 1) drain what is already queued: a failing entry starts nothing
     krex_status st = drain_stream(s, opts->drain_timeout_us);
     if (st) {
+        if (opts->gate) krex_gate_exit(opts->gate, opts->tenant, epoch);
         unmark();
         return st;
     }
     krex_region *reg = new krex_region();
     reg->stream = s;
+    reg->gate = opts->gate;
+    reg->tenant = opts->tenant;
+    reg->epoch = epoch;
     reg->max_iters = opts->max_iters;
     reg->n_begun = reg->n_ended = 0;
     reg->pinned = false;

@@ -46,7 +46,7 @@ def test_binding_covers_every_declared_symbol():
 def test_struct_layouts_match_the_header():
     assert ctypes.sizeof(krex.krex_buf) == 40
     assert ctypes.sizeof(krex.krex_check_result) == 16
-    assert ctypes.sizeof(krex.krex_region_opts) == 40
+    assert ctypes.sizeof(krex.krex_region_opts) == 56
     assert ctypes.sizeof(krex.krex_command) == 80
     assert ctypes.sizeof(krex.krex_command_result) == 88
 
@@ -111,11 +111,11 @@ def test_invalid_arguments_fail_before_any_cuda_call(lib):
         == krex.KREX_ERR_INVALID
     # region misuse
     h = ctypes.c_void_p()
-    o = krex.krex_region_opts(0, 0, 0, 0, 0, None, 0)
+    o = krex.krex_region_opts(0, 0, 0, 0, 0, None, 0, None, 0, 0)
     assert lib.krex_region_begin(ctypes.byref(h), None, ctypes.byref(o)) == krex.KREX_ERR_INVALID
-    o = krex.krex_region_opts(krex.KREX_MAX_ITERS + 1, 0, 0, 0, 0, None, 0)
+    o = krex.krex_region_opts(krex.KREX_MAX_ITERS + 1, 0, 0, 0, 0, None, 0, None, 0, 0)
     assert lib.krex_region_begin(ctypes.byref(h), None, ctypes.byref(o)) == krex.KREX_ERR_INVALID
-    o = krex.krex_region_opts(10, 1, 0, 0, 0, None, 1 << 20)
+    o = krex.krex_region_opts(10, 1, 0, 0, 0, None, 1 << 20, None, 0, 0)
     assert lib.krex_region_begin(ctypes.byref(h), None, ctypes.byref(o)) == krex.KREX_ERR_INVALID
     assert lib.krex_iter_begin(None) == krex.KREX_ERR_INVALID
     assert lib.krex_iter_end(None) == krex.KREX_ERR_INVALID
