@@ -320,6 +320,10 @@ def main():
         wall = time.perf_counter() - t0
     barrier()
     launches = int(replicas.sum_over_ranks(dist, krex.krex_launch_count() - launches0, device="cuda"))
+    # a kernel whose bounded wait ran out returned early: no valid number
+    status = krex.krex_device_status()
+    if status:
+        raise SystemExit(f"a kernel reported device status {status:#x} during the timed region")
     elapsed_ms = replicas.max_over_ranks(dist, ev0.elapsed_time(ev1), device="cuda")
     value = replicas.aggregate_throughput(args.steps, world, elapsed_ms / 1e3)
 

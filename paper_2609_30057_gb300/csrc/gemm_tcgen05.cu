@@ -964,6 +964,18 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
     }
     if (M > (1ll << 31) - BM || N > (1ll << 31) - BN || K > (1ll << 31) - BK)
         return set_error(KREX_ERR_UNSUPPORTED, "GEMM dimension too large for the tcgen05 path");
+    // Tensor-map encoding is a driver call and needs a current context on this
+    // thread; a thread whose first CUDA work is this GEMM has none yet, so bind
+    // the runtime's current device (its primary context) once per thread.
+    static thread_local int bound_dev = -1;
+    {
+        int d = 0;
+        KREX_CUDA_TRY(cudaGetDevice(&d));
+        if (bound_dev != d) {
+            KREX_CUDA_TRY(cudaSetDevice(d));
+            bound_dev = d;
+        }
+    }
     CUtensorMap ma, mb;
     krex_status st = make_map(a, (uint64_t)K, (uint64_t)M, (uint64_t)lda, BK, BM, &ma);
     if (st != KREX_OK) return st;
