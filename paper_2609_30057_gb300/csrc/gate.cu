@@ -13,8 +13,10 @@
 //  - Entry: lock, claim the gate (holder, epoch), then for each sibling wait
 //    for its counter to reach zero, synchronise its stream and record the
 //    epoch as acknowledged.  The holder proceeds only when every sibling has
-//    acknowledged this epoch with a zero counter; a previous epoch's
-//    acknowledgement never counts.  A drain that runs out of time releases the
+//    acknowledged this epoch; a previous epoch's acknowledgement never counts.
+//    (After the acknowledgement a sibling's counter may still rise for a
+//    moment: the increment of a submission that then sees the closed gate and
+//    retracts.)  A drain that runs out of time releases the
 //    gate and the lock and fails the entry: measurement never starts.
 //  - Registration is serialised with gate closure: a tenant registering while
 //    the gate is closed waits for it to reopen.
@@ -217,11 +219,15 @@ krex_status krex_gate_enter(krex_gate *g, int32_t holder, int64_t timeout_us, ui
         }
         x.acked_epoch.store(e, std::memory_order_seq_cst);
     }
-    // the holder proceeds only on acknowledgements of this epoch with zero counters
+    // The holder proceeds only on acknowledgements of this epoch.  Each was
+    // recorded after that sibling's counter was seen at zero with the gate
+    // already closed; a non-zero counter seen now can only be the transient
+    // increment of a submission that will see the closed gate and retract, so
+    // the counters are not read again here.
     for (int32_t t = 0; t < g->max_tenants; ++t) {
         Tenant &x = g->tenants[t];
         if (!x.registered || t == holder) continue;
-        if (x.acked_epoch.load() != e || x.inflight.load() != 0) {
+        if (x.acked_epoch.load() != e) {
             g->holder.store(-1, std::memory_order_seq_cst);
             wake_parked(g);
             g->region_locked.store(false, std::memory_order_seq_cst);
