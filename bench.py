@@ -175,7 +175,7 @@ def kernel_table(ws, w, peaks, stream):
     rec("fill_uniform_bf16", lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, A, stream), nbytes=A.numel() * 2)
     rec("flush_l2", flush, nbytes=flush_t.numel(), do_flush=False)
     rec("gemm_ref_simt", lambda: krex.krex_run_reference(0, ws.inputs, ws.ref, stream), flops=w.flops, n=3)
-    rec("gemm_tcgen05", lambda: krex.krex_run_candidate(0, ws.inputs, ws.out, stream), flops=w.flops)
+    rec("gemm_tcgen05", lambda: krex.krex_run_candidate_ws(0, ws.inputs, ws.out, ws.gemm_ws, stream), flops=w.flops)
     scratch = ws.check_scratch
     rec("check_bf16_f32", lambda: krex.krex_check_launch(ws.out, ws.ref, w.atol, w.rtol, scratch, stream),
         nbytes=ws.out.numel() * 6, n=10)
@@ -426,7 +426,7 @@ def kernel_only(args):
         krex.krex_run_reference(w.op, ws.inputs, ws.ref, stream)
         krex.krex_run_candidate(w.op, ws.inputs, ws.out, stream)
     fn = {
-        "gemm": lambda: krex.krex_run_candidate(0, ws.inputs, ws.out, stream),
+        "gemm": lambda: krex.krex_run_candidate_ws(0, ws.inputs, ws.out, ws.gemm_ws, stream),
         "gemm_ref": lambda: krex.krex_run_reference(0, ws.inputs, ws.ref, stream),
         "fill_uniform": lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, ws.inputs[0], stream),
         "fill_normal": lambda: krex.krex_gen_inputs(w.seed, 0, 1, w.sigma, ws.inputs[0], stream),

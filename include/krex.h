@@ -142,6 +142,20 @@ krex_status krex_gen_inputs(uint64_t seed, uint32_t tensor_id, int32_t dist, flo
 krex_status krex_run_candidate(int32_t op, const krex_buf *in, int32_t n_in, krex_buf out,
                                krex_stream_t stream);
 
+/* Bytes of the optional GEMM workspace (16 MiB + 4 KiB). */
+size_t krex_gemm_workspace_bytes(void);
+
+/* krex_run_candidate with an optional GEMM workspace (device memory of >=
+ * krex_gemm_workspace_bytes(), 16-byte aligned, zero-filled before its first
+ * use; may be NULL).  With it, the tiles of the GEMM's final partial wave are
+ * split into two K halves whose fp32 partial sums meet in the workspace (the
+ * kernel leaves it ready for the next call); without it they are split into
+ * column halves.  One workspace per GEMM in flight: calls that overlap on the
+ * GPU must not share it.  After a KREX_ERR_DEVICE status, zero it again.
+ * Other ops ignore the workspace.  Asynchronous. */
+krex_status krex_run_candidate_ws(int32_t op, const krex_buf *in, int32_t n_in, krex_buf out,
+                                  void *workspace, size_t workspace_bytes, krex_stream_t stream);
+
 /* The reference the check compares against (Section 2.1: the command checks
  * its result against a reference implementation).  CUDA cores only, fp32
  * accumulation and fp32 output: GEMM ref = fp32 M x N; softmax ref = fp32,
@@ -272,7 +286,8 @@ krex_status krex_gate_submit_end(krex_gate *gate, int32_t tenant);
 /* Enter as holder (steps 1-3): take the region lock, claim the gate with a new
  * epoch (*epoch), then for every sibling wait for its in-flight counter to
  * reach zero, synchronise its stream and acknowledge the epoch.  Returns only
- * when every sibling acknowledged this epoch with a zero counter.  On TIMEOUT
+ * when every sibling acknowledged this epoch (its counter seen at zero with
+ * the gate closed).  On TIMEOUT
  * or a CUDA error the gate is reopened and the lock released: a failing entry
  * never starts measurement.  STATE if the caller already holds the gate. */
 krex_status krex_gate_enter(krex_gate *gate, int32_t holder, int64_t timeout_us, uint64_t *epoch);
@@ -292,11 +307,12 @@ krex_status krex_gate_state(krex_gate *gate, int32_t *holder, uint64_t *epoch, i
  * iterations, each = L2 flush (opts->flush_bytes of opts->flush_scratch,
  * outside the event pair) then the candidate between a start and an end event
  * (Section 2.1; warm-up belongs inside the region, Section 4.1), then region
- * end.  durations_ms needs room for `iters` values. */
+ * end.  durations_ms needs room for `iters` values.  workspace / workspace_bytes:
+ * the optional GEMM workspace of krex_run_candidate_ws (may be NULL). */
 krex_status krex_bench_candidate(int32_t op, const krex_buf *in, int32_t n_in, krex_buf out,
                                  const krex_region_opts *opts, int32_t warmup, int32_t iters,
                                  float *durations_ms, double *p50_ms, double *p95_ms,
-                                 krex_stream_t stream);
+                                 void *workspace, size_t workspace_bytes, krex_stream_t stream);
 
 /* ------------------------------------------------------- one command ----- */
 
@@ -326,6 +342,8 @@ typedef struct {
     void *flush_scratch;
     void *check_scratch;
     size_t check_scratch_bytes;
+    void *gemm_workspace;      /* optional (may be NULL), see krex_run_candidate_ws */
+    size_t gemm_workspace_bytes;
 } krex_command_bufs;
 
 typedef struct {
@@ -357,6 +375,17 @@ krex_status krex_percentile(const float *x, int32_t n, double q, double *out);
 /* Read and clear the device-side status word written by kernels whose
  * bounded waits ran out (0 = none).  Synchronises the device. */
 krex_status krex_device_status(uint32_t *code);
+
+/* Where the first time-out since the status word was last cleared happened
+ * (all zero if none), as 8 words: 0 status code | wait parity << 32;
+ * 1 CTA index | grid size << 32; 2 SM id | rank in the cluster << 32;
+ * 3 nanoseconds waited; then that CTA's progress: 4 producer work item |
+ * K stage << 32; 5 MMA issuer work item | K stage << 32 (0xFFFFFFFF: waiting
+ * for an accumulator); 6 first epilogue warp's work item | step << 32
+ * (1 waiting for an accumulator, 2 draining it, 3 released); 7 M | N << 21 |
+ * K << 42 (each mod 2^21).  Read it before krex_device_status, which clears
+ * both.  Synchronises the device. */
+krex_status krex_device_status_detail(uint64_t *words);
 
 /* Kernels this library has launched in this process, over all entry points
  * (host-side counter; the bench reports its change over the timed region). */

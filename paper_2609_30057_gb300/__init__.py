@@ -54,7 +54,8 @@ class krex_command(ctypes.Structure):
 class krex_command_bufs(ctypes.Structure):
     _fields_ = [("in_", krex_buf * 2), ("out", krex_buf), ("ref", krex_buf),
                 ("flush_scratch", ctypes.c_void_p), ("check_scratch", ctypes.c_void_p),
-                ("check_scratch_bytes", ctypes.c_size_t)]
+                ("check_scratch_bytes", ctypes.c_size_t), ("gemm_workspace", ctypes.c_void_p),
+                ("gemm_workspace_bytes", ctypes.c_size_t)]
 
 
 class krex_command_result(ctypes.Structure):
@@ -72,6 +73,8 @@ _vp, _i32, _u32, _i64, _u64, _f32, _f64, _sz = (ctypes.c_void_p, ctypes.c_int32,
 SIGNATURES = {
     "krex_gen_inputs": (_i32, [_u64, _u32, _i32, _f32, krex_buf, _vp]),
     "krex_run_candidate": (_i32, [_i32, _P(krex_buf), _i32, krex_buf, _vp]),
+    "krex_gemm_workspace_bytes": (_sz, []),
+    "krex_run_candidate_ws": (_i32, [_i32, _P(krex_buf), _i32, krex_buf, _vp, _sz, _vp]),
     "krex_run_reference": (_i32, [_i32, _P(krex_buf), _i32, krex_buf, _vp]),
     "krex_flush_l2": (_i32, [_vp, _sz, _vp]),
     "krex_l2_bytes": (_i32, [_P(_sz)]),
@@ -86,11 +89,12 @@ SIGNATURES = {
     "krex_region_end": (_i32, [_vp, _P(_f32), _i32, _P(_i32), _P(_f64), _P(_f64)]),
     "krex_region_abort": (_i32, [_vp]),
     "krex_bench_candidate": (_i32, [_i32, _P(krex_buf), _i32, krex_buf, _P(krex_region_opts), _i32, _i32,
-                                    _P(_f32), _P(_f64), _P(_f64), _vp]),
+                                    _P(_f32), _P(_f64), _P(_f64), _vp, _sz, _vp]),
     "krex_command_run": (_i32, [_P(krex_command), _P(krex_command_bufs), _P(_vp), _vp, _P(_f32),
                                 _P(krex_command_result), _vp]),
     "krex_percentile": (_i32, [_P(_f32), _i32, _f64, _P(_f64)]),
     "krex_device_status": (_i32, [_P(_u32)]),
+    "krex_device_status_detail": (_i32, [_P(_u64)]),
     "krex_launch_count": (_u64, []),
     "krex_status_string": (ctypes.c_char_p, [_i32]),
     "krex_last_error_string": (ctypes.c_char_p, []),
@@ -187,6 +191,31 @@ def krex_run_candidate(op: int, inputs, out, stream=None):
     arr, n = _bufs(inputs)
     b = out if isinstance(out, krex_buf) else buf(out)
     _ok(lib().krex_run_candidate(op, arr, n, b, _stream(stream)), "krex_run_candidate")
+
+
+def krex_gemm_workspace_bytes() -> int:
+    return lib().krex_gemm_workspace_bytes()
+
+
+def gemm_workspace(device="cuda"):
+    """A zero-filled GEMM workspace (a uint8 tensor) for krex_run_candidate_ws."""
+    import torch
+    return torch.zeros(krex_gemm_workspace_bytes(), dtype=torch.uint8, device=device)
+
+
+def _ptr_bytes(workspace):
+    if workspace is None:
+        return None, 0
+    if isinstance(workspace, int):
+        return workspace, krex_gemm_workspace_bytes()
+    return workspace.data_ptr(), workspace.numel() * workspace.element_size()
+
+
+def krex_run_candidate_ws(op: int, inputs, out, workspace, stream=None):
+    arr, n = _bufs(inputs)
+    b = out if isinstance(out, krex_buf) else buf(out)
+    p, nb = _ptr_bytes(workspace)
+    _ok(lib().krex_run_candidate_ws(op, arr, n, b, p, nb, _stream(stream)), "krex_run_candidate_ws")
 
 
 def krex_run_reference(op: int, inputs, ref, stream=None):
@@ -318,7 +347,8 @@ def region(stream=None, max_iters: int = 100, flush_scratch=None, flush_bytes: i
 
 
 def krex_bench_candidate(op: int, inputs, out, warmup: int, iters: int, flush_scratch=None, flush_bytes: int = 0,
-                         pin_cpu: bool = False, drain_timeout_us: int = 0, stream=None, gate=None, tenant: int = 0):
+                         pin_cpu: bool = False, drain_timeout_us: int = 0, stream=None, gate=None, tenant: int = 0,
+                         workspace=None):
     """Native timing loop (optionally gated); returns (durations_ms, p50_ms, p95_ms)."""
     arr, n = _bufs(inputs)
     bo = out if isinstance(out, krex_buf) else buf(out)
@@ -327,8 +357,9 @@ def krex_bench_candidate(op: int, inputs, out, warmup: int, iters: int, flush_sc
                          None if gate is None else gate.handle, tenant, 0)
     d = (_f32 * max(iters, 1))()
     p50, p95 = _f64(math.nan), _f64(math.nan)
+    wp, wn = _ptr_bytes(workspace)
     _ok(lib().krex_bench_candidate(op, arr, n, bo, ctypes.byref(o), warmup, iters, d, ctypes.byref(p50),
-                                   ctypes.byref(p95), _stream(stream)), "krex_bench_candidate")
+                                   ctypes.byref(p95), wp, wn, _stream(stream)), "krex_bench_candidate")
     return list(d[:iters]), p50.value, p95.value
 
 
@@ -357,6 +388,18 @@ def krex_device_status() -> int:
     code = _u32(0)
     _ok(lib().krex_device_status(ctypes.byref(code)), "krex_device_status")
     return code.value
+
+
+def krex_device_status_detail() -> dict:
+    """Where the first time-out happened (all zero if none); does not clear."""
+    w = (_u64 * 8)()
+    _ok(lib().krex_device_status_detail(w), "krex_device_status_detail")
+    m = (1 << 21) - 1
+    lo, hi = (lambda x: x & 0xFFFFFFFF), (lambda x: x >> 32)
+    return {"code": lo(w[0]), "parity": hi(w[0]), "cta": lo(w[1]), "grid": hi(w[1]), "sm": lo(w[2]),
+            "cluster_rank": hi(w[2]), "waited_ns": w[3], "producer": (lo(w[4]), hi(w[4])),
+            "mma": (lo(w[5]), hi(w[5])), "epilogue": (lo(w[6]), hi(w[6])),
+            "MNK": (w[7] & m, (w[7] >> 21) & m, (w[7] >> 42) & m)}
 
 
 def krex_launch_count() -> int:

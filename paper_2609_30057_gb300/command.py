@@ -15,7 +15,7 @@ import math
 from dataclasses import dataclass, replace
 
 from . import (KREX_BF16, KREX_F32, KREX_OP_GEMM_BF16, KREX_OP_SOFTMAX_F32, buf, krex_check_scratch_bytes,
-               krex_command, krex_command_bufs, krex_command_run)
+               krex_command, krex_command_bufs, krex_command_run, krex_gemm_workspace_bytes)
 
 MiB = 1 << 20
 
@@ -92,12 +92,17 @@ class Workspace:
         self.ref = torch.empty(w.M, w.N, dtype=f32, device=device)
         self.flush = torch.empty(max(w.flush_bytes, 16), dtype=torch.uint8, device=device)
         self.check_scratch = torch.empty(krex_check_scratch_bytes(), dtype=torch.uint8, device=device)
+        # the GEMM's split-K meeting place: zero-filled once, left ready by every call
+        self.gemm_ws = (torch.zeros(krex_gemm_workspace_bytes(), dtype=torch.uint8, device=device)
+                        if w.op == KREX_OP_GEMM_BF16 else None)
         self.durations = (ctypes.c_float * w.iters)()
         self.cmd = krex_command(w.op, w.warmup, w.iters, 0, w.M, w.N, w.K, w.seed, w.sigma, w.atol, w.rtol, 0, 0,
                                 w.flush_bytes)
         ins = [buf(t) for t in self.inputs] + [buf(self.inputs[0])] * (2 - len(self.inputs))
         self.bufs = krex_command_bufs((type(ins[0]) * 2)(*ins), buf(self.out), buf(self.ref), self.flush.data_ptr(),
-                                      self.check_scratch.data_ptr(), krex_check_scratch_bytes())
+                                      self.check_scratch.data_ptr(), krex_check_scratch_bytes(),
+                                      None if self.gemm_ws is None else self.gemm_ws.data_ptr(),
+                                      0 if self.gemm_ws is None else self.gemm_ws.numel())
 
     def run(self, host_in=None, host_out=None, stream=None):
         """One benchmarking command; returns the krex_command_result."""

@@ -108,6 +108,15 @@ static krex_status check_buf(const krex_buf &b, const char *name) {
 
 static bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// The optional GEMM workspace: NULL, or 16-byte aligned and large enough.
+static krex_status check_gemm_workspace(const void *ws, size_t bytes) {
+    if (!ws) return KREX_OK;
+    if (!aligned16(ws)) return set_error(KREX_ERR_UNSUPPORTED, "GEMM workspace must be 16-byte aligned");
+    if (bytes < gemm_workspace_bytes())
+        return set_error(KREX_ERR_INVALID, "GEMM workspace of %zu bytes, need %zu", bytes, gemm_workspace_bytes());
+    return KREX_OK;
+}
+
 static krex_status check_op_shapes(int32_t op, const krex_buf *in, int32_t n_in, const krex_buf &out,
                                    int32_t out_dtype, const char *out_name) {
     if (!in) return set_error(KREX_ERR_INVALID, "in is null");
@@ -137,7 +146,8 @@ static krex_status check_op_shapes(int32_t op, const krex_buf *in, int32_t n_in,
 }
 
 // Candidate/reference dispatch after validation.
-static krex_status do_candidate(int32_t op, const krex_buf *in, const krex_buf &out, cudaStream_t s) {
+static krex_status do_candidate(int32_t op, const krex_buf *in, const krex_buf &out, cudaStream_t s,
+                                void *ws = nullptr, size_t ws_bytes = 0) {
     if (op == KREX_OP_GEMM_BF16) {
         const krex_buf &A = in[0], &B = in[1];
         const int64_t M = A.rows, K = A.cols, N = B.cols;
@@ -150,7 +160,7 @@ static krex_status do_candidate(int32_t op, const krex_buf *in, const krex_buf &
         }
         krex_status st = launch_gemm_tcgen05(static_cast<const uint16_t *>(A.ptr), A.ld,
                                              static_cast<const uint16_t *>(B.ptr), B.ld,
-                                             static_cast<uint16_t *>(out.ptr), out.ld, M, N, K, s);
+                                             static_cast<uint16_t *>(out.ptr), out.ld, M, N, K, ws, ws_bytes, s);
         if (st != KREX_OK) return st;
         if (K > 0) count_launches(1);
         return ok();
@@ -345,6 +355,16 @@ krex_status krex_run_candidate(int32_t op, const krex_buf *in, int32_t n_in, kre
     return do_candidate(op, in, out, reinterpret_cast<cudaStream_t>(stream));
 }
 
+size_t krex_gemm_workspace_bytes(void) { return gemm_workspace_bytes(); }
+
+krex_status krex_run_candidate_ws(int32_t op, const krex_buf *in, int32_t n_in, krex_buf out, void *workspace,
+                                  size_t workspace_bytes, krex_stream_t stream) {
+    krex_status st = check_op_shapes(op, in, n_in, out, op == KREX_OP_GEMM_BF16 ? KREX_BF16 : KREX_F32, "out");
+    if (st) return st;
+    if ((st = check_gemm_workspace(workspace, workspace_bytes))) return st;
+    return do_candidate(op, in, out, reinterpret_cast<cudaStream_t>(stream), workspace, workspace_bytes);
+}
+
 krex_status krex_run_reference(int32_t op, const krex_buf *in, int32_t n_in, krex_buf ref, krex_stream_t stream) {
     krex_status st = check_op_shapes(op, in, n_in, ref, KREX_F32, "ref");
     if (st) return st;
@@ -532,24 +552,27 @@ krex_status krex_region_end(krex_region *r, float *durations_ms, int32_t cap, in
 
 krex_status krex_bench_candidate(int32_t op, const krex_buf *in, int32_t n_in, krex_buf out,
                                  const krex_region_opts *opts, int32_t warmup, int32_t iters, float *durations_ms,
-                                 double *p50_ms, double *p95_ms, krex_stream_t stream) {
+                                 double *p50_ms, double *p95_ms, void *workspace, size_t workspace_bytes,
+                                 krex_stream_t stream) {
     if (!opts) return set_error(KREX_ERR_INVALID, "opts is null");
     if (warmup < 0 || iters < 0 || iters > opts->max_iters)
         return set_error(KREX_ERR_INVALID, "need 0 <= warmup and 0 <= iters <= max_iters");
     krex_status st = check_op_shapes(op, in, n_in, out, op == KREX_OP_GEMM_BF16 ? KREX_BF16 : KREX_F32, "out");
     if (st) return st;
+    if ((st = check_gemm_workspace(workspace, workspace_bytes))) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     krex_region *r = nullptr;
     if ((st = krex_region_begin(&r, stream, opts))) return st;
     for (int32_t w = 0; w < warmup; ++w) {
-        if ((st = do_flush(opts->flush_scratch, opts->flush_bytes, s)) || (st = do_candidate(op, in, out, s))) {
+        if ((st = do_flush(opts->flush_scratch, opts->flush_bytes, s)) ||
+            (st = do_candidate(op, in, out, s, workspace, workspace_bytes))) {
             krex_region_abort(r);
             return st;
         }
     }
     for (int32_t i = 0; i < iters; ++i) {
         if ((st = do_flush(opts->flush_scratch, opts->flush_bytes, s)) || (st = krex_iter_begin(r)) ||
-            (st = do_candidate(op, in, out, s)) || (st = krex_iter_end(r))) {
+            (st = do_candidate(op, in, out, s, workspace, workspace_bytes)) || (st = krex_iter_end(r))) {
             krex_region_abort(r);
             return st;
         }
@@ -576,6 +599,7 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
         return set_error(KREX_ERR_INVALID, "command: buffers do not match rows M, cols N");
     }
     if (cmd->flush_bytes > 0 && !bufs->flush_scratch) return set_error(KREX_ERR_INVALID, "command: flush scratch is null");
+    if (krex_status st0 = check_gemm_workspace(bufs->gemm_workspace, bufs->gemm_workspace_bytes)) return st0;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     memset(result, 0, sizeof(*result));
     const uint64_t launches0 = g_launches.load();
@@ -607,7 +631,7 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
     result->phase_ms[1] = ms_since(t);
     // 3) candidate once, for the check
     t = clk::now();
-    if ((st = do_candidate(op, bufs->in, bufs->out, s))) return st;
+    if ((st = do_candidate(op, bufs->in, bufs->out, s, bufs->gemm_workspace, bufs->gemm_workspace_bytes))) return st;
     KREX_CUDA_TRY(cudaStreamSynchronize(s));
     result->phase_ms[2] = ms_since(t);
     // 4) check
@@ -630,7 +654,8 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
         o.flush_scratch = bufs->flush_scratch;
         o.flush_bytes = cmd->flush_bytes;
         if ((st = krex_bench_candidate(op, bufs->in, n_in, bufs->out, &o, cmd->warmup, cmd->iters, durations_ms,
-                                       &result->p50_ms, &result->p95_ms, stream)))
+                                       &result->p50_ms, &result->p95_ms, bufs->gemm_workspace,
+                                       bufs->gemm_workspace_bytes, stream)))
             return st;
         result->n_iters = cmd->iters;
     }
@@ -659,6 +684,14 @@ krex_status krex_device_status(uint32_t *code) {
     if (!code) return set_error(KREX_ERR_INVALID, "code is null");
     KREX_CUDA_TRY(read_and_clear_device_status(code));
     if (*code) return set_error(KREX_ERR_DEVICE, "a kernel's bounded wait ran out (status 0x%x)", *code);
+    return ok();
+}
+
+krex_status krex_device_status_detail(uint64_t *words) {
+    if (!words) return set_error(KREX_ERR_INVALID, "words is null");
+    unsigned long long w[8];
+    KREX_CUDA_TRY(read_device_status_detail(w));
+    for (int i = 0; i < 8; ++i) words[i] = (uint64_t)w[i];
     return ok();
 }
 

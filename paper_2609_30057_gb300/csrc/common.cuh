@@ -39,11 +39,14 @@ cudaError_t launch_gemm_ref(const uint16_t *a, int64_t lda, const uint16_t *b, i
                             float *c, int64_t ldc, int64_t M, int64_t N, int64_t K,
                             cudaStream_t s);
 // K4: tcgen05 GEMM.  Returns KREX_OK or an error status with a message set.
+// `workspace` (may be NULL) enables the split-K tail; see gemm_workspace_bytes.
 krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb,
                                 uint16_t *c, int64_t ldc, int64_t M, int64_t N, int64_t K,
-                                cudaStream_t s);
+                                void *workspace, size_t workspace_bytes, cudaStream_t s);
+size_t gemm_workspace_bytes();
 // Device status word of the GEMM kernel's bounded waits (read and clear).
 cudaError_t read_and_clear_device_status(uint32_t *code);
+cudaError_t read_device_status_detail(unsigned long long *words);
 
 // Count kernels launched outside api.cu in krex_launch_count().
 void note_launches(int n);

@@ -25,6 +25,7 @@
 #include <cuda_bf16.h>
 #include <cudaTypedefs.h>
 
+#include <atomic>
 #include <mutex>
 #include <unordered_map>
 
@@ -33,6 +34,9 @@
 namespace krex {
 
 __device__ uint32_t g_gemm_status;  // 0 = ok; else 0x1000 | role << 4 | site
+// Where the first time-out happened (written by the thread whose CAS set
+// g_gemm_status): see record_timeout.
+__device__ unsigned long long g_gemm_diag[8];
 
 namespace {
 
@@ -49,7 +53,7 @@ constexpr int GROUP_M = 16;
 constexpr int EPI_THREADS = 128;
 constexpr int NUM_BARS = 2 * STAGES + 4 + 1;        // full, empty, tmem_full[2], tmem_empty[2], mma_done
 constexpr size_t SMEM_BYTES = 1024 /*align slack*/ + (size_t)STAGES * (A_STAGE_BYTES + B_STAGE_BYTES) +
-                              NUM_BARS * 8 + 16;
+                              NUM_BARS * 8 + 48;
 
 // Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (bits 7-9 =
 // 1), B bf16 (bits 10-12 = 1), A K-major (bit 15 = 0), B MN-major (bit 16 = 1),
@@ -74,6 +78,23 @@ __device__ __forceinline__ uint64_t globaltimer() {
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
     return t;
 }
+
+// Elapsed time of a bounded wait, summed over the steps between successive
+// checks.  A step that goes backwards or forward by more than 50 ms is a
+// timer adjustment, not waiting, and is not counted: an unsigned difference
+// against the start would turn a timer that steps back into an immediate
+// time-out.
+struct WaitClock {
+    uint64_t last, elapsed;
+    __device__ __forceinline__ WaitClock() : last(globaltimer()), elapsed(0) {}
+    __device__ __forceinline__ bool expired(uint64_t limit_ns) {
+        const uint64_t now = globaltimer();
+        const int64_t d = (int64_t)(now - last);
+        last = now;
+        if (d > 0 && d < 50000000ll) elapsed += (uint64_t)d;
+        return elapsed > limit_ns;
+    }
+};
 
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
@@ -113,17 +134,47 @@ __device__ __forceinline__ bool mbar_test_wait(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
+// Per-CTA progress words that follow the abort flag in shared memory
+// (prog[0] is the abort flag): 1-2 producer item / K stage, 3-4 MMA item / K
+// stage, 5-6 first epilogue warp's item / step, 7-9 M, N, K.  Plain stores by
+// one thread per role; read only when a wait runs out.
+constexpr int PROG_WORDS = 10;
+
+__device__ __forceinline__ uint32_t smid() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
+    return r;
+}
+
+// First time-out of the device: set the status word and, if this thread set
+// it, record where every role of this CTA was.
+__device__ __noinline__ void record_timeout(uint32_t code, volatile uint32_t *prog, uint64_t elapsed_ns,
+                                            uint32_t parity) {
+    prog[0] = 1u;  // abort
+    if (atomicCAS(&g_gemm_status, 0u, code) != 0u) return;
+    uint32_t rank;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
+    g_gemm_diag[0] = code | ((unsigned long long)parity << 32);
+    g_gemm_diag[1] = blockIdx.x | ((unsigned long long)gridDim.x << 32);
+    g_gemm_diag[2] = smid() | ((unsigned long long)rank << 32);
+    g_gemm_diag[3] = elapsed_ns;
+    g_gemm_diag[4] = prog[1] | ((unsigned long long)prog[2] << 32);
+    g_gemm_diag[5] = prog[3] | ((unsigned long long)prog[4] << 32);
+    g_gemm_diag[6] = prog[5] | ((unsigned long long)prog[6] << 32);
+    g_gemm_diag[7] = prog[7] | ((unsigned long long)prog[8] << 21) | ((unsigned long long)prog[9] << 42);
+    __threadfence();
+}
+
 // Slow path of mbar_wait: bounded polling with try_wait.
 __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, volatile uint32_t *abort_flag,
                                             uint64_t timeout_ns, uint32_t site, bool drain) {
-    const uint64_t t0 = globaltimer();
+    WaitClock clk;
     for (uint32_t spin = 1;; ++spin) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((spin & 63u) == 0) {
             if (!drain && *abort_flag) return false;
-            if (globaltimer() - t0 > timeout_ns) {
-                *abort_flag = 1u;
-                atomicCAS(&g_gemm_status, 0u, 0x1000u | site);
+            if (clk.expired(timeout_ns)) {
+                record_timeout(0x1000u | site, abort_flag, clk.elapsed, parity);
                 return false;
             }
         }
@@ -233,7 +284,10 @@ gemm_bf16_tcgen05(const __grid_constant__ CUtensorMap tmA, const __grid_constant
             mbar_init(tempty_bar(a), EPI_THREADS);
         }
         mbar_init(mma_done_bar, 1);
-        *abort_flag = 0u;
+        for (int i = 0; i < PROG_WORDS; ++i) abort_flag[i] = 0u;
+        abort_flag[7] = (uint32_t)M;
+        abort_flag[8] = (uint32_t)N;
+        abort_flag[9] = (uint32_t)K;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
@@ -430,7 +484,7 @@ struct Cfg {
     static constexpr int A_STAGE_BYTES = KSUB * A_SUB_BYTES;
     static constexpr int B_STAGE_BYTES = KSUB * B_SUB_BYTES;
     static constexpr int NUM_BARS = 2 * STAGES + 4 + 1;
-    static constexpr size_t SMEM_BYTES = 1024 + (size_t)RING_BYTES + EPI_BYTES + NUM_BARS * 8 + 16;
+    static constexpr size_t SMEM_BYTES = 1024 + (size_t)RING_BYTES + EPI_BYTES + NUM_BARS * 8 + 48;
 };
 // kind::f16, D fp32, A/B bf16, A K-major, B MN-major, M = 256 (pair); N is
 // added at run time in bits 17-22
@@ -458,6 +512,14 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
 
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
+                 : "memory");
+}
+
+// Arrive without ordering: a count only (publishes no data).  The release
+// form costs a cluster-scope fence, which on the producer's per-stage path
+// took a third off the GEMM's throughput (measured on GB300).
+__device__ __forceinline__ void mbar_arrive_remote_relaxed(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
                  : "memory");
 }
 
@@ -527,31 +589,72 @@ __device__ __forceinline__ void tile_coords_pair(int tile, int tiles_m, int tile
     nb = in_g / gsize;
 }
 
-// Work item w of the 2-SM kernel -> pair tile (mb, nb), its first column and
-// its width.  Items below full_items are whole pair tiles (width bn); the rest
-// are halves (width bn/2) of the last tiles, so a final partial wave keeps
-// twice as many SM pairs busy.
-__device__ __forceinline__ void work_item(int w, int full_items, int tiles_m, int tiles_n, int group_m, int bn,
-                                          int &mb, int &nb, int &col0, int &width) {
+// Work item w of the 2-SM kernel.  Items below full_items are whole pair
+// tiles: width bn, all K stages.  The rest split the tiles of a final partial
+// wave in two, so that wave keeps twice as many SM pairs busy: into K halves
+// (split_k: stages [0, mid) and [mid, num_kb), partial sums combined through
+// the workspace; slot = tile - full_items) or, without a workspace, into
+// column halves of width bn/2.
+struct WorkItem {
+    int mb, nb, col0, width, kb0, kb1, slot;
+};
+
+__device__ __forceinline__ WorkItem work_item(int w, int full_items, int tiles_m, int tiles_n, int group_m, int bn,
+                                              int num_kb, int split_k) {
+    WorkItem it;
     int tile = w, half = -1;
     if (w >= full_items) {
         const int u = w - full_items;
         tile = full_items + (u >> 1);
         half = u & 1;
     }
-    tile_coords_pair(tile, tiles_m, tiles_n, group_m, mb, nb);
-    if (half < 0) {
-        col0 = nb * bn;
-        width = bn;
-    } else {
-        width = bn >> 1;
-        col0 = nb * bn + half * width;
+    tile_coords_pair(tile, tiles_m, tiles_n, group_m, it.mb, it.nb);
+    it.col0 = it.nb * bn;
+    it.width = bn;
+    it.kb0 = 0;
+    it.kb1 = num_kb;
+    it.slot = -1;
+    if (half >= 0) {
+        if (split_k) {
+            const int mid = num_kb >> 1;
+            it.kb0 = half ? mid : 0;
+            it.kb1 = half ? num_kb : mid;
+            it.slot = tile - full_items;
+        } else {
+            it.width = bn >> 1;
+            it.col0 += half * it.width;
+        }
+    }
+    return it;
+}
+
+__device__ __forceinline__ void flag_store_release(uint32_t *p, uint32_t v) {
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ uint32_t flag_load_acquire(const uint32_t *p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+// Bounded wait until *p == v (a peer CTA that is already running publishes it).
+__device__ __noinline__ uint32_t flag_wait_acquire(const uint32_t *p, uint32_t v, volatile uint32_t *abort_flag,
+                                                   uint64_t timeout_ns, uint32_t site) {
+    WaitClock clk;
+    for (uint32_t spin = 1;; ++spin) {
+        if (flag_load_acquire(p) == v) return 1u;
+        if ((spin & 63u) == 0) {
+            if (*abort_flag) return 0u;
+            if (clk.expired(timeout_ns)) {
+                record_timeout(0x1000u | site, abort_flag, clk.elapsed, v);
+                return 0u;
+            }
+        }
     }
 }
 
 __device__ __forceinline__ void spin_ns(uint64_t ns) {
-    const uint64_t t0 = globaltimer();
-    while (globaltimer() - t0 < ns) {
+    WaitClock clk;
+    while (!clk.expired(ns)) {
     }
 }
 
@@ -562,7 +665,8 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ CUtensorMap tmC, uint16_t *__restrict__ C, int64_t ldc, int M,
                       int N, int K, int bn, int tiles_m, int tiles_n, int full_items, int num_items,
-                      int group_m, int c_vec, int c_tma, int stages, uint64_t timeout_ns) {
+                      int group_m, int c_vec, int c_tma, int stages, uint64_t timeout_ns, int split_k,
+                      float *ws_partial, uint32_t *ws_count, uint32_t *ws_flag, uint32_t launch_id) {
     // this kernel's tile constants shadow the 1-SM ones
     using CF = v2::Cfg<KSUB>;
     constexpr int BM = v2::BM, BN = v2::BN, BK = v2::BK, STAGES = CF::STAGES;
@@ -596,7 +700,7 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
-            mbar_init(full_bar(s), 1);
+            mbar_init(full_bar(s), 2);  // leader's expect_tx + the peer producer's arrive
             mbar_init(empty_bar(s), 1);
         }
         for (int a = 0; a < 2; ++a) {
@@ -604,7 +708,10 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
             mbar_init(tempty_bar(a), 2 * EPI_WARPS);  // one arrive per epilogue warp of both CTAs
         }
         mbar_init(mma_done_bar, 1);
-        *abort_flag = 0u;
+        for (int i = 0; i < PROG_WORDS; ++i) abort_flag[i] = 0u;
+        abort_flag[7] = (uint32_t)M;
+        abort_flag[8] = (uint32_t)N;
+        abort_flag[9] = (uint32_t)K;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
@@ -629,8 +736,9 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
         uint32_t phase = 0;
         bool ok = true;
         for (int w = cluster_id; ok && w < num_items; w += nclusters) {
-            int mb, nb, col0, width;
-            work_item(w, full_items, tiles_m, tiles_n, group_m, bn, mb, nb, col0, width);
+            const WorkItem it = work_item(w, full_items, tiles_m, tiles_n, group_m, bn, num_kb, split_k);
+            const int mb = it.mb, nb = it.nb, col0 = it.col0, width = it.width;
+            (void)nb;
             const int b_half = width >> 1;                            // B columns per CTA
             const int b_boxes = (b_half + B_BOX_N - 1) / B_BOX_N;     // TMA boxes per CTA and stage
             // what each CTA of the pair loads (boxes wholly outside the matrix are skipped)
@@ -644,14 +752,22 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                                                   (nbox[0] + nbox[1]) * B_BOX_BYTES);  // per K sub-block
             const int m0 = mb * 2 * BM + (int)rank * BM;
             const int n0 = col0 + (int)rank * b_half;
-            for (int kb = 0; kb < num_kb; ++kb) {
+            abort_flag[1] = (uint32_t)w;
+            for (int kb = it.kb0; kb < it.kb1; ++kb) {
+                abort_flag[2] = (uint32_t)kb;
                 if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, timeout_ns, 0x31)) {
                     ok = false;
                     break;
                 }
                 const int nsub = min(KSUB, num_ksub - kb * KSUB);  // sub-blocks inside K
-                if (leader) mbar_expect_tx(full_bar(stage), sub_bytes * (uint32_t)nsub);
                 const uint32_t fb = mapa_shared(full_bar(stage), 0);
+                // Both producers arrive on the leader's full barrier, so the MMA
+                // never consumes a stage the peer producer has not reached.  A
+                // peer whose rows and columns of this item all lie outside the
+                // matrix loads nothing; without its arrive it could fall two
+                // phases behind its empty barrier and wait on an aliased parity.
+                if (leader) mbar_expect_tx(full_bar(stage), sub_bytes * (uint32_t)nsub);
+                else mbar_arrive_remote_relaxed(fb);
                 for (int h = 0; h < nsub; ++h) {
                     const int k0 = (kb * KSUB + h) * BK;
                     if (a_ok[rank])
@@ -674,18 +790,20 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
         bool ok = true;
         int local = 0;
         for (int w = cluster_id; ok && w < num_items; w += nclusters, ++local) {
-            int mb, nb, col0, width;
-            work_item(w, full_items, tiles_m, tiles_n, group_m, bn, mb, nb, col0, width);
-            const uint32_t idesc = v2::IDESC_NO_N | ((uint32_t)(width >> 3) << 17);
+            const WorkItem it = work_item(w, full_items, tiles_m, tiles_n, group_m, bn, num_kb, split_k);
+            const uint32_t idesc = v2::IDESC_NO_N | ((uint32_t)(it.width >> 3) << 17);
             const int acc = local & 1;
             const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
+            abort_flag[3] = (uint32_t)w;
+            abort_flag[4] = 0xFFFFFFFFu;  // waiting for the accumulator
             if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, timeout_ns, 0x41)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
             const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
-            for (int kb = 0; kb < num_kb; ++kb) {
+            for (int kb = it.kb0; kb < it.kb1; ++kb) {
+                abort_flag[4] = (uint32_t)kb;
                 if (!mbar_wait(full_bar(stage), phase, abort_flag, timeout_ns, 0x42)) {
                     ok = false;
                     break;
@@ -702,7 +820,7 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
 #pragma unroll
                         for (int k = 0; k < BK / 16; ++k)
                             mma_bf16_pair(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(128 * k), idesc,
-                                          (kb | h | k) != 0 ? 1u : 0u);
+                                          ((kb - it.kb0) | h | k) != 0 ? 1u : 0u);
                     }
                 }
                 mma_commit_pair(empty_bar(stage));
@@ -723,18 +841,65 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
         uint32_t epi_buf = 0;  // staging buffers used so far by this warp
         int local = 0;
         for (int w = cluster_id; w < num_items; w += nclusters, ++local) {
-            int mb, nb, col0, width;
-            work_item(w, full_items, tiles_m, tiles_n, group_m, bn, mb, nb, col0, width);
+            const WorkItem it = work_item(w, full_items, tiles_m, tiles_n, group_m, bn, num_kb, split_k);
+            const int mb = it.mb, nb = it.nb, col0 = it.col0, width = it.width;
+            (void)nb;
             const int acc = local & 1;
             const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
+            if (ew == 0 && lane == 0) {
+                abort_flag[5] = (uint32_t)w;
+                abort_flag[6] = 1u;  // waiting for the accumulator
+            }
             const bool waited = mbar_wait(tfull_bar(acc), acc_phase, abort_flag, timeout_ns, 0x51);
+            if (ew == 0 && lane == 0) abort_flag[6] = 2u;  // draining it
             if (!__all_sync(0xffffffffu, waited)) break;
             tc_fence_after();
             const int row0 = mb * 2 * BM + (int)rank * BM + ew * 32;  // this warp's 32 rows
             const int row = row0 + lane;
             const int n0 = col0;
             const uint32_t tbase = tmem_base + ((uint32_t)(ew * 32) << 16) + (uint32_t)(acc * BN);
-            if (c_tma) {
+            // Split-K half: of the two halves of a tile, the first to get here
+            // parks its fp32 partial for these 32 rows in the workspace
+            // ([column][row], coalesced) and publishes it with a flag tagged by
+            // this launch; the second waits for the flag, adds the partial and
+            // stores C.  The arrival counter resets itself (atomicInc wraps).
+            // Partials are written and read at L2 (st.cg / ld.cg): they cross SMs
+            // inside one launch.
+            bool store_c = true;
+            const float *add = nullptr;
+            if (it.slot >= 0) {
+                const int sidx = (it.slot * 2 + (int)rank) * EPI_WARPS + ew;
+                float *part = ws_partial + (size_t)sidx * (32 * BN);
+                uint32_t first = 0;
+                if (lane == 0) first = atomicInc(&ws_count[sidx], 1u) == 0u ? 1u : 0u;
+                first = __shfl_sync(0xffffffffu, first, 0);
+                if (first) {
+#pragma unroll 1
+                    for (int c = 0; c < width / 32; ++c) {
+                        uint32_t v[32];
+                        tmem_ld32(tbase + (uint32_t)(c * 32), v);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) __stcg(part + (c * 32 + i) * 32 + lane, __uint_as_float(v[i]));
+                    }
+                    __threadfence();
+                    __syncwarp();
+                    if (lane == 0) flag_store_release(ws_flag + sidx, launch_id);
+                    store_c = false;
+                } else {
+                    uint32_t ok = 1u;
+                    if (lane == 0) ok = flag_wait_acquire(ws_flag + sidx, launch_id, abort_flag, timeout_ns, 0x52);
+                    ok = __shfl_sync(0xffffffffu, ok, 0);
+                    if (ok) {
+                        (void)flag_load_acquire(ws_flag + sidx);  // every lane acquires the partial
+                        add = part;
+                    } else {
+                        store_c = false;
+                    }
+                }
+            }
+            if (!store_c) {
+                // nothing to store for this item
+            } else if (c_tma) {
                 // 64-column chunks: TMEM -> registers -> bf16 -> 128B-swizzled staging
                 // buffer (row = lane, 16-byte chunk j at j ^ (lane % 8)) -> one TMA store of
                 // the 32 x 64 box; two buffers per warp alternate.
@@ -750,6 +915,12 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                         for (int h = 0; h < 2; ++h) {
                             uint32_t v[32];
                             tmem_ld32(tbase + (uint32_t)(c * v2::EPI_BOX_COLS + h * 32), v);
+                            if (add) {
+                                const float *pc = add + (c * v2::EPI_BOX_COLS + h * 32) * 32 + lane;
+#pragma unroll
+                                for (int i = 0; i < 32; ++i)
+                                    v[i] = __float_as_uint(__uint_as_float(v[i]) + __ldcg(pc + i * 32));
+                            }
 #pragma unroll
                             for (int q = 0; q < 4; ++q) {
                                 uint32_t w[4];
@@ -781,6 +952,11 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                     if (col0 >= N) break;  // warp-uniform
                     uint32_t v[32];
                     tmem_ld32(tbase + (uint32_t)(c * 32), v);
+                    if (add) {
+                        const float *pc = add + (c * 32) * 32 + lane;
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) + __ldcg(pc + i * 32));
+                    }
                     if (row < M) {
                         uint32_t p[16];
 #pragma unroll
@@ -805,6 +981,7 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_remote(acc ? tempty_leader1 : tempty_leader0);
+            if (ew == 0 && lane == 0) abort_flag[6] = 3u;  // released
         }
         if (lane == 0) bulk_wait_group_all();  // stores complete before shared memory goes away
         __syncwarp();
@@ -954,9 +1131,19 @@ uint64_t wait_timeout_ns() {
 
 }  // namespace
 
+// Split-K workspace: fp32 partials of up to WS_SLOTS split tiles (2 CTAs x 4
+// epilogue warps x 32 rows x 256 columns each), then one arrival counter and
+// one flag per 32-row slab.
+constexpr int WS_SLOTS = 64;
+constexpr size_t WS_SLABS = (size_t)WS_SLOTS * 2 * 4;
+constexpr size_t WS_PARTIAL_BYTES = WS_SLABS * 32 * 256 * sizeof(float);
+constexpr size_t WS_BYTES = WS_PARTIAL_BYTES + 2 * WS_SLABS * sizeof(uint32_t);
+
+size_t gemm_workspace_bytes() { return WS_BYTES; }
+
 krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb,
                                 uint16_t *c, int64_t ldc, int64_t M, int64_t N, int64_t K,
-                                cudaStream_t s) {
+                                void *workspace, size_t workspace_bytes, cudaStream_t s) {
     if (M == 0 || N == 0) return KREX_OK;
     if (K == 0) {
         KREX_CUDA_TRY(cudaMemset2DAsync(c, (size_t)ldc * 2, 0, (size_t)N * 2, (size_t)M, s));
@@ -1029,14 +1216,33 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         const int64_t full_items = split ? tiles - rem : tiles;
         const int64_t items = split ? tiles + rem : tiles;
         const int clusters = (int)(items < max_clusters ? items : max_clusters);
-        if (stage_ksub() == 2)
+        // K halves (full-width MMAs) when a zero-initialised workspace is given,
+        // K has at least two ring stages and the split tiles are the whole
+        // GEMM (one partial wave); else column halves.  Measured on GB300: K
+        // halves load a third less than column halves (1024 x 2048 x 8192:
+        // 8 % faster), but the partial sums' hand-over sits on the last wave's
+        // critical path (4096^3, 28 of 256 tiles split: 2 % slower).
+        const int ksub = stage_ksub();
+        const int64_t num_kb = (((K + 63) / 64) + ksub - 1) / ksub;
+        const int split_k = split && full_items == 0 && workspace && workspace_bytes >= WS_BYTES &&
+                            rem <= WS_SLOTS && num_kb >= 2 && clusters >= 2;
+        static std::atomic<uint32_t> launch_counter{0};
+        uint32_t launch_id = launch_counter.fetch_add(1) + 1;
+        if (launch_id == 0) launch_id = launch_counter.fetch_add(1) + 1;  // 0 never tags a published partial
+        float *ws_partial = split_k ? static_cast<float *>(workspace) : nullptr;
+        uint32_t *ws_count =
+            split_k ? reinterpret_cast<uint32_t *>(static_cast<uint8_t *>(workspace) + WS_PARTIAL_BYTES) : nullptr;
+        uint32_t *ws_flag = split_k ? ws_count + WS_SLABS : nullptr;
+        if (ksub == 2)
             gemm_bf16_tcgen05_2sm<2><<<2 * clusters, THREADS, v2::Cfg<2>::SMEM_BYTES, s>>>(
                 ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, (int)full_items, (int)items,
-                raster_group(), c_vec, c_tma, ring_stages(v2::Cfg<2>::STAGES), wait_timeout_ns());
+                raster_group(), c_vec, c_tma, ring_stages(v2::Cfg<2>::STAGES), wait_timeout_ns(), split_k, ws_partial,
+                ws_count, ws_flag, launch_id);
         else
             gemm_bf16_tcgen05_2sm<1><<<2 * clusters, THREADS, v2::Cfg<1>::SMEM_BYTES, s>>>(
                 ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, (int)full_items, (int)items,
-                raster_group(), c_vec, c_tma, ring_stages(v2::Cfg<1>::STAGES), wait_timeout_ns());
+                raster_group(), c_vec, c_tma, ring_stages(v2::Cfg<1>::STAGES), wait_timeout_ns(), split_k, ws_partial,
+                ws_count, ws_flag, launch_id);
     } else {
         const int tiles_m = (int)((M + BM - 1) / BM), tiles_n = (int)((N + BN - 1) / BN);
         const int64_t tiles = (int64_t)tiles_m * tiles_n;
@@ -1048,13 +1254,22 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
     return KREX_OK;
 }
 
+cudaError_t read_device_status_detail(unsigned long long *words) {
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return e;
+    return cudaMemcpyFromSymbol(words, g_gemm_diag, sizeof(g_gemm_diag));
+}
+
 cudaError_t read_and_clear_device_status(uint32_t *code) {
     cudaError_t e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return e;
     e = cudaMemcpyFromSymbol(code, g_gemm_status, sizeof(uint32_t));
     if (e != cudaSuccess) return e;
     const uint32_t zero = 0;
-    return cudaMemcpyToSymbol(g_gemm_status, &zero, sizeof(uint32_t));
+    e = cudaMemcpyToSymbol(g_gemm_status, &zero, sizeof(uint32_t));
+    if (e != cudaSuccess) return e;
+    const unsigned long long zeros[8] = {};
+    return cudaMemcpyToSymbol(g_gemm_diag, zeros, sizeof(zeros));
 }
 
 }  // namespace krex

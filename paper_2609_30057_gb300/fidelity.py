@@ -29,14 +29,18 @@ import threading
 import time
 
 from . import (KREX_OP_GEMM_BF16, KREX_OP_SOFTMAX_F32, Gate, KrexError, build, krex_bench_candidate,
-               krex_device_status, krex_gen_inputs, krex_run_candidate)
+               krex_device_status, krex_device_status_detail, krex_gen_inputs, krex_run_candidate)
 
 
-def _device_status() -> int:
-    """The kernels' status word (non-zero: a bounded wait ran out); read and cleared."""
+def _device_status(details: dict | None = None, phase: str = "") -> int:
+    """The kernels' status word (non-zero: a bounded wait ran out); read and
+    cleared.  Where a wait ran out is added to `details` under `phase`."""
+    detail = krex_device_status_detail()
     try:
         return krex_device_status()
     except KrexError as e:
+        if details is not None:
+            details[phase] = detail
         return int(str(e).split("status 0x")[-1].rstrip(")"), 16) if "status 0x" in str(e) else -1
 
 
@@ -209,15 +213,15 @@ def run(tenants: int = 2, iters: int = 20, quick: bool = False) -> dict:
     flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
     cands = candidates(quick=quick)
     names = [c[0] for c in cands]
-    status = {}
+    status, details = {}, {}
     time_candidates(cands, flush, 3, stream)                       # warm everything up
     native = time_candidates(cands, flush, iters, stream)
     repeat = time_candidates(cands, flush, iters, stream)
-    status["native"] = _device_status()
+    status["native"] = _device_status(details, "native")
     with Background(tenants, None) as bg:
         ungated = time_candidates(cands, flush, iters, stream)
         ungated_bg = sum(bg.launched)
-    status["ungated"] = _device_status()
+    status["ungated"] = _device_status(details, "ungated")
     gate = Gate(16)
     holder = gate.register(stream)
     with Background(tenants, gate) as bg:
@@ -225,9 +229,9 @@ def run(tenants: int = 2, iters: int = 20, quick: bool = False) -> dict:
         gated_bg = sum(bg.launched)
     gate.unregister(holder)
     gate.close()
-    status["gated"] = _device_status()
+    status["gated"] = _device_status(details, "gated")
     return {
-        "device_status": status,
+        "device_status": status, "device_status_detail": details,
         "candidates": names, "native_ms": native,
         "conditions": {"repeat": {"ms": repeat, **summarize(repeat, native)},
                        "ungated": {"ms": ungated, "background_launches": ungated_bg, **summarize(ungated, native)},

@@ -49,6 +49,7 @@ def test_struct_layouts_match_the_header():
     assert ctypes.sizeof(krex.krex_region_opts) == 56
     assert ctypes.sizeof(krex.krex_command) == 80
     assert ctypes.sizeof(krex.krex_command_result) == 88
+    assert ctypes.sizeof(krex.krex_command_bufs) == 200
 
 
 def test_status_strings_and_version(lib):
@@ -95,6 +96,13 @@ def test_invalid_arguments_fail_before_any_cuda_call(lib):
     assert lib.krex_run_candidate(0, ins, 2, _b(16, BF, 8, 8), None) == krex.KREX_ERR_INVALID
     assert lib.krex_run_candidate(0, ins, 1, _b(16, BF, 8, 8), None) == krex.KREX_ERR_INVALID
     assert lib.krex_run_candidate(9, ins, 2, _b(16, BF, 8, 8), None) == krex.KREX_ERR_INVALID
+    # an optional GEMM workspace must be large enough and 16-byte aligned
+    # (checked before anything reaches the GPU)
+    ok_ins = (krex.krex_buf * 2)(_b(16, BF, 8, 8), _b(16, BF, 8, 8))
+    nws = lib.krex_gemm_workspace_bytes()
+    assert nws >= 16 << 20
+    assert lib.krex_run_candidate_ws(0, ok_ins, 2, _b(16, BF, 8, 8), 4096, nws - 16, None) == krex.KREX_ERR_INVALID
+    assert lib.krex_run_candidate_ws(0, ok_ins, 2, _b(16, BF, 8, 8), 4104, nws, None) == krex.KREX_ERR_UNSUPPORTED
     # the reference writes fp32
     ins = (krex.krex_buf * 2)(_b(16, BF, 8, 8), _b(16, BF, 8, 8))
     assert lib.krex_run_reference(0, ins, 2, _b(16, BF, 8, 8), None) == krex.KREX_ERR_INVALID

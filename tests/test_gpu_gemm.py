@@ -198,3 +198,76 @@ def test_gemm_large_sampled(n, seed):
     # property at any size: the whole output is finite and bounded by K
     assert torch.isfinite(c.float()).all().item()
     assert c.float().abs().max().item() <= n
+
+
+@pytest.mark.parametrize("ksub", ["2", "1"])
+@pytest.mark.parametrize("M,N,K", [(1024, 2048, 512), (256, 256, 4096), (300, 1000, 520), (640, 384, 4104),
+                                   (1536, 1536, 3072), (2064, 1000, 1032), (4096, 4096, 256)])
+def test_2sm_split_k_tail(M, N, K, ksub, monkeypatch):
+    # with a workspace the tiles of a GEMM that fits in one partial wave are
+    # split into K halves whose fp32 partials meet in the workspace (larger
+    # GEMMs keep column halves); two calls in a row (the arrival counters
+    # reset themselves, the flags are tagged per launch)
+    monkeypatch.setenv("KREX_GEMM_SM", "2")
+    monkeypatch.setenv("KREX_GEMM_KSUB", ksub)
+    seed = 6000 + M + N + K
+    a, b = _gen(seed, M, N, K)
+    ws = krex.gemm_workspace()
+    want = ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N))
+    for _ in range(2):
+        c = Guarded(M, N, torch.bfloat16)
+        krex.krex_run_candidate_ws(krex.KREX_OP_GEMM_BF16, [a, b], c.view, ws)
+        torch.cuda.synchronize()
+        assert krex.krex_device_status() == 0
+        assert c.canaries_intact()
+        ok, worst = _within_tol(bits16(c.view), want, K)
+        assert ok, worst
+        # the workspace ends with 512 arrival counters, then 512 flags (uint32 each)
+        counters = ws[ws.numel() - 4096:ws.numel() - 2048]
+        assert torch.count_nonzero(counters).item() == 0  # every arrival counter back at 0
+
+
+def test_split_k_matches_column_split_closely():
+    # K halves and column halves sum the same products in different orders:
+    # both within tolerance, and equal in most elements
+    M, N, K = 1536, 1536, 3072
+    a, b = _gen(2, M, N, K)
+    c0 = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    c1 = torch.empty_like(c0)
+    krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [a, b], c0)
+    krex.krex_run_candidate_ws(krex.KREX_OP_GEMM_BF16, [a, b], c1, krex.gemm_workspace())
+    torch.cuda.synchronize()
+    assert krex.krex_device_status() == 0
+    same = (c0.view(torch.int16) == c1.view(torch.int16)).float().mean().item()
+    assert same > 0.9
+    want = ref.gemm_f64(gen.uniform_bf16(2, 0, M, K), gen.uniform_bf16(2, 1, K, N))
+    for c in (c0, c1):
+        ok, worst = _within_tol(bits16(c), want, K)
+        assert ok, worst
+
+
+def test_2sm_ragged_edge_items_under_contention():
+    # M = N = K = 2064: the last row of pair tiles holds 16 rows, so on its
+    # items the second CTA of a pair loads nothing, and one column half lies
+    # wholly outside the matrix.  With other kernels sharing the SMs, its
+    # producer must still keep step with the leader's MMAs: every launch ends
+    # without a time-out and with the right product.
+    n = 2064
+    a, b = _gen(2064, n, n, n)
+    c = torch.empty(n, n, dtype=torch.bfloat16, device="cuda")
+    x = torch.empty(16384, 8192, dtype=torch.float32, device="cuda")
+    y = torch.empty_like(x)
+    krex.krex_gen_inputs(7, 0, krex.KREX_DIST_NORMAL, 2.0, x)
+    side = torch.cuda.Stream()
+    for _ in range(80):
+        krex.krex_run_candidate(krex.KREX_OP_SOFTMAX_F32, [x], y, stream=side)
+        krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [a, b], c)
+    torch.cuda.synchronize()
+    detail = krex.krex_device_status_detail()
+    try:
+        krex.krex_device_status()
+    except krex.KrexError as e:
+        pytest.fail(f"{e}: {detail}")
+    want = ref.gemm_f64(gen.uniform_bf16(2064, 0, n, n), gen.uniform_bf16(2064, 1, n, n))
+    ok, worst = _within_tol(bits16(c), want, n)
+    assert ok, worst
