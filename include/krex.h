@@ -286,8 +286,9 @@ krex_status krex_gate_submit_end(krex_gate *gate, int32_t tenant);
 /* Enter as holder (steps 1-3): take the region lock, claim the gate with a new
  * epoch (*epoch), then for every sibling wait for its in-flight counter to
  * reach zero, synchronise its stream and acknowledge the epoch.  Returns only
- * when every sibling acknowledged this epoch (its counter seen at zero with
- * the gate closed).  On TIMEOUT
+ * when every sibling shows this epoch's acknowledgement and a zero counter
+ * (polled: a submission bouncing off the closed gate raises a counter for a
+ * moment).  On TIMEOUT
  * or a CUDA error the gate is reopened and the lock released: a failing entry
  * never starts measurement.  STATE if the caller already holds the gate. */
 krex_status krex_gate_enter(krex_gate *gate, int32_t holder, int64_t timeout_us, uint64_t *epoch);

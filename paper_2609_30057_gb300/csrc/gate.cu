@@ -12,10 +12,10 @@
 //    or sees the closed gate (Dekker-style ordering).
 //  - Entry: lock, claim the gate (holder, epoch), then for each sibling wait
 //    for its counter to reach zero, synchronise its stream and record the
-//    epoch as acknowledged.  The holder proceeds only when every sibling has
-//    acknowledged this epoch; a previous epoch's acknowledgement never counts.
-//    (After the acknowledgement a sibling's counter may still rise for a
-//    moment: the increment of a submission that then sees the closed gate and
+//    epoch as acknowledged.  The holder then polls until every sibling shows
+//    this epoch's acknowledgement and a zero counter; a previous epoch's
+//    acknowledgement never counts.  (A counter may rise for a moment after the
+//    drain: the increment of a submission that then sees the closed gate and
 //    retracts.)  A drain that runs out of time releases the
 //    gate and the lock and fails the entry: measurement never starts.
 //  - Registration is serialised with gate closure: a tenant registering while
@@ -219,11 +219,11 @@ krex_status krex_gate_enter(krex_gate *g, int32_t holder, int64_t timeout_us, ui
         }
         x.acked_epoch.store(e, std::memory_order_seq_cst);
     }
-    // The holder proceeds only on acknowledgements of this epoch.  Each was
-    // recorded after that sibling's counter was seen at zero with the gate
-    // already closed; a non-zero counter seen now can only be the transient
-    // increment of a submission that will see the closed gate and retract, so
-    // the counters are not read again here.
+    // The holder polls until every sibling shows this epoch's acknowledgement
+    // and a zero counter.  A counter can rise for a moment after the drain:
+    // the increment of a submission that then sees the closed gate and
+    // retracts, so the counters are polled (within the entry deadline), not
+    // read once.
     for (int32_t t = 0; t < g->max_tenants; ++t) {
         Tenant &x = g->tenants[t];
         if (!x.registered || t == holder) continue;
@@ -232,6 +232,12 @@ krex_status krex_gate_enter(krex_gate *g, int32_t holder, int64_t timeout_us, ui
             wake_parked(g);
             g->region_locked.store(false, std::memory_order_seq_cst);
             return set_error(KREX_ERR_STATE, "gate_enter: tenant %d acknowledgement does not match epoch", t);
+        }
+        if (!spin_park([&] { return x.inflight.load(std::memory_order_seq_cst) == 0; }, deadline)) {
+            g->holder.store(-1, std::memory_order_seq_cst);
+            wake_parked(g);
+            g->region_locked.store(false, std::memory_order_seq_cst);
+            return set_error(KREX_ERR_TIMEOUT, "gate_enter: tenant %d counter stayed non-zero", t);
         }
     }
     *epoch = e;
