@@ -301,6 +301,70 @@ krex_status krex_gate_exit(krex_gate *gate, int32_t holder, uint64_t epoch);
 /* Current holder (-1 = open), last epoch, and number of parked submitters. */
 krex_status krex_gate_state(krex_gate *gate, int32_t *holder, uint64_t *epoch, int32_t *parked);
 
+/* ------------------------------------------- cross-process gate -------- */
+
+/* The same gate with its state in shared memory, so that tenants in several
+ * processes take part (Section 4.2: region lock, gate with holder and epoch,
+ * per-tenant in-flight counters, registration serialised with closure,
+ * drainer threads that acknowledge the epoch; Section 4.2 "Region entry and
+ * exit": a participant's death fails the entry, a dead holder's gate is
+ * reclaimed bound to holder and epoch).  Host-side only.
+ *
+ * `mem` is caller-owned shared memory (for example a POSIX shared-memory
+ * object or a file mapped MAP_SHARED by every participant), 64-byte aligned,
+ * of at least krex_gate_shared_bytes(max_tenants) bytes; it holds only
+ * address-free atomics, so each process may map it anywhere.  One process
+ * formats it with krex_gate_shared_init before any process attaches. */
+size_t krex_gate_shared_bytes(int32_t max_tenants);
+krex_status krex_gate_shared_init(void *mem, size_t bytes, int32_t max_tenants);
+
+/* Attach this process to a formatted gate.  The returned handle works with
+ * every krex_gate_* call above and as krex_region_opts.gate; tenants it
+ * registers belong to this process (their streams are drained by this
+ * process's drainer thread, started here).  krex_gate_destroy detaches: the
+ * drainer stops, this process's tenants finish their stream work and leave
+ * (STATE while one of them holds the gate); the shared memory is untouched.
+ * In this form: unregister is refused (STATE) while another tenant holds the
+ * gate, so drained entries stay until the region ends; registration and
+ * entry free the slots of tenants whose process no longer exists; an entry
+ * fails with STATE when a sibling's process dies while it is being drained,
+ * and with CUDA when a sibling's stream synchronisation fails. */
+krex_status krex_gate_shared_attach(void *mem, size_t bytes, krex_gate **gate);
+
+/* Reclaim a gate whose holder died inside (the dispatcher's recovery of
+ * Section 4.2): if `holder` still holds it with `epoch` and the holder's
+ * process no longer exists, free the holder's slot, reopen the gate and
+ * release the region lock.  Bound to holder and epoch, so a delayed recovery
+ * never reopens a later entry.  STATE if the holder is alive or the gate has
+ * moved on; INVALID for an in-process gate. */
+krex_status krex_gate_recover(krex_gate *gate, int32_t holder, uint64_t epoch);
+
+/* ------------------------------------------------ shared-memory ring ---- */
+
+/* Single-producer single-consumer ring in caller-owned shared memory, the
+ * transport between a client and its context process (Section 4.3, "minimal
+ * shared-memory transport": fixed-layout entries, one producer and one
+ * consumer per ring; a request/reply pair is two rings).  Waiting follows the
+ * spin-park policy of Section 4.3: a side that finds the ring empty (pop) or
+ * full (push) spins for the ring's spin interval (default 20 us), then parks
+ * on a futex until the other side's wake or the timeout; the other side
+ * issues a wake only when a peer has announced that it parks.
+ * `mem`: 64-byte aligned, krex_ring_bytes(capacity, entry_bytes) bytes;
+ * capacity a power of two in [2, 2^24], entry_bytes a multiple of 8 in
+ * [8, 4096].  Timeouts in microseconds (<= 0: 10 s); TIMEOUT when the ring
+ * stayed full / empty.  At most one thread (in any process) pushes and one
+ * pops. */
+size_t krex_ring_bytes(uint32_t capacity, uint32_t entry_bytes);
+krex_status krex_ring_init(void *mem, size_t bytes, uint32_t capacity, uint32_t entry_bytes);
+krex_status krex_ring_push(void *ring, const void *entry, int64_t timeout_us);
+krex_status krex_ring_pop(void *ring, void *entry, int64_t timeout_us);
+/* Entries currently queued. */
+krex_status krex_ring_count(void *ring, uint64_t *n);
+/* The spinning interval of the spin-park policy (0: park at once). */
+krex_status krex_ring_set_spin(void *ring, int64_t spin_us);
+/* Counters: pushes, pops, consumer parks, producer parks, wakes sent. */
+krex_status krex_ring_stats(void *ring, uint64_t *out5);
+
 /* ------------------------------------------------ timing loop (native) --- */
 
 /* The whole timed loop of a benchmarking command in native code: region

@@ -100,6 +100,17 @@ SIGNATURES = {
     "krex_last_error_string": (ctypes.c_char_p, []),
     "krex_version": (_i32, []),
     "krex_debug_hold_stream": (_i32, [_vp, _P(_i32), _i32]),
+    "krex_gate_shared_bytes": (_sz, [_i32]),
+    "krex_gate_shared_init": (_i32, [_vp, _sz, _i32]),
+    "krex_gate_shared_attach": (_i32, [_vp, _sz, _P(_vp)]),
+    "krex_gate_recover": (_i32, [_vp, _i32, _u64]),
+    "krex_ring_bytes": (_sz, [_u32, _u32]),
+    "krex_ring_init": (_i32, [_vp, _sz, _u32, _u32]),
+    "krex_ring_push": (_i32, [_vp, _vp, _i64]),
+    "krex_ring_pop": (_i32, [_vp, _vp, _i64]),
+    "krex_ring_count": (_i32, [_vp, _P(_u64)]),
+    "krex_ring_set_spin": (_i32, [_vp, _i64]),
+    "krex_ring_stats": (_i32, [_vp, _P(_u64)]),
     "krex_gate_create": (_i32, [_P(_vp), _i32]),
     "krex_gate_destroy": (_i32, [_vp]),
     "krex_gate_register": (_i32, [_vp, _vp, _i64, _P(_i32)]),
@@ -414,14 +425,28 @@ def krex_debug_hold_stream(gate, hold_ms: int, stream=None):
 # ------------------------------------------------------------------ gate --
 
 class Gate:
-    """The in-region gate (paper Section 4.2, in-process form): tenants bracket
-    submissions with ``submission(t)``; a holder's ``enter``/``exit`` (or a
-    ``region(..., gate=g, tenant=t)``) blocks and drains sibling tenants."""
+    """The in-region gate (paper Section 4.2): tenants bracket submissions
+    with ``submission(t)``; a holder's ``enter``/``exit`` (or a
+    ``region(..., gate=g, tenant=t)``) blocks and drains sibling tenants.
+    ``Gate(n)`` is the in-process form; ``Gate.attach(addr, nbytes)`` joins a
+    gate formatted in shared memory by ``gate_shared_init`` (cross-process)."""
 
-    def __init__(self, max_tenants: int = 64):
+    def __init__(self, max_tenants: int = 64, _handle=None):
+        if _handle is not None:
+            self.handle = _handle
+            return
         h = _vp()
         _ok(lib().krex_gate_create(ctypes.byref(h), max_tenants), "krex_gate_create")
         self.handle = h.value
+
+    @classmethod
+    def attach(cls, addr: int, nbytes: int) -> "Gate":
+        h = _vp()
+        _ok(lib().krex_gate_shared_attach(addr, nbytes, ctypes.byref(h)), "krex_gate_shared_attach")
+        return cls(_handle=h.value)
+
+    def recover(self, holder: int, epoch: int):
+        _ok(lib().krex_gate_recover(self.handle, holder, epoch), "krex_gate_recover")
 
     def close(self):
         if self.handle:
@@ -463,3 +488,74 @@ class Gate:
         h, e, p = _i32(0), _u64(0), _i32(0)
         _ok(lib().krex_gate_state(self.handle, ctypes.byref(h), ctypes.byref(e), ctypes.byref(p)), "krex_gate_state")
         return h.value, e.value, p.value
+
+
+def gate_shared_bytes(max_tenants: int) -> int:
+    return int(lib().krex_gate_shared_bytes(max_tenants))
+
+
+def gate_shared_init(addr: int, nbytes: int, max_tenants: int):
+    _ok(lib().krex_gate_shared_init(addr, nbytes, max_tenants), "krex_gate_shared_init")
+
+
+class Ring:
+    """View of a single-producer single-consumer ring in shared memory
+    (paper Section 4.3); ``Ring.init`` formats the memory first."""
+
+    def __init__(self, addr: int):
+        self.addr = addr
+        n = _u64(0)
+        _ok(lib().krex_ring_count(addr, ctypes.byref(n)), "krex_ring_count")  # validates the header
+
+    @staticmethod
+    def nbytes(capacity: int, entry_bytes: int) -> int:
+        return int(lib().krex_ring_bytes(capacity, entry_bytes))
+
+    @classmethod
+    def init(cls, addr: int, nbytes: int, capacity: int, entry_bytes: int) -> "Ring":
+        _ok(lib().krex_ring_init(addr, nbytes, capacity, entry_bytes), "krex_ring_init")
+        return cls(addr)
+
+    def push(self, entry, timeout_us: int = 0):
+        """entry: a ctypes object or a bytes-like object of the ring's entry size."""
+        if isinstance(entry, (bytes, bytearray, memoryview)):
+            entry = ctypes.create_string_buffer(bytes(entry), len(entry))
+        _ok(lib().krex_ring_push(self.addr, ctypes.byref(entry), timeout_us), "krex_ring_push")
+
+    def pop_into(self, entry, timeout_us: int = 0):
+        _ok(lib().krex_ring_pop(self.addr, ctypes.byref(entry), timeout_us), "krex_ring_pop")
+        return entry
+
+    def count(self) -> int:
+        n = _u64(0)
+        _ok(lib().krex_ring_count(self.addr, ctypes.byref(n)), "krex_ring_count")
+        return n.value
+
+    def set_spin(self, spin_us: int):
+        _ok(lib().krex_ring_set_spin(self.addr, spin_us), "krex_ring_set_spin")
+
+    def stats(self) -> dict:
+        o = (_u64 * 5)()
+        _ok(lib().krex_ring_stats(self.addr, o), "krex_ring_stats")
+        return dict(zip(("pushes", "pops", "consumer_parks", "producer_parks", "wakes"), list(o)))
+
+
+class SharedMap:
+    """A file mapped MAP_SHARED (e.g. under /dev/shm): memory every process can
+    map for a shared gate or ring.  ``addr`` is this process's address of it."""
+
+    def __init__(self, path: str, nbytes: int, create: bool = False):
+        import mmap
+        import os
+        self.path, self.nbytes = path, nbytes
+        flags = os.O_RDWR | (os.O_CREAT if create else 0)
+        fd = os.open(path, flags, 0o600)
+        try:
+            if create:
+                os.ftruncate(fd, nbytes)
+            self.mm = mmap.mmap(fd, nbytes, mmap.MAP_SHARED, mmap.PROT_READ | mmap.PROT_WRITE)
+        finally:
+            os.close(fd)
+        self._anchor = ctypes.c_char.from_buffer(self.mm)
+        self.addr = ctypes.addressof(self._anchor)
+

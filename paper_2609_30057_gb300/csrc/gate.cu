@@ -35,6 +35,7 @@
 #include <vector>
 
 #include "common.cuh"
+#include "xproc.h"
 
 namespace {
 
@@ -50,6 +51,7 @@ struct Tenant {
 }  // namespace
 
 struct krex_gate {
+    krex::XGate *x = nullptr;             // non-null: the gate lives in shared memory (xproc.cu)
     int32_t max_tenants = 0;
     std::unique_ptr<Tenant[]> tenants;
     std::atomic<int32_t> holder{-1};      // -1: gate open
@@ -111,6 +113,11 @@ krex_status krex_gate_create(krex_gate **g, int32_t max_tenants) {
 
 krex_status krex_gate_destroy(krex_gate *g) {
     if (!g) return set_error(KREX_ERR_INVALID, "gate is null");
+    if (g->x) {
+        krex_status st = krex::xgate_detach(g->x);
+        if (st == KREX_OK) delete g;
+        return st;
+    }
     if (g->holder.load() != -1) return set_error(KREX_ERR_STATE, "gate_destroy while a holder is inside");
     delete g;
     return KREX_OK;
@@ -118,6 +125,7 @@ krex_status krex_gate_destroy(krex_gate *g) {
 
 krex_status krex_gate_register(krex_gate *g, krex_stream_t stream, int64_t timeout_us, int32_t *tenant) {
     if (!g || !tenant) return set_error(KREX_ERR_INVALID, "gate_register: null argument");
+    if (g->x) return krex::xgate_register(g->x, stream, timeout_us, tenant);
     const auto deadline = deadline_from(timeout_us);
     for (;;) {
         {
@@ -143,6 +151,7 @@ krex_status krex_gate_register(krex_gate *g, krex_stream_t stream, int64_t timeo
 }
 
 krex_status krex_gate_unregister(krex_gate *g, int32_t tenant) {
+    if (g && g->x) return krex::xgate_unregister(g->x, tenant);
     if (!valid_tenant(g, tenant)) return set_error(KREX_ERR_INVALID, "gate_unregister: bad tenant");
     std::lock_guard<std::mutex> lk(g->reg_mu);
     if (g->holder.load() == tenant) return set_error(KREX_ERR_STATE, "gate_unregister: tenant holds the gate");
@@ -152,6 +161,7 @@ krex_status krex_gate_unregister(krex_gate *g, int32_t tenant) {
 }
 
 krex_status krex_gate_submit_begin(krex_gate *g, int32_t tenant, int64_t timeout_us) {
+    if (g && g->x) return krex::xgate_submit_begin(g->x, tenant, timeout_us);
     if (!valid_tenant(g, tenant)) return set_error(KREX_ERR_INVALID, "gate_submit_begin: bad tenant");
     Tenant &x = g->tenants[tenant];
     const auto deadline = deadline_from(timeout_us);
@@ -175,6 +185,7 @@ krex_status krex_gate_submit_begin(krex_gate *g, int32_t tenant, int64_t timeout
 }
 
 krex_status krex_gate_submit_end(krex_gate *g, int32_t tenant) {
+    if (g && g->x) return krex::xgate_submit_end(g->x, tenant);
     if (!valid_tenant(g, tenant)) return set_error(KREX_ERR_INVALID, "gate_submit_end: bad tenant");
     Tenant &x = g->tenants[tenant];
     if (x.inflight.fetch_sub(1, std::memory_order_seq_cst) <= 0) {
@@ -185,6 +196,7 @@ krex_status krex_gate_submit_end(krex_gate *g, int32_t tenant) {
 }
 
 krex_status krex_gate_enter(krex_gate *g, int32_t holder, int64_t timeout_us, uint64_t *epoch) {
+    if (g && g->x) return krex::xgate_enter(g->x, holder, timeout_us, epoch);
     if (!valid_tenant(g, holder) || !epoch) return set_error(KREX_ERR_INVALID, "gate_enter: bad holder or epoch");
     if (g->holder.load() == holder) return set_error(KREX_ERR_STATE, "gate_enter: already holding the gate");
     const auto deadline = deadline_from(timeout_us);
@@ -245,6 +257,7 @@ krex_status krex_gate_enter(krex_gate *g, int32_t holder, int64_t timeout_us, ui
 }
 
 krex_status krex_gate_exit(krex_gate *g, int32_t holder, uint64_t epoch) {
+    if (g && g->x) return krex::xgate_exit(g->x, holder, epoch);
     if (!valid_tenant(g, holder)) return set_error(KREX_ERR_INVALID, "gate_exit: bad holder");
     if (g->holder.load() != holder || g->epoch.load() != epoch)
         return set_error(KREX_ERR_STATE, "gate_exit: not the holder of epoch %llu", (unsigned long long)epoch);
@@ -259,10 +272,27 @@ krex_status krex_gate_exit(krex_gate *g, int32_t holder, uint64_t epoch) {
 
 krex_status krex_gate_state(krex_gate *g, int32_t *holder, uint64_t *epoch, int32_t *parked) {
     if (!g) return set_error(KREX_ERR_INVALID, "gate is null");
+    if (g->x) return krex::xgate_state(g->x, holder, epoch, parked);
     if (holder) *holder = g->holder.load();
     if (epoch) *epoch = g->epoch.load();
     if (parked) *parked = g->parked.load();
     return KREX_OK;
+}
+
+krex_status krex_gate_shared_attach(void *mem, size_t bytes, krex_gate **g) {
+    if (!g) return set_error(KREX_ERR_INVALID, "gate_shared_attach: null out");
+    krex::XGate *x = nullptr;
+    krex_status st = krex::xgate_attach(mem, bytes, &x);
+    if (st) return st;
+    krex_gate *h = new krex_gate();
+    h->x = x;
+    *g = h;
+    return KREX_OK;
+}
+
+krex_status krex_gate_recover(krex_gate *g, int32_t holder, uint64_t epoch) {
+    if (!g || !g->x) return set_error(KREX_ERR_INVALID, "gate_recover: needs a shared gate");
+    return krex::xgate_recover(g->x, holder, epoch);
 }
 
 }  // extern "C"
