@@ -18,7 +18,10 @@ of ratios within 5 %, the pairwise ordering-flip rate grouped by native gap
 (pairs whose durations differ by less than 2 %, 2–10 %, more than 10 %), and
 Kendall's τ_b between measured and native rankings.
 
-    python -m paper_2609_30057_gb300.fidelity [--tenants 2] [--iters 20] [--json out.json]
+    python -m paper_2609_30057_gb300.fidelity [--tenants 2] [--iters 20] [--processes] [--json out.json]
+
+With ``--processes`` the background tenants run in their own processes (own
+CUDA contexts) and the gate lives in shared memory (``run_xproc``).
 """
 from __future__ import annotations
 
@@ -132,15 +135,26 @@ def candidates(device="cuda", quick: bool = False):
     return cands
 
 
-def time_candidates(cands, flush, iters, stream, gate=None, tenant=0):
+def time_candidates(cands, flush, iters, stream, gate=None, tenant=0, per_iter=None):
     """Median of `iters` flushed, timed iterations of each candidate (the
-    command's timed loop), optionally inside a gated region."""
+    command's timed loop), optionally inside a gated region.  `per_iter`, if
+    a list, receives every candidate's iteration durations."""
     out = []
     for name, op, ins, o in cands:
-        _, p50, _ = krex_bench_candidate(op, ins, o, warmup=3, iters=iters, flush_scratch=flush,
+        d, p50, _ = krex_bench_candidate(op, ins, o, warmup=3, iters=iters, flush_scratch=flush,
                                          flush_bytes=flush.numel(), stream=stream, gate=gate, tenant=tenant)
         out.append(p50)
+        if per_iter is not None:
+            per_iter.append(list(d))
     return out
+
+
+def iteration_stats(per_iter, native) -> dict:
+    """Interference seen by single iterations rather than by medians: every
+    iteration's duration over its candidate's native median."""
+    r = [x / n for d, n in zip(per_iter, native) for x in d]
+    return {"iter_p95_inflation": percentile(r, 0.95) - 1.0, "iter_max_ratio": max(r),
+            "iter_share_over_1_5x": sum(x > 1.5 for x in r) / len(r)}
 
 
 # ------------------------------------------------------------- background --
@@ -214,18 +228,19 @@ def run(tenants: int = 2, iters: int = 20, quick: bool = False) -> dict:
     cands = candidates(quick=quick)
     names = [c[0] for c in cands]
     status, details = {}, {}
+    it = {k: [] for k in ("repeat", "ungated", "gated")}
     time_candidates(cands, flush, 3, stream)                       # warm everything up
     native = time_candidates(cands, flush, iters, stream)
-    repeat = time_candidates(cands, flush, iters, stream)
+    repeat = time_candidates(cands, flush, iters, stream, per_iter=it["repeat"])
     status["native"] = _device_status(details, "native")
     with Background(tenants, None) as bg:
-        ungated = time_candidates(cands, flush, iters, stream)
+        ungated = time_candidates(cands, flush, iters, stream, per_iter=it["ungated"])
         ungated_bg = sum(bg.launched)
     status["ungated"] = _device_status(details, "ungated")
     gate = Gate(16)
     holder = gate.register(stream)
     with Background(tenants, gate) as bg:
-        gated = time_candidates(cands, flush, iters, stream, gate=gate, tenant=holder)
+        gated = time_candidates(cands, flush, iters, stream, gate=gate, tenant=holder, per_iter=it["gated"])
         gated_bg = sum(bg.launched)
     gate.unregister(holder)
     gate.close()
@@ -233,11 +248,131 @@ def run(tenants: int = 2, iters: int = 20, quick: bool = False) -> dict:
     return {
         "device_status": status, "device_status_detail": details,
         "candidates": names, "native_ms": native,
-        "conditions": {"repeat": {"ms": repeat, **summarize(repeat, native)},
-                       "ungated": {"ms": ungated, "background_launches": ungated_bg, **summarize(ungated, native)},
-                       "gated": {"ms": gated, "background_launches": gated_bg, **summarize(gated, native)}},
+        "conditions": {"repeat": {"ms": repeat, **summarize(repeat, native), **iteration_stats(it["repeat"], native)},
+                       "ungated": {"ms": ungated, "background_launches": ungated_bg, **summarize(ungated, native),
+                                   **iteration_stats(it["ungated"], native)},
+                       "gated": {"ms": gated, "background_launches": gated_bg, **summarize(gated, native),
+                                 **iteration_stats(it["gated"], native)}},
         "tenants": tenants, "iters": iters,
     }
+
+
+# ------------------------------------------------- tenants in processes --
+
+# control words (int64) after the shared gate: stop, pause, then per tenant
+# ready, launches, device status
+_X_STOP, _X_PAUSE, _X_BASE = 0, 1, 2
+
+
+def _xproc_tenant(path: str, nbytes: int, gate_bytes: int, idx: int):
+    """A tenant in its own process (own CUDA context): attaches to the shared
+    gate and keeps launching a 4096^3 GEMM and a 16384x8192 softmax on its
+    stream, each submission bracketed by the gate, until told to stop."""
+    import ctypes
+    import torch
+    from . import SharedMap
+    m = SharedMap(path, nbytes)
+    ctl = (ctypes.c_int64 * 32).from_address(m.addr + gate_bytes)
+    torch.cuda.set_device(0)
+    build()
+    g = Gate.attach(m.addr, gate_bytes)
+    s = torch.cuda.Stream()
+    a = torch.empty(4096, 4096, dtype=torch.bfloat16, device="cuda")
+    b, c = torch.empty_like(a), torch.empty_like(a)
+    x = torch.empty(16384, 8192, dtype=torch.float32, device="cuda")
+    y = torch.empty_like(x)
+    krex_gen_inputs(100 + idx, 0, 0, 0.0, a, stream=s)
+    krex_gen_inputs(100 + idx, 1, 0, 0.0, b, stream=s)
+    krex_gen_inputs(100 + idx, 2, 1, 2.0, x, stream=s)
+    s.synchronize()
+    t = g.register(s)
+    base = _X_BASE + 3 * idx
+    ctl[base] = 1
+    launched = 0
+    while not ctl[_X_STOP]:
+        if ctl[_X_PAUSE]:
+            s.synchronize()
+            time.sleep(0.002)
+            continue
+        g.submit_begin(t, timeout_us=60_000_000)
+        try:
+            krex_run_candidate(KREX_OP_GEMM_BF16, [a, b], c, stream=s)
+            krex_run_candidate(KREX_OP_SOFTMAX_F32, [x], y, stream=s)
+        finally:
+            g.submit_end(t)
+        launched += 2
+        if s.query() is False:
+            s.synchronize()
+    s.synchronize()
+    ctl[base + 1] = launched
+    ctl[base + 2] = _device_status()
+    g.unregister(t)
+    g.close()
+
+
+def run_xproc(tenants: int = 2, iters: int = 20, quick: bool = False, shm_dir: str = "/dev/shm") -> dict:
+    """The fidelity experiment with the background tenants in other processes
+    (each its own CUDA context, as the paper's tenants are) and the gate in
+    shared memory: native, repeat, ungated, gated."""
+    import ctypes
+    import multiprocessing as mp
+    import os
+    import torch
+    from . import SharedMap, gate_shared_bytes, gate_shared_init
+    build()
+    torch.cuda.set_device(0)
+    gate_bytes = (gate_shared_bytes(16) + 63) // 64 * 64
+    nbytes = gate_bytes + 32 * 8
+    path = os.path.join(shm_dir if os.path.isdir(shm_dir) else "/tmp", f"krex_fid_{os.getpid()}_{time.monotonic_ns()}")
+    m = SharedMap(path, nbytes, create=True)
+    try:
+        gate_shared_init(m.addr, gate_bytes, 16)
+        ctl = (ctypes.c_int64 * 32).from_address(m.addr + gate_bytes)
+        ctl[_X_PAUSE] = 1
+        procs = [mp.get_context("spawn").Process(target=_xproc_tenant, args=(path, nbytes, gate_bytes, i), daemon=True)
+                 for i in range(tenants)]
+        for p in procs:
+            p.start()
+        stream = torch.cuda.Stream()
+        flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+        cands = candidates(quick=quick)
+        t0 = time.monotonic()
+        while not all(ctl[_X_BASE + 3 * i] for i in range(tenants)):
+            if time.monotonic() - t0 > 120 or any(p.exitcode not in (None, 0) for p in procs):
+                raise RuntimeError("tenant processes did not start")
+            time.sleep(0.05)
+        status, details = {}, {}
+        it = {k: [] for k in ("repeat", "ungated", "gated")}
+        time_candidates(cands, flush, 3, stream)
+        native = time_candidates(cands, flush, iters, stream)
+        repeat = time_candidates(cands, flush, iters, stream, per_iter=it["repeat"])
+        status["native"] = _device_status(details, "native")
+        ctl[_X_PAUSE] = 0
+        time.sleep(0.5)
+        ungated = time_candidates(cands, flush, iters, stream, per_iter=it["ungated"])
+        status["ungated"] = _device_status(details, "ungated")
+        g = Gate.attach(m.addr, gate_bytes)
+        holder = g.register(stream)
+        gated = time_candidates(cands, flush, iters, stream, gate=g, tenant=holder, per_iter=it["gated"])
+        status["gated"] = _device_status(details, "gated")
+        ctl[_X_STOP] = 1
+        for p in procs:
+            p.join(120)
+        g.unregister(holder)
+        g.close()
+        tenant_launches = [int(ctl[_X_BASE + 3 * i + 1]) for i in range(tenants)]
+        tenant_status = [int(ctl[_X_BASE + 3 * i + 2]) for i in range(tenants)]
+        return {
+            "device_status": status, "device_status_detail": details,
+            "tenant_exitcodes": [p.exitcode for p in procs], "tenant_launches": tenant_launches,
+            "tenant_device_status": tenant_status,
+            "candidates": [c[0] for c in cands], "native_ms": native,
+            "conditions": {k: {"ms": v, **summarize(v, native), **iteration_stats(it[k], native)}
+                           for k, v in (("repeat", repeat), ("ungated", ungated), ("gated", gated))},
+            "tenants": tenants, "iters": iters, "tenant_form": "processes",
+        }
+    finally:
+        os.unlink(path)
 
 
 def main():
@@ -245,8 +380,9 @@ def main():
     ap.add_argument("--tenants", type=int, default=2)
     ap.add_argument("--iters", type=int, default=20)
     ap.add_argument("--json", default=None)
+    ap.add_argument("--processes", action="store_true", help="tenants in their own processes, gate in shared memory")
     args = ap.parse_args()
-    res = run(args.tenants, args.iters)
+    res = run_xproc(args.tenants, args.iters) if args.processes else run(args.tenants, args.iters)
     text = json.dumps(res, indent=1)
     if args.json:
         with open(args.json, "w") as f:

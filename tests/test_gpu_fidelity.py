@@ -19,3 +19,18 @@ def test_gate_restores_native_timings():
     assert 0.95 < c["gated"]["median_ratio"] < 1.05     # gated: as if alone
     assert c["gated"]["P_p95_inflation"] < 0.10
     assert c["gated"]["P_p95_inflation"] < c["ungated"]["P_p95_inflation"]
+
+
+def test_gate_across_processes_restores_native_timings():
+    # tenants in their own processes (own CUDA contexts, time-sliced with the
+    # measuring one), gate in shared memory, drained by their drainer threads.
+    # Time slicing hits whole iterations rather than every iteration, so the
+    # iteration-level figures carry the signal.
+    res = fidelity.run_xproc(tenants=2, iters=20, quick=False)
+    assert res["device_status"] == {"native": 0, "ungated": 0, "gated": 0}, json.dumps(res["device_status_detail"])
+    assert res["tenant_exitcodes"] == [0, 0] and res["tenant_device_status"] == [0, 0]
+    assert all(n > 0 for n in res["tenant_launches"])
+    c = res["conditions"]
+    assert c["ungated"]["iter_max_ratio"] > 2.0 and c["ungated"]["iter_share_over_1_5x"] > 0.005
+    assert c["gated"]["iter_share_over_1_5x"] == 0.0 and c["gated"]["iter_max_ratio"] < 1.5
+    assert 0.95 < c["gated"]["median_ratio"] < 1.05
