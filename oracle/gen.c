@@ -12,6 +12,7 @@
  * and N(0, 4) via Box-Muller in fp32 for the softmax input.  Where that
  * definition is silent this code takes these readings: each tensor has its own
  * stream key; one 64-bit draw feeds an element pair (bits 63..40 and 31..8);
+ * fp16 GEMM operands take the same 24-bit values rounded RNE to IEEE binary16;
  * "N(0, 4)" means variance 4 (sigma = 2); Box-Muller's ln and sincos are the
  * fp32 series routines below, evaluated operation by operation.
  *
@@ -84,6 +85,61 @@ uint16_t oracle_uniform_bf16_at(uint64_t key, uint64_t e)
     uint32_t b = (e & 1u) ? (uint32_t)((z >> 8) & 0xFFFFFFu) : (uint32_t)(z >> 40);
     float x = (float)((int32_t)b - (int32_t)(1 << 23)) * 0x1p-23f;
     return oracle_f32_to_bf16_rne(x);
+}
+
+/* ------------------------------------------------------------ fp16 ------- */
+
+/* IEEE binary16 round-to-nearest-even from fp32, subnormals included.  With
+ * x = m 2^(e-23) (m the 24-bit significand), a normal binary16 keeps 11
+ * significant bits, quantum 2^(e-10), for e >= -14; below, the quantum is the
+ * subnormal step 2^-24.  Magnitudes past the largest binary16 give infinity;
+ * NaN stays NaN (quiet). */
+uint16_t oracle_f32_to_f16_rne(float x)
+{
+    uint32_t u = f32_bits(x);
+    uint16_t sign = (uint16_t)((u >> 16) & 0x8000u);
+    uint32_t a = u & 0x7FFFFFFFu;
+    if (a >= 0x7F800000u) return (uint16_t)(sign | 0x7C00u | (a > 0x7F800000u ? 0x200u : 0u));
+    int32_t e;
+    uint32_t m;
+    if (a >= 0x00800000u) {
+        e = (int32_t)(a >> 23) - 127;
+        m = (a & 0x7FFFFFu) | 0x800000u;
+    } else {
+        e = -126;
+        m = a;
+    }
+    int32_t shift = (e >= -14) ? 13 : (-1 - e);
+    if (shift > 24) return sign;  /* below half the smallest subnormal */
+    uint32_t q = m >> shift;
+    uint32_t rem = m & ((1u << shift) - 1u);
+    uint32_t half = 1u << (shift - 1);
+    if (rem > half || (rem == half && (q & 1u))) q += 1u;
+    if (e >= -14) {
+        int32_t E = e + 15;
+        if (q == 0x800u) {  /* rounding carried into the next binade */
+            q = 0x400u;
+            E += 1;
+        }
+        if (E >= 31) return (uint16_t)(sign | 0x7C00u);
+        return (uint16_t)(sign | (uint32_t)(E << 10) | (q & 0x3FFu));
+    }
+    return (uint16_t)(sign | q);  /* q == 0x400 is the smallest normal: same encoding */
+}
+
+/* Element e of a uniform fp16 tensor: the same 24-bit value as the bf16 form,
+ * x = (b - 2^23) 2^-23 exact in fp32, rounded RNE to binary16. */
+uint16_t oracle_uniform_f16_at(uint64_t key, uint64_t e)
+{
+    uint64_t z = oracle_draw(key, e >> 1);
+    uint32_t b = (e & 1u) ? (uint32_t)((z >> 8) & 0xFFFFFFu) : (uint32_t)(z >> 40);
+    float x = (float)((int32_t)b - (int32_t)(1 << 23)) * 0x1p-23f;
+    return oracle_f32_to_f16_rne(x);
+}
+
+void oracle_f32_to_f16_many(const float *x, int64_t n, uint16_t *out)
+{
+    for (int64_t i = 0; i < n; ++i) out[i] = oracle_f32_to_f16_rne(x[i]);
 }
 
 /* ------------------------------------------------ fp32 ln and sincos ----- */
@@ -231,6 +287,15 @@ void oracle_fill_uniform_bf16(uint64_t seed, uint32_t tensor_id, int64_t rows,
             out[r * ld + c] = oracle_uniform_bf16_at(key, (uint64_t)(r * cols + c));
 }
 
+void oracle_fill_uniform_f16(uint64_t seed, uint32_t tensor_id, int64_t rows,
+                             int64_t cols, int64_t ld, uint16_t *out)
+{
+    uint64_t key = oracle_stream_key(seed, tensor_id);
+    for (int64_t r = 0; r < rows; ++r)
+        for (int64_t c = 0; c < cols; ++c)
+            out[r * ld + c] = oracle_uniform_f16_at(key, (uint64_t)(r * cols + c));
+}
+
 void oracle_fill_normal_f32(uint64_t seed, uint32_t tensor_id, float sigma,
                             int64_t rows, int64_t cols, int64_t ld, float *out)
 {
@@ -246,6 +311,13 @@ void oracle_gather_uniform_bf16(uint64_t seed, uint32_t tensor_id,
 {
     uint64_t key = oracle_stream_key(seed, tensor_id);
     for (int64_t i = 0; i < n; ++i) out[i] = oracle_uniform_bf16_at(key, (uint64_t)idx[i]);
+}
+
+void oracle_gather_uniform_f16(uint64_t seed, uint32_t tensor_id,
+                               const int64_t *idx, int64_t n, uint16_t *out)
+{
+    uint64_t key = oracle_stream_key(seed, tensor_id);
+    for (int64_t i = 0; i < n; ++i) out[i] = oracle_uniform_f16_at(key, (uint64_t)idx[i]);
 }
 
 void oracle_gather_normal_f32(uint64_t seed, uint32_t tensor_id, float sigma,

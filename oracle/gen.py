@@ -11,7 +11,7 @@ generates seeded inputs, Section 2.1):
 * ``key(seed, t)   = mix64(seed + (t+1)·γ)`` — one stream per tensor id t
 * ``draw(key, j)   = mix64(key + (j+1)·γ)`` — SplitMix64's j-th output
 * uniform element e: draw e>>1, bits 63..40 (e even) or 31..8 (e odd),
-  ``x = (b − 2²³)·2⁻²³``, bf16 = RNE(x)
+  ``x = (b − 2²³)·2⁻²³``, bf16 = RNE(x) (binary16 = RNE(x) for fp16 operands)
 * normal pair j: ``u1 = (hi24+1)·2⁻²⁴``, ``u2 = lo24·2⁻²⁴``,
   ``y = σ·(sqrt(−2 ln u1)·(cos, sin)(2π u2))``
 """
@@ -62,6 +62,10 @@ def _load():
             "oracle_ln_u1": (f32, [u32]),
             "oracle_coefficients": (None, [vp]),
             "oracle_fill_uniform_bf16": (None, [u64, u32, i64, i64, i64, vp]),
+            "oracle_fill_uniform_f16": (None, [u64, u32, i64, i64, i64, vp]),
+            "oracle_gather_uniform_f16": (None, [u64, u32, vp, i64, vp]),
+            "oracle_uniform_f16_at": (ctypes.c_uint16, [u64, u64]),
+            "oracle_f32_to_f16_many": (None, [vp, i64, vp]),
             "oracle_fill_normal_f32": (None, [u64, u32, f32, i64, i64, i64, vp]),
             "oracle_gather_uniform_bf16": (None, [u64, u32, vp, i64, vp]),
             "oracle_gather_normal_f32": (None, [u64, u32, f32, vp, i64, vp]),
@@ -112,6 +116,31 @@ def uniform_bf16(seed: int, tensor_id: int, rows: int, cols: int) -> np.ndarray:
     return out
 
 
+def uniform_f16(seed: int, tensor_id: int, rows: int, cols: int) -> np.ndarray:
+    """Row-major rows×cols binary16 tensor as uint16 bit patterns (the same
+    24-bit values as uniform_bf16, rounded to binary16)."""
+    out = np.empty((rows, cols), dtype=np.uint16)
+    if out.size:
+        _load().oracle_fill_uniform_f16(seed & MASK64, tensor_id, rows, cols, cols, _ptr(out))
+    return out
+
+
+def uniform_f16_at(seed: int, tensor_id: int, idx) -> np.ndarray:
+    idx = np.ascontiguousarray(np.asarray(idx, dtype=np.int64).ravel())
+    out = np.empty(idx.size, dtype=np.uint16)
+    if idx.size:
+        _load().oracle_gather_uniform_f16(seed & MASK64, tensor_id, _ptr(idx), idx.size, _ptr(out))
+    return out
+
+
+def uniform_at(dtype: str, seed: int, tensor_id: int, idx) -> np.ndarray:
+    return (uniform_f16_at if dtype == "f16" else uniform_bf16_at)(seed, tensor_id, idx)
+
+
+def uniform(dtype: str, seed: int, tensor_id: int, rows: int, cols: int) -> np.ndarray:
+    return (uniform_f16 if dtype == "f16" else uniform_bf16)(seed, tensor_id, rows, cols)
+
+
 def normal_f32(seed: int, tensor_id: int, rows: int, cols: int, sigma: float = 2.0) -> np.ndarray:
     out = np.empty((rows, cols), dtype=np.float32)
     if out.size:
@@ -138,6 +167,25 @@ def normal_f32_at(seed: int, tensor_id: int, idx, sigma: float = 2.0) -> np.ndar
 def bf16_to_f32(h: np.ndarray) -> np.ndarray:
     """Exact widening of bf16 bit patterns (uint16) to fp32."""
     return (np.asarray(h, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def f16_to_f32(h: np.ndarray) -> np.ndarray:
+    """Exact widening of binary16 bit patterns (uint16) to fp32."""
+    return np.asarray(h, dtype=np.uint16).view(np.float16).astype(np.float32)
+
+
+def f32_to_f16(x: np.ndarray) -> np.ndarray:
+    """RNE narrowing fp32 → binary16 bit patterns (gen.c's routine)."""
+    x = np.ascontiguousarray(np.asarray(x, dtype=np.float32).ravel())
+    out = np.empty(x.size, dtype=np.uint16)
+    if x.size:
+        _load().oracle_f32_to_f16_many(_ptr(x), x.size, _ptr(out))
+    return out
+
+
+def widen(dtype: str, h: np.ndarray) -> np.ndarray:
+    """Exact fp32 values of 16-bit patterns of `dtype` ("bf16" or "f16")."""
+    return f16_to_f32(h) if dtype == "f16" else bf16_to_f32(h)
 
 
 def f32_to_bf16(x: np.ndarray) -> np.ndarray:

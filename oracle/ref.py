@@ -15,32 +15,36 @@ from . import gen
 
 # ------------------------------------------------------------------ GEMM ----
 
-def gemm_f64(a_bf16: np.ndarray, b_bf16: np.ndarray) -> np.ndarray:
-    """C = A·B in fp64 from bf16 operands (bit patterns).
+def gemm_f64(a_bits: np.ndarray, b_bits: np.ndarray, dtype: str = "bf16") -> np.ndarray:
+    """C = A·B in fp64 from 16-bit operands (bit patterns of `dtype`, "bf16"
+    or "f16").
 
     The candidate of the paper's GEMM benchmarking command (Section 2.1,
     Figure 1a) computes C[i,j] = Σ_k A[i,k]·B[k,j]; a single fp64 matmul is
-    that sum (each bf16 product is exact in fp64; only the additions round).
+    that sum (each 16-bit product is exact in fp64; only the additions round).
     """
-    a = gen.bf16_to_f32(a_bf16).astype(np.float64)
-    b = gen.bf16_to_f32(b_bf16).astype(np.float64)
+    a = gen.widen(dtype, a_bits).astype(np.float64)
+    b = gen.widen(dtype, b_bits).astype(np.float64)
     return a @ b
 
 
-def gemm_exact_scaled(a_bf16: np.ndarray, b_bf16: np.ndarray) -> np.ndarray:
-    """Exact C·2⁴⁶ as int64, for operands that are multiples of 2⁻²³ in [-1, 1].
+def gemm_exact_scaled(a_bits: np.ndarray, b_bits: np.ndarray, dtype: str = "bf16") -> np.ndarray:
+    """Exact C·2^(2s) as int64, for operands that are multiples of 2^-s in
+    [-1, 1] (s = 23 for bf16, 24 for fp16).
 
-    Every generated bf16 value x satisfies x·2²³ ∈ ℤ and |x·2²³| ≤ 2²³, so each
-    product is an integer ≤ 2⁴⁶ and a K ≤ 2¹⁴ sum stays below 2⁶⁰: int64
-    arithmetic is exact.  Plain triple loop over k for clarity (tiny shapes).
+    Every generated bf16 value x satisfies x·2²³ ∈ ℤ (binary16 values in
+    [-1, 1]: x·2²⁴ ∈ ℤ, the subnormal step) and |x·2^s| ≤ 2^s, so each
+    product is an integer ≤ 2^(2s) and a K ≤ 2¹⁴ sum stays below 2⁶²: int64
+    arithmetic is exact.  Plain loop over k for clarity (tiny shapes).
     """
-    a = gen.bf16_to_f32(a_bf16).astype(np.float64) * 2.0 ** 23
-    b = gen.bf16_to_f32(b_bf16).astype(np.float64) * 2.0 ** 23
+    sc = 24 if dtype == "f16" else 23
+    a = gen.widen(dtype, a_bits).astype(np.float64) * 2.0 ** sc
+    b = gen.widen(dtype, b_bits).astype(np.float64) * 2.0 ** sc
     ai = a.astype(np.int64)
     bi = b.astype(np.int64)
     if not (np.array_equal(ai, a) and np.array_equal(bi, b)):
-        raise ValueError("operands are not multiples of 2^-23")
-    if np.abs(ai).max(initial=0) > 2 ** 23 or np.abs(bi).max(initial=0) > 2 ** 23:
+        raise ValueError(f"operands are not multiples of 2^-{sc}")
+    if np.abs(ai).max(initial=0) > 2 ** sc or np.abs(bi).max(initial=0) > 2 ** sc:
         raise ValueError("operands exceed |x| <= 1")
     m, k = ai.shape
     n = bi.shape[1]
@@ -53,7 +57,7 @@ def gemm_exact_scaled(a_bf16: np.ndarray, b_bf16: np.ndarray) -> np.ndarray:
 
 
 def gemm_sampled_f64(seed: int, M: int, N: int, K: int, rows, cols,
-                     tid_a: int = 0, tid_b: int = 1) -> np.ndarray:
+                     tid_a: int = 0, tid_b: int = 1, dtype: str = "bf16") -> np.ndarray:
     """C[rows[s], cols[s]] in fp64, regenerating only the needed row of A and
     column of B from the counter-based generator (no GPU data involved)."""
     rows = np.asarray(rows, dtype=np.int64)
@@ -64,17 +68,23 @@ def gemm_sampled_f64(seed: int, M: int, N: int, K: int, rows, cols,
     cache_b: dict = {}
     for s, (i, j) in enumerate(zip(rows.tolist(), cols.tolist())):
         if i not in cache_a:
-            cache_a[i] = gen.bf16_to_f32(gen.uniform_bf16_at(seed, tid_a, i * K + kk)).astype(np.float64)
+            cache_a[i] = gen.widen(dtype, gen.uniform_at(dtype, seed, tid_a, i * K + kk)).astype(np.float64)
         if j not in cache_b:
-            cache_b[j] = gen.bf16_to_f32(gen.uniform_bf16_at(seed, tid_b, kk * N + j)).astype(np.float64)
+            cache_b[j] = gen.widen(dtype, gen.uniform_at(dtype, seed, tid_b, kk * N + j)).astype(np.float64)
         out[s] = float(np.dot(cache_a[i], cache_b[j]))
     return out
 
 
-def gemm_tolerance(c_ref: np.ndarray, K: int) -> np.ndarray:
-    """|C_gpu − C_ref| ≤ 2⁻⁷·|C_ref| + 2⁻¹²·√K (workload definition: bf16 output
-    rounding ≤ 2⁻⁸ relative, fp32 accumulation-order error ≪ 2⁻¹²·√K)."""
-    return 2.0 ** -7 * np.abs(c_ref) + 2.0 ** -12 * math.sqrt(K)
+GEMM_RTOL = {"bf16": 2.0 ** -7, "f16": 2.0 ** -10}
+
+
+def gemm_tolerance(c_ref: np.ndarray, K: int, dtype: str = "bf16") -> np.ndarray:
+    """|C_gpu − C_ref| ≤ rtol·|C_ref| + 2⁻¹²·√K with rtol = 2⁻⁷ for bf16 output
+    (workload definition: bf16 rounding ≤ 2⁻⁸ relative, fp32 accumulation-order
+    error ≪ 2⁻¹²·√K) and, by the same reasoning, 2⁻¹⁰ for binary16 output
+    (rounding ≤ 2⁻¹¹ relative in the normal range; the absolute term covers
+    the subnormal range, whose step 2⁻²⁴ is far below it)."""
+    return GEMM_RTOL[dtype] * np.abs(c_ref) + 2.0 ** -12 * math.sqrt(K)
 
 
 # --------------------------------------------------------------- softmax ----

@@ -217,3 +217,60 @@ def test_gather_matches_bulk():
     x = gen.normal_f32(9, 0, 7, 13)
     idx = np.array([0, 1, 12, 13, 90])
     assert np.array_equal(gen.normal_f32_at(9, 0, idx), x.ravel()[idx])
+
+
+# ------------------------------------------------------------------ fp16 ----
+
+def _f16_numpy(x):
+    """numpy's independent fp32 -> binary16 conversion (round to nearest even,
+    subnormals included), as bit patterns."""
+    with np.errstate(over="ignore"):
+        return np.asarray(x, dtype=np.float32).astype(np.float16).view(np.uint16)
+
+
+def test_f16_rounding_matches_numpy_on_edges_and_random_values():
+    edges = [0.0, -0.0, 2.0 ** -24, 2.0 ** -25, 1.5 * 2.0 ** -25, 2.0 ** -26, 3 * 2.0 ** -26,
+             2.0 ** -14, 2.0 ** -14 - 2.0 ** -25, 2.0 ** -14 - 2.0 ** -26, 2.0 ** -15 + 2.0 ** -25,
+             1.0, 1.0 + 2.0 ** -11, 1.0 + 3 * 2.0 ** -11, 1.0 - 2.0 ** -12, 65504.0, 65519.0,
+             65520.0, 1e6, 1e-30, float(np.finfo(np.float32).tiny), 0.333333]
+    x = np.array(edges + [-v for v in edges], dtype=np.float32)
+    assert np.array_equal(gen.f32_to_f16(x), _f16_numpy(x))
+    rng = np.random.default_rng(5)
+    # random fp32 bit patterns with exponents around the binary16 range
+    u = (rng.integers(0, 1 << 23, 2_000_000, dtype=np.uint32) |
+         (rng.integers(127 - 30, 127 + 17, 2_000_000).astype(np.uint32) << 23) |
+         (rng.integers(0, 2, 2_000_000).astype(np.uint32) << 31))
+    x = u.view(np.float32)
+    assert np.array_equal(gen.f32_to_f16(x), _f16_numpy(x))
+    inf_nan = np.array([np.inf, -np.inf, np.nan], dtype=np.float32)
+    got = gen.f32_to_f16(inf_nan)
+    assert got[0] == 0x7C00 and got[1] == 0xFC00 and (got[2] & 0x7C00) == 0x7C00 and (got[2] & 0x3FF)
+
+
+def test_uniform_f16_is_the_same_draw_rounded_to_binary16():
+    # the fp16 operand generator: the bf16 generator's 24-bit values, rounded
+    # to binary16 by numpy's independent conversion
+    seed, tid, n = 11, 1, 4096
+    key = gen.stream_key(seed, tid)
+    z = gen.draws(key, 0, n // 2)
+    b = np.empty(n, dtype=np.int64)
+    b[0::2] = (z >> np.uint64(40)).astype(np.int64)
+    b[1::2] = ((z >> np.uint64(8)) & np.uint64(0xFFFFFF)).astype(np.int64)
+    x = ((b - 2 ** 23).astype(np.float64) / 2.0 ** 23).astype(np.float32)   # exact
+    assert np.array_equal(gen.uniform_f16(seed, tid, 64, 64).ravel(), _f16_numpy(x))
+
+
+def test_uniform_f16_exhaustive_over_all_24bit_values():
+    b = np.arange(1 << 24, dtype=np.int64)
+    x = ((b - 2 ** 23).astype(np.float64) / 2.0 ** 23).astype(np.float32)
+    assert np.array_equal(gen.f32_to_f16(x), _f16_numpy(x))
+
+
+def test_uniform_f16_values_are_multiples_of_2m24_in_closed_unit_interval():
+    v = gen.f16_to_f32(gen.uniform_f16(3, 0, 256, 256)).astype(np.float64)
+    assert v.min() >= -1.0 and v.max() <= 1.0
+    s = v * 2.0 ** 24
+    assert np.array_equal(s, np.round(s))
+    # and the gather form agrees with the bulk form
+    idx = np.arange(0, 256 * 256, 37)
+    assert np.array_equal(gen.uniform_f16_at(3, 0, idx), gen.uniform_f16(3, 0, 256, 256).ravel()[idx])

@@ -248,3 +248,37 @@ def test_kendall_tau_b_against_scipy():
     assert math.isclose(ref.kendall_tau_b(x, y), stats.kendalltau(x, y).statistic, rel_tol=1e-12)
     assert ref.kendall_tau_b([1, 2, 3], [1, 2, 3]) == 1.0
     assert ref.kendall_tau_b([1, 2, 3], [3, 2, 1]) == -1.0
+
+
+def test_gemm_f16_exact_int64_matches_fraction_brute_force():
+    a = gen.uniform_f16(5, 0, 5, 7)
+    b = gen.uniform_f16(5, 1, 7, 3)
+    s = ref.gemm_exact_scaled(a, b, dtype="f16")
+    af = gen.f16_to_f32(a).astype(np.float64)
+    bf = gen.f16_to_f32(b).astype(np.float64)
+    for i in range(5):
+        for j in range(3):
+            exact = sum(Fraction(af[i, k]) * Fraction(bf[k, j]) for k in range(7))
+            assert Fraction(int(s[i, j]), 2 ** 48) == exact
+
+
+def test_gemm_f16_f64_within_rounding_bound_of_exact():
+    M, N, K = 16, 24, 512
+    a = gen.uniform_f16(6, 0, M, K)
+    b = gen.uniform_f16(6, 1, K, N)
+    exact = ref.gemm_exact_scaled(a, b, dtype="f16").astype(np.float64) * 2.0 ** -48
+    c64 = ref.gemm_f64(a, b, dtype="f16")
+    absab = np.abs(gen.f16_to_f32(a).astype(np.float64)) @ np.abs(gen.f16_to_f32(b).astype(np.float64))
+    assert np.all(np.abs(c64 - exact) <= (K + 1) * 2.0 ** -53 * absab + 2.0 ** -60)
+
+
+def test_gemm_f16_sampled_matches_full():
+    seed, M, N, K = 9, 64, 48, 80
+    a = gen.uniform_f16(seed, 0, M, K)
+    b = gen.uniform_f16(seed, 1, K, N)
+    full = ref.gemm_f64(a, b, dtype="f16")
+    i, j = ref.sample_indices(seed, 2, 200, M, N)
+    got = ref.gemm_sampled_f64(seed, M, N, K, i, j, dtype="f16")
+    assert np.allclose(got, full[i, j], rtol=1e-13, atol=1e-13)
+    # the f16 operands are not the bf16 ones: the products differ
+    assert not np.array_equal(full, ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N)))
