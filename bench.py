@@ -174,8 +174,9 @@ def kernel_table(ws, w, peaks, stream):
     A, B = ws.inputs
     rec("fill_uniform_bf16", lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, A, stream), nbytes=A.numel() * 2)
     rec("flush_l2", flush, nbytes=flush_t.numel(), do_flush=False)
-    rec("gemm_ref_simt", lambda: krex.krex_run_reference(0, ws.inputs, ws.ref, stream), flops=w.flops, n=3)
-    rec("gemm_tcgen05", lambda: krex.krex_run_candidate_ws(0, ws.inputs, ws.out, ws.gemm_ws, stream), flops=w.flops)
+    rec("gemm_ref_simt", lambda: krex.krex_run_reference(w.op, ws.inputs, ws.ref, stream), flops=w.flops, n=3)
+    rec("gemm_tcgen05", lambda: krex.krex_run_candidate_ws(w.op, ws.inputs, ws.out, ws.gemm_ws, stream),
+        flops=w.flops)
     scratch = ws.check_scratch
     rec("check_bf16_f32", lambda: krex.krex_check_launch(ws.out, ws.ref, w.atol, w.rtol, scratch, stream),
         nbytes=ws.out.numel() * 6, n=10)
@@ -188,6 +189,16 @@ def kernel_table(ws, w, peaks, stream):
     rec("softmax_f32", lambda: krex.krex_run_candidate(1, [x], y, stream), nbytes=x.numel() * 8, n=10)
     rec("check_f32_f32", lambda: krex.krex_check_launch(y, x, 1e-6, 0.0, scratch, stream), nbytes=x.numel() * 8, n=5)
     del x, y
+    # the fp16 form of the GEMM candidate at the same size
+    fw = WORKLOADS["gemm_f16_4096"]
+    a16 = torch.empty(fw.M, fw.K, dtype=torch.float16, device=A.device)
+    b16 = torch.empty(fw.K, fw.N, dtype=torch.float16, device=A.device)
+    c16 = torch.empty(fw.M, fw.N, dtype=torch.float16, device=A.device)
+    rec("fill_uniform_f16", lambda: krex.krex_gen_inputs(fw.seed, 0, 0, 0.0, a16, stream), nbytes=a16.numel() * 2)
+    krex.krex_gen_inputs(fw.seed, 1, 0, 0.0, b16, stream)
+    rec("gemm_tcgen05_f16", lambda: krex.krex_run_candidate_ws(fw.op, [a16, b16], c16, ws.gemm_ws, stream),
+        flops=fw.flops)
+    del a16, b16, c16
     torch.cuda.empty_cache()
     return out
 
@@ -203,23 +214,23 @@ def oracle_command_cost(w, budget_s: float = 10.0):
     import numpy as np
     from oracle import gen, ref
     t0 = time.perf_counter()
-    if w.op == 0:
-        a = gen.uniform_bf16(w.seed, 0, w.M, w.K)
-        b = gen.uniform_bf16(w.seed, 1, w.K, w.N)
+    if w.is_gemm:
+        a = gen.uniform(w.dtype, w.seed, 0, w.M, w.K)
+        b = gen.uniform(w.dtype, w.seed, 1, w.K, w.N)
     else:
         x = gen.normal_f32(w.seed, 0, min(w.M, 2048), w.N, w.sigma)
     t_gen = time.perf_counter() - t0
-    if w.op != 0:
+    if not w.is_gemm:
         t_gen *= w.M / min(w.M, 2048)
     rows = 0
     t_work = 0.0
     reps = 0
     tb = time.perf_counter()
-    block = 64 if w.op == 0 else 256
+    block = 64 if w.is_gemm else 256
     while time.perf_counter() - tb < budget_s * 0.6 and rows < w.M:
         t1 = time.perf_counter()
-        if w.op == 0:
-            c = ref.gemm_f64(a[rows % w.M:rows % w.M + block], b)
+        if w.is_gemm:
+            c = ref.gemm_f64(a[rows % w.M:rows % w.M + block], b, dtype=w.dtype)
         else:
             c = ref.softmax_rows_f64(x[:block].astype(np.float64))
         t_work += time.perf_counter() - t1
@@ -228,13 +239,13 @@ def oracle_command_cost(w, budget_s: float = 10.0):
     per_full = t_work * (w.M / rows)
     t1 = time.perf_counter()
     n_chk = min(w.M, 2048)
-    o32 = c[:1].astype(np.float32).repeat(n_chk, axis=0) if w.op == 0 else c[:1].astype(np.float32).repeat(n_chk, 0)
+    o32 = c[:1].astype(np.float32).repeat(n_chk, axis=0)
     ref.check_f32(o32, o32, w.atol, w.rtol)
     t_chk = (time.perf_counter() - t1) * (w.M / n_chk)
     runs = 1 + 1 + w.warmup + w.iters
     total = t_gen + runs * per_full + t_chk
     info = (f"oracle command of {w.name}: input generation in full (single thread), "
-            f"{'fp64 GEMM' if w.op == 0 else 'fp64 softmax'} on {rows} of {w.M} output rows scaled to the full "
+            f"{'fp64 GEMM' if w.is_gemm else 'fp64 softmax'} on {rows} of {w.M} output rows scaled to the full "
             f"output and counted {runs}x (reference + check run + {w.warmup} warm-up + {w.iters} timed), "
             f"fp32 check on {n_chk} rows scaled; sample wall {time.perf_counter() - t0:.1f} s")
     return total, info
@@ -417,7 +428,7 @@ def kernel_only(args):
     ws = Workspace(w)
     k = args.kernel_only
     # minimal set-up: inputs, and for the check the two outputs it compares
-    if w.op == 0:
+    if w.is_gemm:
         krex.krex_gen_inputs(w.seed, 0, 0, 0.0, ws.inputs[0], stream)
         krex.krex_gen_inputs(w.seed, 1, 0, 0.0, ws.inputs[1], stream)
     else:
@@ -426,8 +437,8 @@ def kernel_only(args):
         krex.krex_run_reference(w.op, ws.inputs, ws.ref, stream)
         krex.krex_run_candidate(w.op, ws.inputs, ws.out, stream)
     fn = {
-        "gemm": lambda: krex.krex_run_candidate_ws(0, ws.inputs, ws.out, ws.gemm_ws, stream),
-        "gemm_ref": lambda: krex.krex_run_reference(0, ws.inputs, ws.ref, stream),
+        "gemm": lambda: krex.krex_run_candidate_ws(w.op, ws.inputs, ws.out, ws.gemm_ws, stream),
+        "gemm_ref": lambda: krex.krex_run_reference(w.op, ws.inputs, ws.ref, stream),
         "fill_uniform": lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, ws.inputs[0], stream),
         "fill_normal": lambda: krex.krex_gen_inputs(w.seed, 0, 1, w.sigma, ws.inputs[0], stream),
         "flush": lambda: krex.krex_flush_l2(ws.flush, stream=stream),

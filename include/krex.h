@@ -49,16 +49,17 @@ typedef enum {
     KREX_ERR_DEVICE = 6        /* a kernel reported an error through its status word */
 } krex_status;
 
-typedef enum { KREX_BF16 = 1, KREX_F32 = 2 } krex_dtype;
+typedef enum { KREX_BF16 = 1, KREX_F32 = 2, KREX_F16 = 3 } krex_dtype;
 
 typedef enum {
-    KREX_DIST_UNIFORM_PM1 = 0, /* U[-1,1] rounded to bf16 (out must be KREX_BF16) */
-    KREX_DIST_NORMAL = 1       /* N(0, sigma^2) in fp32 (out must be KREX_F32)    */
+    KREX_DIST_UNIFORM_PM1 = 0, /* U[-1,1] rounded to bf16 or binary16 (out KREX_BF16 or KREX_F16) */
+    KREX_DIST_NORMAL = 1       /* N(0, sigma^2) in fp32 (out must be KREX_F32)                     */
 } krex_dist;
 
 typedef enum {
-    KREX_OP_GEMM_BF16 = 0,     /* C[MxN] = A[MxK] B[KxN]; bf16 in, fp32 accumulate */
-    KREX_OP_SOFTMAX_F32 = 1    /* Y = row softmax of X, fp32                        */
+    KREX_OP_GEMM_BF16 = 0,     /* C[MxN] = A[MxK] B[KxN]; bf16 in, fp32 accumulate, bf16 out */
+    KREX_OP_SOFTMAX_F32 = 1,   /* Y = row softmax of X, fp32                                  */
+    KREX_OP_GEMM_F16 = 2       /* the same GEMM with IEEE binary16 A, B and C                 */
 } krex_op;
 
 /* A caller-owned device matrix.  dtype is a krex_dtype; ld >= cols, in elements. */
@@ -118,7 +119,8 @@ typedef struct krex_region krex_region; /* opaque; created by begin, released by
  *   key = mix64(seed + (tensor_id+1)*G), draw j = mix64(key + (j+1)*G),
  * G = 0x9E3779B97F4A7C15, mix64 = the SplitMix64 output mix.
  * KREX_DIST_UNIFORM_PM1: elements 2j, 2j+1 take bits 63..40 and 31..8 of draw
- * j; b -> (b - 2^23) 2^-23 rounded to bf16 (RNE).  KREX_DIST_NORMAL: pair j is
+ * j; b -> (b - 2^23) 2^-23 rounded to bf16 (RNE; to IEEE binary16 with
+ * subnormals, RNE, when out is KREX_F16).  KREX_DIST_NORMAL: pair j is
  * a Box-Muller pair from draw j (u1 = (hi24+1) 2^-24, u2 = lo24 2^-24) scaled by
  * sigma, in fp32.  Output is bit-identical for any launch shape.
  * Errors: INVALID for a null/empty-but-nonzero buffer, dtype/dist mismatch,
@@ -134,6 +136,7 @@ krex_status krex_gen_inputs(uint64_t seed, uint32_t tensor_id, int32_t dist, flo
  *   (M x N, bf16, RNE from the fp32 accumulator).  tcgen05 tensor cores with
  *   TMEM accumulators, TMA loads.  Needs K, N, lda, ldb multiples of 8 and
  *   16-byte aligned A, B (TMA), else UNSUPPORTED.  K = 0 gives C = 0.
+ * KREX_OP_GEMM_F16: the same with IEEE binary16 A, B and C (RNE out).
  * KREX_OP_SOFTMAX_F32: in[0] = X (rows x cols, fp32), out = Y (same shape,
  *   fp32); y = exp(x - max) / sum exp(x - max) per row, one HBM pass.
  * Errors: INVALID for wrong n_in, dtypes or shapes; DEVICE if the kernel's

@@ -19,9 +19,9 @@ LIB_PATH = os.path.join(_PKG, "libkrex.so")
 
 KREX_OK, KREX_ERR_INVALID, KREX_ERR_UNSUPPORTED, KREX_ERR_CUDA, KREX_ERR_STATE, KREX_ERR_TIMEOUT, \
     KREX_ERR_DEVICE = range(7)
-KREX_BF16, KREX_F32 = 1, 2
+KREX_BF16, KREX_F32, KREX_F16 = 1, 2, 3
 KREX_DIST_UNIFORM_PM1, KREX_DIST_NORMAL = 0, 1
-KREX_OP_GEMM_BF16, KREX_OP_SOFTMAX_F32 = 0, 1
+KREX_OP_GEMM_BF16, KREX_OP_SOFTMAX_F32, KREX_OP_GEMM_F16 = 0, 1, 2
 KREX_MAX_ITERS = 100000
 
 
@@ -170,7 +170,7 @@ def buf(t, rows: int | None = None, cols: int | None = None) -> krex_buf:
         t = t.view(1, -1)
     if t.dim() != 2 or (t.size(1) > 1 and t.stride(1) != 1):
         raise ValueError("need a 2-D tensor with unit column stride")
-    dt = {torch.bfloat16: KREX_BF16, torch.float32: KREX_F32}.get(t.dtype)
+    dt = {torch.bfloat16: KREX_BF16, torch.float32: KREX_F32, torch.float16: KREX_F16}.get(t.dtype)
     if dt is None:
         raise ValueError(f"unsupported dtype {t.dtype}")
     r = t.size(0) if rows is None else rows

@@ -14,7 +14,8 @@ import ctypes
 import math
 from dataclasses import dataclass, replace
 
-from . import (KREX_BF16, KREX_F32, KREX_OP_GEMM_BF16, KREX_OP_SOFTMAX_F32, buf, krex_check_scratch_bytes,
+from . import (KREX_BF16, KREX_F32, KREX_OP_GEMM_BF16, KREX_OP_GEMM_F16, KREX_OP_SOFTMAX_F32, buf,
+               krex_check_scratch_bytes,
                krex_command, krex_command_bufs, krex_command_run, krex_gemm_workspace_bytes)
 
 MiB = 1 << 20
@@ -36,23 +37,33 @@ class Workload:
     repeat: int = 1                     # commands per measurement
 
     @property
+    def is_gemm(self) -> bool:
+        return self.op in (KREX_OP_GEMM_BF16, KREX_OP_GEMM_F16)
+
+    @property
+    def dtype(self) -> str:
+        """Operand dtype: "bf16", "f16" (GEMMs) or "f32" (softmax)."""
+        return {KREX_OP_GEMM_BF16: "bf16", KREX_OP_GEMM_F16: "f16"}.get(self.op, "f32")
+
+    @property
     def atol(self) -> float:
         # GEMM: 2^-12 sqrt(K) (fp32 accumulation order); softmax: 1e-6 absolute
-        return 2.0 ** -12 * math.sqrt(self.K) if self.op == KREX_OP_GEMM_BF16 else 1e-6
+        return 2.0 ** -12 * math.sqrt(self.K) if self.is_gemm else 1e-6
 
     @property
     def rtol(self) -> float:
-        # GEMM: 2^-7 (bf16 output rounding is <= 2^-8 relative); softmax: 0
-        return 2.0 ** -7 if self.op == KREX_OP_GEMM_BF16 else 0.0
+        # GEMM: 2^-7 for bf16 output (rounding <= 2^-8 relative), 2^-10 for
+        # binary16 output (<= 2^-11); softmax: 0
+        return {KREX_OP_GEMM_BF16: 2.0 ** -7, KREX_OP_GEMM_F16: 2.0 ** -10}.get(self.op, 0.0)
 
     @property
     def flops(self) -> int:
-        return 2 * self.M * self.N * self.K if self.op == KREX_OP_GEMM_BF16 else 0
+        return 2 * self.M * self.N * self.K if self.is_gemm else 0
 
     @property
     def candidate_bytes(self) -> int:
         """Algorithmic HBM bytes of one candidate launch."""
-        if self.op == KREX_OP_GEMM_BF16:
+        if self.is_gemm:
             return 2 * (self.M * self.K + self.K * self.N + self.M * self.N)
         return 8 * self.M * self.N
 
@@ -66,6 +77,8 @@ WORKLOADS = {
                                        iters=100, flush_bytes=256 * MiB, oracle_samples=4096),
     "gemm_bf16_8192": Workload("gemm_bf16_8192", KREX_OP_GEMM_BF16, 8192, 8192, 8192, seed=4, iters=50,
                                flush_bytes=256 * MiB, oracle_samples=4096),
+    "gemm_f16_4096": Workload("gemm_f16_4096", KREX_OP_GEMM_F16, 4096, 4096, 4096, seed=2, iters=100,
+                              flush_bytes=256 * MiB),
     "gemm_bf16_16384": Workload("gemm_bf16_16384", KREX_OP_GEMM_BF16, 16384, 16384, 16384, seed=5, iters=20,
                                 flush_bytes=256 * MiB, oracle_samples=4096, repeat=32),
 }
@@ -81,11 +94,12 @@ class Workspace:
     def __init__(self, w: Workload, device="cuda"):
         import torch
         self.w = w
-        bf16, f32 = torch.bfloat16, torch.float32
-        if w.op == KREX_OP_GEMM_BF16:
-            self.inputs = [torch.empty(w.M, w.K, dtype=bf16, device=device),
-                           torch.empty(w.K, w.N, dtype=bf16, device=device)]
-            self.out = torch.empty(w.M, w.N, dtype=bf16, device=device)
+        f32 = torch.float32
+        if w.is_gemm:
+            t16 = torch.float16 if w.op == KREX_OP_GEMM_F16 else torch.bfloat16
+            self.inputs = [torch.empty(w.M, w.K, dtype=t16, device=device),
+                           torch.empty(w.K, w.N, dtype=t16, device=device)]
+            self.out = torch.empty(w.M, w.N, dtype=t16, device=device)
         else:
             self.inputs = [torch.empty(w.M, w.N, dtype=f32, device=device)]
             self.out = torch.empty(w.M, w.N, dtype=f32, device=device)
@@ -94,7 +108,7 @@ class Workspace:
         self.check_scratch = torch.empty(krex_check_scratch_bytes(), dtype=torch.uint8, device=device)
         # the GEMM's split-K meeting place: zero-filled once, left ready by every call
         self.gemm_ws = (torch.zeros(krex_gemm_workspace_bytes(), dtype=torch.uint8, device=device)
-                        if w.op == KREX_OP_GEMM_BF16 else None)
+                        if w.is_gemm else None)
         self.durations = (ctypes.c_float * w.iters)()
         self.cmd = krex_command(w.op, w.warmup, w.iters, 0, w.M, w.N, w.K, w.seed, w.sigma, w.atol, w.rtol, 0, 0,
                                 w.flush_bytes)

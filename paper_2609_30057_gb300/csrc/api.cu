@@ -94,7 +94,14 @@ static uint64_t stream_key(uint64_t seed, uint32_t tensor_id) {
 
 // -------------------------------------------------------------- validation --
 
-static size_t elem_size(int32_t dt) { return dt == KREX_BF16 ? 2 : (dt == KREX_F32 ? 4 : 0); }
+static size_t elem_size(int32_t dt) { return (dt == KREX_BF16 || dt == KREX_F16) ? 2 : (dt == KREX_F32 ? 4 : 0); }
+
+static bool is_gemm(int32_t op) { return op == KREX_OP_GEMM_BF16 || op == KREX_OP_GEMM_F16; }
+
+// dtype of a GEMM op's operands and output; fp32 for the softmax
+static int32_t op_dtype(int32_t op) {
+    return op == KREX_OP_GEMM_BF16 ? KREX_BF16 : (op == KREX_OP_GEMM_F16 ? KREX_F16 : KREX_F32);
+}
 
 static krex_status check_buf(const krex_buf &b, const char *name) {
     if (elem_size(b.dtype) == 0) return set_error(KREX_ERR_INVALID, "%s: bad dtype %d", name, b.dtype);
@@ -121,11 +128,11 @@ static krex_status check_op_shapes(int32_t op, const krex_buf *in, int32_t n_in,
                                    int32_t out_dtype, const char *out_name) {
     if (!in) return set_error(KREX_ERR_INVALID, "in is null");
     krex_status st;
-    if (op == KREX_OP_GEMM_BF16) {
+    if (is_gemm(op)) {
         if (n_in != 2) return set_error(KREX_ERR_INVALID, "GEMM takes 2 inputs, got %d", n_in);
         if ((st = check_buf(in[0], "A")) || (st = check_buf(in[1], "B")) || (st = check_buf(out, out_name))) return st;
-        if (in[0].dtype != KREX_BF16 || in[1].dtype != KREX_BF16)
-            return set_error(KREX_ERR_INVALID, "GEMM inputs must be bf16");
+        if (in[0].dtype != op_dtype(op) || in[1].dtype != op_dtype(op))
+            return set_error(KREX_ERR_INVALID, "GEMM inputs must be %s", op == KREX_OP_GEMM_F16 ? "fp16" : "bf16");
         if (out.dtype != out_dtype) return set_error(KREX_ERR_INVALID, "%s has the wrong dtype", out_name);
         if (in[0].cols != in[1].rows) return set_error(KREX_ERR_INVALID, "A.cols %lld != B.rows %lld",
                                                        (long long)in[0].cols, (long long)in[1].rows);
@@ -148,7 +155,7 @@ static krex_status check_op_shapes(int32_t op, const krex_buf *in, int32_t n_in,
 // Candidate/reference dispatch after validation.
 static krex_status do_candidate(int32_t op, const krex_buf *in, const krex_buf &out, cudaStream_t s,
                                 void *ws = nullptr, size_t ws_bytes = 0) {
-    if (op == KREX_OP_GEMM_BF16) {
+    if (is_gemm(op)) {
         const krex_buf &A = in[0], &B = in[1];
         const int64_t M = A.rows, K = A.cols, N = B.cols;
         if (M == 0 || N == 0) return ok();
@@ -160,7 +167,8 @@ static krex_status do_candidate(int32_t op, const krex_buf *in, const krex_buf &
         }
         krex_status st = launch_gemm_tcgen05(static_cast<const uint16_t *>(A.ptr), A.ld,
                                              static_cast<const uint16_t *>(B.ptr), B.ld,
-                                             static_cast<uint16_t *>(out.ptr), out.ld, M, N, K, ws, ws_bytes, s);
+                                             static_cast<uint16_t *>(out.ptr), out.ld, M, N, K,
+                                             op == KREX_OP_GEMM_F16, ws, ws_bytes, s);
         if (st != KREX_OK) return st;
         if (K > 0) count_launches(1);
         return ok();
@@ -173,11 +181,11 @@ static krex_status do_candidate(int32_t op, const krex_buf *in, const krex_buf &
 }
 
 static krex_status do_reference(int32_t op, const krex_buf *in, const krex_buf &ref, cudaStream_t s) {
-    if (op == KREX_OP_GEMM_BF16) {
+    if (is_gemm(op)) {
         const krex_buf &A = in[0], &B = in[1];
         KREX_CUDA_TRY(launch_gemm_ref(static_cast<const uint16_t *>(A.ptr), A.ld,
                                       static_cast<const uint16_t *>(B.ptr), B.ld, static_cast<float *>(ref.ptr),
-                                      ref.ld, A.rows, B.cols, A.cols, s));
+                                      ref.ld, A.rows, B.cols, A.cols, op == KREX_OP_GEMM_F16, s));
         if (A.rows * B.cols > 0) count_launches(1);
         return ok();
     }
@@ -330,7 +338,8 @@ krex_status krex_gen_inputs(uint64_t seed, uint32_t tensor_id, int32_t dist, flo
     krex_status st = check_buf(out, "out");
     if (st) return st;
     if (dist == KREX_DIST_UNIFORM_PM1) {
-        if (out.dtype != KREX_BF16) return set_error(KREX_ERR_INVALID, "uniform inputs are bf16");
+        if (out.dtype != KREX_BF16 && out.dtype != KREX_F16)
+            return set_error(KREX_ERR_INVALID, "uniform inputs are bf16 or fp16");
     } else if (dist == KREX_DIST_NORMAL) {
         if (out.dtype != KREX_F32) return set_error(KREX_ERR_INVALID, "normal inputs are fp32");
         if (!std::isfinite(sigma)) return set_error(KREX_ERR_INVALID, "sigma must be finite");
@@ -342,7 +351,7 @@ krex_status krex_gen_inputs(uint64_t seed, uint32_t tensor_id, int32_t dist, flo
     const uint64_t key = stream_key(seed, tensor_id);
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     if (dist == KREX_DIST_UNIFORM_PM1)
-        KREX_CUDA_TRY(launch_fill_uniform_bf16(key, out.ptr, out.rows, out.cols, out.ld, s));
+        KREX_CUDA_TRY(launch_fill_uniform_16(key, out.dtype == KREX_F16, out.ptr, out.rows, out.cols, out.ld, s));
     else
         KREX_CUDA_TRY(launch_fill_normal_f32(key, sigma, static_cast<float *>(out.ptr), out.rows, out.cols, out.ld, s));
     count_launches(1);
@@ -350,7 +359,7 @@ krex_status krex_gen_inputs(uint64_t seed, uint32_t tensor_id, int32_t dist, flo
 }
 
 krex_status krex_run_candidate(int32_t op, const krex_buf *in, int32_t n_in, krex_buf out, krex_stream_t stream) {
-    krex_status st = check_op_shapes(op, in, n_in, out, op == KREX_OP_GEMM_BF16 ? KREX_BF16 : KREX_F32, "out");
+    krex_status st = check_op_shapes(op, in, n_in, out, op_dtype(op), "out");
     if (st) return st;
     return do_candidate(op, in, out, reinterpret_cast<cudaStream_t>(stream));
 }
@@ -359,7 +368,7 @@ size_t krex_gemm_workspace_bytes(void) { return gemm_workspace_bytes(); }
 
 krex_status krex_run_candidate_ws(int32_t op, const krex_buf *in, int32_t n_in, krex_buf out, void *workspace,
                                   size_t workspace_bytes, krex_stream_t stream) {
-    krex_status st = check_op_shapes(op, in, n_in, out, op == KREX_OP_GEMM_BF16 ? KREX_BF16 : KREX_F32, "out");
+    krex_status st = check_op_shapes(op, in, n_in, out, op_dtype(op), "out");
     if (st) return st;
     if ((st = check_gemm_workspace(workspace, workspace_bytes))) return st;
     return do_candidate(op, in, out, reinterpret_cast<cudaStream_t>(stream), workspace, workspace_bytes);
@@ -557,7 +566,7 @@ krex_status krex_bench_candidate(int32_t op, const krex_buf *in, int32_t n_in, k
     if (!opts) return set_error(KREX_ERR_INVALID, "opts is null");
     if (warmup < 0 || iters < 0 || iters > opts->max_iters)
         return set_error(KREX_ERR_INVALID, "need 0 <= warmup and 0 <= iters <= max_iters");
-    krex_status st = check_op_shapes(op, in, n_in, out, op == KREX_OP_GEMM_BF16 ? KREX_BF16 : KREX_F32, "out");
+    krex_status st = check_op_shapes(op, in, n_in, out, op_dtype(op), "out");
     if (st) return st;
     if ((st = check_gemm_workspace(workspace, workspace_bytes))) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
@@ -588,11 +597,11 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
     if (cmd->iters < 1 || cmd->iters > KREX_MAX_ITERS || cmd->warmup < 0)
         return set_error(KREX_ERR_INVALID, "command: iters must be in [1, %d], warmup >= 0", KREX_MAX_ITERS);
     const int32_t op = cmd->op;
-    const int n_in = op == KREX_OP_GEMM_BF16 ? 2 : 1;
-    krex_status st = check_op_shapes(op, bufs->in, n_in, bufs->out, op == KREX_OP_GEMM_BF16 ? KREX_BF16 : KREX_F32, "out");
+    const int n_in = is_gemm(op) ? 2 : 1;
+    krex_status st = check_op_shapes(op, bufs->in, n_in, bufs->out, op_dtype(op), "out");
     if (st) return st;
     if ((st = check_op_shapes(op, bufs->in, n_in, bufs->ref, KREX_F32, "ref"))) return st;
-    if (op == KREX_OP_GEMM_BF16) {
+    if (is_gemm(op)) {
         if (bufs->in[0].rows != cmd->M || bufs->in[0].cols != cmd->K || bufs->in[1].cols != cmd->N)
             return set_error(KREX_ERR_INVALID, "command: buffers do not match M, N, K");
     } else if (bufs->in[0].rows != cmd->M || bufs->in[0].cols != cmd->N) {
@@ -616,7 +625,7 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
             KREX_CUDA_TRY(cudaMemcpy2DAsync(b.ptr, (size_t)b.ld * es, host_in[i], (size_t)b.cols * es,
                                             (size_t)b.cols * es, (size_t)b.rows, cudaMemcpyHostToDevice, s));
         } else {
-            st = op == KREX_OP_GEMM_BF16
+            st = is_gemm(op)
                      ? krex_gen_inputs(cmd->seed, (uint32_t)i, KREX_DIST_UNIFORM_PM1, 0.0f, b, stream)
                      : krex_gen_inputs(cmd->seed, 0u, KREX_DIST_NORMAL, cmd->sigma, b, stream);
             if (st) return st;

@@ -15,9 +15,10 @@ size_t l2_bytes_current();      // L2 size of the current device
 
 // ---- kernel launchers (return the launch error, never synchronise) --------
 
-// K1: SplitMix64 -> U[-1,1] -> bf16, 16-byte stores.  `key` is the stream key.
-cudaError_t launch_fill_uniform_bf16(uint64_t key, void *out, int64_t rows, int64_t cols,
-                                     int64_t ld, cudaStream_t s);
+// K1: SplitMix64 -> U[-1,1] -> bf16 (f16: binary16), 16-byte stores.  `key`
+// is the stream key.
+cudaError_t launch_fill_uniform_16(uint64_t key, bool f16, void *out, int64_t rows, int64_t cols,
+                                   int64_t ld, cudaStream_t s);
 // K2: SplitMix64 -> Box-Muller -> N(0, sigma^2) fp32, 16-byte stores.
 cudaError_t launch_fill_normal_f32(uint64_t key, float sigma, float *out, int64_t rows,
                                    int64_t cols, int64_t ld, cudaStream_t s);
@@ -34,14 +35,15 @@ cudaError_t launch_softmax(const float *x, int64_t ldx, float *y, int64_t ldy, i
 // K8: three-pass reference softmax.
 cudaError_t launch_softmax_ref(const float *x, int64_t ldx, float *y, int64_t ldy,
                                int64_t rows, int64_t cols, cudaStream_t s);
-// K7: SIMT fp32 reference GEMM (bf16 in, fp32 out).
+// K7: SIMT fp32 reference GEMM (bf16 or, with f16, binary16 in; fp32 out).
 cudaError_t launch_gemm_ref(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb,
-                            float *c, int64_t ldc, int64_t M, int64_t N, int64_t K,
+                            float *c, int64_t ldc, int64_t M, int64_t N, int64_t K, bool f16,
                             cudaStream_t s);
 // K4: tcgen05 GEMM.  Returns KREX_OK or an error status with a message set.
 // `workspace` (may be NULL) enables the split-K tail; see gemm_workspace_bytes.
+// f16: binary16 A, B and C (else bf16).
 krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb,
-                                uint16_t *c, int64_t ldc, int64_t M, int64_t N, int64_t K,
+                                uint16_t *c, int64_t ldc, int64_t M, int64_t N, int64_t K, bool f16,
                                 void *workspace, size_t workspace_bytes, cudaStream_t s);
 size_t gemm_workspace_bytes();
 // Device status word of the GEMM kernel's bounded waits (read and clear).

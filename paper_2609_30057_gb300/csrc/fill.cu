@@ -6,6 +6,7 @@
 //   draw j of a stream   z_j = mix64(key + (j+1) * G)
 //   uniform element e    bits 63..40 (e even) / 31..8 (e odd) of z_{e/2},
 //                        x = (b - 2^23) 2^-23 (exact), bf16 = RNE(x)
+//                        (fp16 operands: binary16 = RNE(x))
 //   normal pair j        u1 = (hi24 + 1) 2^-24, u2 = lo24 2^-24,
 //                        (y0, y1) = sigma * sqrt(-2 ln u1) * (cos, sin)(2 pi u2)
 //
@@ -18,6 +19,7 @@
 // Layout: one thread writes 16 bytes per step (8 bf16 = 4 draws, or 4 fp32 =
 // 2 Box-Muller pairs); rows of a strided buffer are handled by a 2-D grid.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include "common.cuh"
 
@@ -42,26 +44,35 @@ __device__ __forceinline__ float u24_to_pm1(uint32_t b) {
     return __fsub_rn(f, sub);
 }
 
-// Elements 2j (low half) and 2j+1 (high half) from draw z_j.
-__device__ __forceinline__ uint32_t uniform_bf16x2(uint64_t z) {
+// Elements 2j (low half) and 2j+1 (high half) from draw z_j, rounded to
+// bf16 or (F16) to IEEE binary16, both round-to-nearest-even.
+template <bool F16>
+__device__ __forceinline__ uint32_t uniform_16x2(uint64_t z) {
     uint32_t hi = (uint32_t)(z >> 32), lo = (uint32_t)z;
     float x0 = u24_to_pm1(hi >> 8);
     float x1 = u24_to_pm1(lo >> 8);
-    __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
-    return *reinterpret_cast<uint32_t *>(&h);
+    if constexpr (F16) {
+        __half2 h = __floats2half2_rn(x0, x1);
+        return *reinterpret_cast<uint32_t *>(&h);
+    } else {
+        __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
+        return *reinterpret_cast<uint32_t *>(&h);
+    }
 }
 
-__device__ __forceinline__ uint16_t uniform_bf16_at(uint64_t key, uint64_t e) {
-    uint32_t p = uniform_bf16x2(mix64(key + ((e >> 1) + 1ull) * kGamma));
+template <bool F16>
+__device__ __forceinline__ uint16_t uniform_16_at(uint64_t key, uint64_t e) {
+    uint32_t p = uniform_16x2<F16>(mix64(key + ((e >> 1) + 1ull) * kGamma));
     return (uint16_t)((e & 1ull) ? (p >> 16) : (p & 0xFFFFu));
 }
 
 // Contiguous rows (ld == cols) are treated as one row of rows*cols elements.
 // Vector path: cols % 8 == 0 within each row of a strided buffer, or any
 // length for a contiguous buffer (the scalar tail is done by thread 0).
+template <bool F16>
 __global__ void __launch_bounds__(256)
-fill_uniform_bf16_vec(uint64_t key, uint16_t *__restrict__ out, int64_t rows, int64_t cols,
-                      int64_t ld) {
+fill_uniform_16_vec(uint64_t key, uint16_t *__restrict__ out, int64_t rows, int64_t cols,
+                    int64_t ld) {
     const int64_t groups = cols >> 3;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t r = blockIdx.y; r < rows; r += gridDim.y) {
@@ -70,18 +81,18 @@ fill_uniform_bf16_vec(uint64_t key, uint16_t *__restrict__ out, int64_t rows, in
         for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < groups; g += stride) {
             uint64_t s = key + (((e_row + (uint64_t)(g << 3)) >> 1) + 1ull) * kGamma;
             uint4 v;
-            v.x = uniform_bf16x2(mix64(s));
+            v.x = uniform_16x2<F16>(mix64(s));
             s += kGamma;
-            v.y = uniform_bf16x2(mix64(s));
+            v.y = uniform_16x2<F16>(mix64(s));
             s += kGamma;
-            v.z = uniform_bf16x2(mix64(s));
+            v.z = uniform_16x2<F16>(mix64(s));
             s += kGamma;
-            v.w = uniform_bf16x2(mix64(s));
+            v.w = uniform_16x2<F16>(mix64(s));
             *reinterpret_cast<uint4 *>(row + (g << 3)) = v;
         }
         if (blockIdx.x == 0 && threadIdx.x == 0) {
             for (int64_t c = groups << 3; c < cols; ++c)
-                row[c] = uniform_bf16_at(key, e_row + (uint64_t)c);
+                row[c] = uniform_16_at<F16>(key, e_row + (uint64_t)c);
         }
     }
 }
@@ -193,13 +204,14 @@ fill_normal_f32_vec(uint64_t key, float sigma, float *__restrict__ out, int64_t 
 }
 
 // Any layout: one element per thread step (each element recomputes its draw).
+template <bool F16>
 __global__ void __launch_bounds__(256)
-fill_uniform_bf16_scalar(uint64_t key, uint16_t *__restrict__ out, int64_t rows, int64_t cols,
-                         int64_t ld) {
+fill_uniform_16_scalar(uint64_t key, uint16_t *__restrict__ out, int64_t rows, int64_t cols,
+                       int64_t ld) {
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t r = blockIdx.y; r < rows; r += gridDim.y)
         for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < cols; c += stride)
-            out[r * ld + c] = uniform_bf16_at(key, (uint64_t)(r * cols + c));
+            out[r * ld + c] = uniform_16_at<F16>(key, (uint64_t)(r * cols + c));
 }
 
 __global__ void __launch_bounds__(256)
@@ -235,22 +247,31 @@ dim3 fill_grid(int64_t rows, int64_t per_row_items) {
     return dim3((unsigned)bx, (unsigned)by, 1);
 }
 
-}  // namespace
-
-cudaError_t launch_fill_uniform_bf16(uint64_t key, void *out, int64_t rows, int64_t cols,
-                                     int64_t ld, cudaStream_t s) {
-    if (rows == 0 || cols == 0) return cudaSuccess;
-    uint16_t *p = static_cast<uint16_t *>(out);
-    bool aligned = (reinterpret_cast<uintptr_t>(out) & 15u) == 0;
+template <bool F16>
+void launch_uniform(uint64_t key, uint16_t *p, bool aligned, int64_t rows, int64_t cols, int64_t ld,
+                    cudaStream_t s) {
     if (aligned && ld == cols) {
         // one logical row of rows*cols elements
         int64_t n = rows * cols;
-        fill_uniform_bf16_vec<<<fill_grid(1, n >> 3), 256, 0, s>>>(key, p, 1, n, n);
+        fill_uniform_16_vec<F16><<<fill_grid(1, n >> 3), 256, 0, s>>>(key, p, 1, n, n);
     } else if (aligned && (cols & 7) == 0 && (ld & 7) == 0) {
-        fill_uniform_bf16_vec<<<fill_grid(rows, cols >> 3), 256, 0, s>>>(key, p, rows, cols, ld);
+        fill_uniform_16_vec<F16><<<fill_grid(rows, cols >> 3), 256, 0, s>>>(key, p, rows, cols, ld);
     } else {
-        fill_uniform_bf16_scalar<<<fill_grid(rows, cols), 256, 0, s>>>(key, p, rows, cols, ld);
+        fill_uniform_16_scalar<F16><<<fill_grid(rows, cols), 256, 0, s>>>(key, p, rows, cols, ld);
     }
+}
+
+}  // namespace
+
+cudaError_t launch_fill_uniform_16(uint64_t key, bool f16, void *out, int64_t rows, int64_t cols,
+                                   int64_t ld, cudaStream_t s) {
+    if (rows == 0 || cols == 0) return cudaSuccess;
+    uint16_t *p = static_cast<uint16_t *>(out);
+    bool aligned = (reinterpret_cast<uintptr_t>(out) & 15u) == 0;
+    if (f16)
+        launch_uniform<true>(key, p, aligned, rows, cols, ld, s);
+    else
+        launch_uniform<false>(key, p, aligned, rows, cols, ld, s);
     return cudaGetLastError();
 }
 

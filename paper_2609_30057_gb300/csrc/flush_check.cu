@@ -14,6 +14,9 @@
 // block to take a ticket combines the partials and re-arms the ticket.  Max
 // and count are exact, so the result does not depend on the launch shape.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include <type_traits>
 
 #include <mutex>
 
@@ -62,6 +65,7 @@ struct CheckScratch {
 __device__ __forceinline__ float widen(const __nv_bfloat16 *p, int64_t i) {
     return __uint_as_float((uint32_t)(*reinterpret_cast<const uint16_t *>(p + i)) << 16);
 }
+__device__ __forceinline__ float widen(const __half *p, int64_t i) { return __half2float(p[i]); }
 __device__ __forceinline__ float widen(const float *p, int64_t i) { return p[i]; }
 
 struct Acc {
@@ -76,12 +80,21 @@ struct Acc {
     }
 };
 
-__device__ __forceinline__ void bf16x8(const uint4 &u, float *f) {
+// Eight packed 16-bit values widened exactly to fp32 (T: __nv_bfloat16 or
+// __half).
+template <typename T>
+__device__ __forceinline__ void x8_to_f32(const uint4 &u, float *f) {
     const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
-        f[2 * k] = __uint_as_float(w[k] << 16);
-        f[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
+        if constexpr (std::is_same<T, __half>::value) {
+            const float2 v = __half22float2(*reinterpret_cast<const __half2 *>(&w[k]));
+            f[2 * k] = v.x;
+            f[2 * k + 1] = v.y;
+        } else {
+            f[2 * k] = __uint_as_float(w[k] << 16);
+            f[2 * k + 1] = __uint_as_float(w[k] & 0xFFFF0000u);
+        }
     }
 }
 
@@ -145,11 +158,13 @@ __device__ __forceinline__ void block_reduce_publish(Acc acc, CheckScratch *sc) 
     }
 }
 
-// Contiguous fast path: bf16 out vs fp32 ref, 8 elements per step.
+// Contiguous fast path: 16-bit out (bf16 or binary16) vs fp32 ref, 8
+// elements per step.
+template <typename T>
 __global__ void __launch_bounds__(kCheckThreads)
-check_bf16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref, int64_t n8,
-                   const __nv_bfloat16 *out_s, const float *ref_s, int64_t n, float atol,
-                   float rtol, CheckScratch *sc) {
+check_16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref, int64_t n8,
+                 const T *out_s, const float *ref_s, int64_t n, float atol,
+                 float rtol, CheckScratch *sc) {
     Acc acc;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < n8; g += stride) {
@@ -157,7 +172,7 @@ check_bf16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref
         float4 r0 = __ldcs(ref + 2 * g);
         float4 r1 = __ldcs(ref + 2 * g + 1);
         float f[8];
-        bf16x8(o, f);
+        x8_to_f32<T>(o, f);
         acc.add(f[0], r0.x, atol, rtol);
         acc.add(f[1], r0.y, atol, rtol);
         acc.add(f[2], r0.z, atol, rtol);
@@ -221,6 +236,37 @@ check_generic(const TO *out, int64_t ldo, const TR *ref, int64_t ldr, int64_t ro
     block_reduce_publish(acc, sc);
 }
 
+template <typename TO, typename TR>
+void launch_generic(const void *out, int64_t ldo, const void *ref, int64_t ldr, int64_t rows, int64_t cols,
+                    float atol, float rtol, CheckScratch *sc, int blocks, cudaStream_t s) {
+    check_generic<TO, TR><<<blocks, kCheckThreads, 0, s>>>(static_cast<const TO *>(out), ldo,
+                                                          static_cast<const TR *>(ref), ldr, rows, cols,
+                                                          atol, rtol, sc);
+}
+
+template <typename TO>
+void launch_generic_out(const void *out, int64_t ldo, const void *ref, int ref_dtype, int64_t ldr, int64_t rows,
+                        int64_t cols, float atol, float rtol, CheckScratch *sc, int blocks, cudaStream_t s) {
+    if (ref_dtype == KREX_F32)
+        launch_generic<TO, float>(out, ldo, ref, ldr, rows, cols, atol, rtol, sc, blocks, s);
+    else if (ref_dtype == KREX_BF16)
+        launch_generic<TO, __nv_bfloat16>(out, ldo, ref, ldr, rows, cols, atol, rtol, sc, blocks, s);
+    else
+        launch_generic<TO, __half>(out, ldo, ref, ldr, rows, cols, atol, rtol, sc, blocks, s);
+}
+
+// Any layout and any pair of krex dtypes (validated by the caller).
+void launch_check_generic(const void *out, int out_dtype, int64_t ldo, const void *ref, int ref_dtype,
+                          int64_t ldr, int64_t rows, int64_t cols, float atol, float rtol, CheckScratch *sc,
+                          int blocks, cudaStream_t s) {
+    if (out_dtype == KREX_F32)
+        launch_generic_out<float>(out, ldo, ref, ref_dtype, ldr, rows, cols, atol, rtol, sc, blocks, s);
+    else if (out_dtype == KREX_BF16)
+        launch_generic_out<__nv_bfloat16>(out, ldo, ref, ref_dtype, ldr, rows, cols, atol, rtol, sc, blocks, s);
+    else
+        launch_generic_out<__half>(out, ldo, ref, ref_dtype, ldr, rows, cols, atol, rtol, sc, blocks, s);
+}
+
 int check_blocks(int64_t items) {
     int64_t b = (items + kCheckThreads - 1) / kCheckThreads;
     int64_t cap = (int64_t)sm_count() * 8;
@@ -258,33 +304,23 @@ cudaError_t launch_check(const void *out, int out_dtype, int64_t ldo, const void
     const bool a16 = ((reinterpret_cast<uintptr_t>(out) | reinterpret_cast<uintptr_t>(ref)) & 15u) == 0;
     if (contiguous && a16 && out_dtype == KREX_BF16 && ref_dtype == KREX_F32) {
         int64_t n8 = n / 8;
-        check_bf16_f32_vec<<<check_blocks(n8), kCheckThreads, 0, s>>>(
+        check_16_f32_vec<__nv_bfloat16><<<check_blocks(n8), kCheckThreads, 0, s>>>(
             static_cast<const uint4 *>(out), static_cast<const float4 *>(ref), n8,
             static_cast<const __nv_bfloat16 *>(out), static_cast<const float *>(ref), n, atol,
             rtol, sc);
+    } else if (contiguous && a16 && out_dtype == KREX_F16 && ref_dtype == KREX_F32) {
+        int64_t n8 = n / 8;
+        check_16_f32_vec<__half><<<check_blocks(n8), kCheckThreads, 0, s>>>(
+            static_cast<const uint4 *>(out), static_cast<const float4 *>(ref), n8,
+            static_cast<const __half *>(out), static_cast<const float *>(ref), n, atol, rtol, sc);
     } else if (contiguous && a16 && out_dtype == KREX_F32 && ref_dtype == KREX_F32) {
         int64_t n4 = n / 4;
         check_f32_f32_vec<<<check_blocks(n4 / 2), kCheckThreads, 0, s>>>(
             static_cast<const float4 *>(out), static_cast<const float4 *>(ref), n4,
             static_cast<const float *>(out), static_cast<const float *>(ref), n, atol, rtol, sc);
     } else {
-        int blocks = check_blocks(n);
-        if (out_dtype == KREX_BF16 && ref_dtype == KREX_F32)
-            check_generic<__nv_bfloat16, float><<<blocks, kCheckThreads, 0, s>>>(
-                static_cast<const __nv_bfloat16 *>(out), ldo, static_cast<const float *>(ref), ldr,
-                rows, cols, atol, rtol, sc);
-        else if (out_dtype == KREX_F32 && ref_dtype == KREX_F32)
-            check_generic<float, float><<<blocks, kCheckThreads, 0, s>>>(
-                static_cast<const float *>(out), ldo, static_cast<const float *>(ref), ldr, rows,
-                cols, atol, rtol, sc);
-        else if (out_dtype == KREX_BF16 && ref_dtype == KREX_BF16)
-            check_generic<__nv_bfloat16, __nv_bfloat16><<<blocks, kCheckThreads, 0, s>>>(
-                static_cast<const __nv_bfloat16 *>(out), ldo,
-                static_cast<const __nv_bfloat16 *>(ref), ldr, rows, cols, atol, rtol, sc);
-        else
-            check_generic<float, __nv_bfloat16><<<blocks, kCheckThreads, 0, s>>>(
-                static_cast<const float *>(out), ldo, static_cast<const __nv_bfloat16 *>(ref), ldr,
-                rows, cols, atol, rtol, sc);
+        launch_check_generic(out, out_dtype, ldo, ref, ref_dtype, ldr, rows, cols, atol, rtol, sc,
+                             check_blocks(n), s);
     }
     return cudaGetLastError();
 }
@@ -317,7 +353,7 @@ extern "C" krex_status krex_check_noalloc(krex_buf out, krex_buf ref, float atol
                                           krex_check_result *host_result, krex_stream_t stream) {
     using namespace krex;
     auto bad_buf = [](const krex_buf &b) {
-        return (b.dtype != KREX_BF16 && b.dtype != KREX_F32) || b.rows < 0 || b.cols < 0 ||
+        return (b.dtype != KREX_BF16 && b.dtype != KREX_F32 && b.dtype != KREX_F16) || b.rows < 0 || b.cols < 0 ||
                (b.rows > 0 && b.ld < b.cols) || (b.rows * b.cols > 0 && b.ptr == nullptr);
     };
     if (bad_buf(out) || bad_buf(ref)) return set_error(KREX_ERR_INVALID, "check_noalloc: bad out or ref buffer");

@@ -1,7 +1,7 @@
 // K7: the reference GEMM the check compares the candidate against (paper
 // Section 2.1: the command checks the candidate against a reference).  CUDA
 // cores only (the tcgen05 candidate is the only tensor-core path):
-// C[i,j] = sum_k A[i,k] B[k,j] with bf16 inputs widened exactly to fp32,
+// C[i,j] = sum_k A[i,k] B[k,j] with bf16 (or binary16) inputs widened exactly to fp32,
 // fp32 fused multiply-add accumulation in k order, fp32 output.
 //
 // Shared-memory tiling on the FP32 pipe: a 128x128 output tile per 256-thread
@@ -11,6 +11,8 @@
 // blocks at rows {ty*4, 64+ty*4} x cols {tx*4, 64+tx*4}, so its per-k operand
 // reads are four conflict-free 16-byte shared loads for 64 FMAs.  Any M, N, K;
 // loads outside the matrix read as zero and stores are guarded.
+#include <cuda_fp16.h>
+
 #include "common.cuh"
 
 namespace krex {
@@ -33,9 +35,20 @@ __device__ __forceinline__ uint4 load8(const uint16_t *__restrict__ p, int64_t l
     return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
-__device__ __forceinline__ float lo_f32(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float hi_f32(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+// Exact widening of the low / high 16-bit element of a word: bf16 is the top
+// half of an fp32; binary16 goes through the hardware conversion (exact).
+template <bool F16>
+__device__ __forceinline__ float lo_f32(uint32_t w) {
+    if constexpr (F16) return __half2float(__ushort_as_half((unsigned short)(w & 0xFFFFu)));
+    return __uint_as_float(w << 16);
+}
+template <bool F16>
+__device__ __forceinline__ float hi_f32(uint32_t w) {
+    if constexpr (F16) return __half2float(__ushort_as_half((unsigned short)(w >> 16)));
+    return __uint_as_float(w & 0xFFFF0000u);
+}
 
+template <bool F16>
 __global__ void __launch_bounds__(256)
 gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__restrict__ B, int64_t ldb,
               float *__restrict__ C, int64_t ldc, int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec,
@@ -52,12 +65,13 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
         const uint32_t wa[4] = {ua.x, ua.y, ua.z, ua.w};
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            As[nb][a_k + 2 * i][a_row] = lo_f32(wa[i]);
-            As[nb][a_k + 2 * i + 1][a_row] = hi_f32(wa[i]);
+            As[nb][a_k + 2 * i][a_row] = lo_f32<F16>(wa[i]);
+            As[nb][a_k + 2 * i + 1][a_row] = hi_f32<F16>(wa[i]);
         }
-        *reinterpret_cast<float4 *>(&Bs[nb][b_k][b_n]) = make_float4(lo_f32(ub.x), hi_f32(ub.x), lo_f32(ub.y), hi_f32(ub.y));
+        *reinterpret_cast<float4 *>(&Bs[nb][b_k][b_n]) =
+            make_float4(lo_f32<F16>(ub.x), hi_f32<F16>(ub.x), lo_f32<F16>(ub.y), hi_f32<F16>(ub.y));
         *reinterpret_cast<float4 *>(&Bs[nb][b_k][b_n + 4]) =
-            make_float4(lo_f32(ub.z), hi_f32(ub.z), lo_f32(ub.w), hi_f32(ub.w));
+            make_float4(lo_f32<F16>(ub.z), hi_f32<F16>(ub.z), lo_f32<F16>(ub.w), hi_f32<F16>(ub.w));
     };
 
     float acc[8][8];
@@ -122,13 +136,16 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
 }  // namespace
 
 cudaError_t launch_gemm_ref(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
-                            int64_t M, int64_t N, int64_t K, cudaStream_t s) {
+                            int64_t M, int64_t N, int64_t K, bool f16, cudaStream_t s) {
     if (M == 0 || N == 0) return cudaSuccess;
     const bool a_vec = ((reinterpret_cast<uintptr_t>(a) & 15u) == 0) && (lda % 8 == 0);
     const bool b_vec = ((reinterpret_cast<uintptr_t>(b) & 15u) == 0) && (ldb % 8 == 0);
     const bool c_vec = ((reinterpret_cast<uintptr_t>(c) & 15u) == 0) && (ldc % 4 == 0);
     dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
-    gemm_ref_simt<<<grid, 256, 0, s>>>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec);
+    if (f16)
+        gemm_ref_simt<true><<<grid, 256, 0, s>>>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec);
+    else
+        gemm_ref_simt<false><<<grid, 256, 0, s>>>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec);
     return cudaGetLastError();
 }
 

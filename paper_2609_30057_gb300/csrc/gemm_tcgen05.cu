@@ -23,6 +23,7 @@
 // has in flight (bounded), TMEM is freed and the kernel returns.
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cudaTypedefs.h>
 
 #include <atomic>
@@ -628,6 +629,18 @@ __device__ __forceinline__ WorkItem work_item(int w, int full_items, int tiles_m
     return it;
 }
 
+// Two fp32 values rounded (RNE) to bf16 or binary16, packed low | high << 16.
+template <bool F16>
+__device__ __forceinline__ uint32_t pack2(float lo, float hi) {
+    if constexpr (F16) {
+        __half2 h = __floats2half2_rn(lo, hi);
+        return *reinterpret_cast<uint32_t *>(&h);
+    } else {
+        __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+        return *reinterpret_cast<uint32_t *>(&h);
+    }
+}
+
 __device__ __forceinline__ void flag_store_release(uint32_t *p, uint32_t v) {
     asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
@@ -660,9 +673,10 @@ __device__ __forceinline__ void spin_ns(uint64_t ns) {
 
 // Pair tiles are 256 x bn (bn a multiple of 64, 128 <= bn <= 256); tiles_m,
 // tiles_n count them.  The host picks bn so the tiles fill whole waves.
-template <int KSUB>
+// F16: IEEE binary16 A, B and C (instruction-descriptor formats 0); else bf16.
+template <int KSUB, bool F16>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
-gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ CUtensorMap tmC, uint16_t *__restrict__ C, int64_t ldc, int M,
                       int N, int K, int bn, int tiles_m, int tiles_n, int full_items, int num_items,
                       int group_m, int c_vec, int c_tma, int stages, uint64_t timeout_ns, int split_k,
@@ -791,7 +805,8 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
         int local = 0;
         for (int w = cluster_id; ok && w < num_items; w += nclusters, ++local) {
             const WorkItem it = work_item(w, full_items, tiles_m, tiles_n, group_m, bn, num_kb, split_k);
-            const uint32_t idesc = v2::IDESC_NO_N | ((uint32_t)(it.width >> 3) << 17);
+            constexpr uint32_t idesc_ab = F16 ? (v2::IDESC_NO_N & ~((7u << 7) | (7u << 10))) : v2::IDESC_NO_N;
+            const uint32_t idesc = idesc_ab | ((uint32_t)(it.width >> 3) << 17);
             const int acc = local & 1;
             const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
             abort_flag[3] = (uint32_t)w;
@@ -926,9 +941,8 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                                 uint32_t w[4];
 #pragma unroll
                                 for (int i = 0; i < 4; ++i) {
-                                    __nv_bfloat162 hv = __floats2bfloat162_rn(__uint_as_float(v[8 * q + 2 * i]),
-                                                                              __uint_as_float(v[8 * q + 2 * i + 1]));
-                                    w[i] = *reinterpret_cast<uint32_t *>(&hv);
+                                    w[i] = pack2<F16>(__uint_as_float(v[8 * q + 2 * i]),
+                                                      __uint_as_float(v[8 * q + 2 * i + 1]));
                                 }
                                 const int j = h * 4 + q;  // 16-byte chunk of the 128-byte row
                                 *reinterpret_cast<uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
@@ -960,11 +974,8 @@ gemm_bf16_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_cons
                     if (row < M) {
                         uint32_t p[16];
 #pragma unroll
-                        for (int i = 0; i < 16; ++i) {
-                            __nv_bfloat162 h =
-                                __floats2bfloat162_rn(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
-                            p[i] = *reinterpret_cast<uint32_t *>(&h);
-                        }
+                        for (int i = 0; i < 16; ++i)
+                            p[i] = pack2<F16>(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
                         if (c_vec && col0 + 32 <= N) {
                             uint4 *dst = reinterpret_cast<uint4 *>(crow + col0);
                             dst[0] = make_uint4(p[0], p[1], p[2], p[3]);
@@ -1018,9 +1029,10 @@ struct MapKey {
     const void *ptr;
     uint64_t inner, outer, stride_bytes;
     uint32_t box_inner, box_outer;
+    bool f16;
     bool operator==(const MapKey &o) const {
-        return ptr == o.ptr && inner == o.inner && outer == o.outer &&
-               stride_bytes == o.stride_bytes && box_inner == o.box_inner && box_outer == o.box_outer;
+        return ptr == o.ptr && inner == o.inner && outer == o.outer && stride_bytes == o.stride_bytes &&
+               box_inner == o.box_inner && box_outer == o.box_outer && f16 == o.f16;
     }
 };
 struct MapKeyHash {
@@ -1028,17 +1040,19 @@ struct MapKeyHash {
         size_t h = std::hash<const void *>()(k.ptr);
         h ^= std::hash<uint64_t>()(k.inner * 0x9E3779B97F4A7C15ull + k.outer) + (h << 6) + (h >> 2);
         h ^= std::hash<uint64_t>()(k.stride_bytes ^ ((uint64_t)k.box_inner << 32 | k.box_outer)) + (h << 6);
+        h ^= (size_t)k.f16;
         return h;
     }
 };
 
-// 2-D bf16 tensor map: inner dimension contiguous, 128-byte swizzle, OOB -> 0.
-// Encoded maps are cached (a map is a pure function of its key).
+// 2-D bf16 (f16: binary16) tensor map: inner dimension contiguous, 128-byte
+// swizzle, OOB -> 0.  Encoded maps are cached (a map is a pure function of
+// its key).
 krex_status make_map(const void *ptr, uint64_t inner, uint64_t outer, uint64_t ld_elems,
-                     uint32_t box_inner, uint32_t box_outer, CUtensorMap *out) {
+                     uint32_t box_inner, uint32_t box_outer, bool f16, CUtensorMap *out) {
     static std::mutex mu;
     static std::unordered_map<MapKey, CUtensorMap, MapKeyHash> cache;
-    MapKey key{ptr, inner, outer, ld_elems * 2, box_inner, box_outer};
+    MapKey key{ptr, inner, outer, ld_elems * 2, box_inner, box_outer, f16};
     {
         std::lock_guard<std::mutex> lk(mu);
         auto it = cache.find(key);
@@ -1053,7 +1067,8 @@ krex_status make_map(const void *ptr, uint64_t inner, uint64_t outer, uint64_t l
     cuuint64_t strides[1] = {ld_elems * 2};
     cuuint32_t box[2] = {box_inner, box_outer};
     cuuint32_t estr[2] = {1, 1};
-    CUresult r = enc(out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides,
+    CUresult r = enc(out, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                     const_cast<void *>(ptr), dims, strides,
                      box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                      CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS)
@@ -1142,7 +1157,7 @@ constexpr size_t WS_BYTES = WS_PARTIAL_BYTES + 2 * WS_SLABS * sizeof(uint32_t);
 size_t gemm_workspace_bytes() { return WS_BYTES; }
 
 krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb,
-                                uint16_t *c, int64_t ldc, int64_t M, int64_t N, int64_t K,
+                                uint16_t *c, int64_t ldc, int64_t M, int64_t N, int64_t K, bool f16,
                                 void *workspace, size_t workspace_bytes, cudaStream_t s) {
     if (M == 0 || N == 0) return KREX_OK;
     if (K == 0) {
@@ -1164,9 +1179,9 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         }
     }
     CUtensorMap ma, mb;
-    krex_status st = make_map(a, (uint64_t)K, (uint64_t)M, (uint64_t)lda, BK, BM, &ma);
+    krex_status st = make_map(a, (uint64_t)K, (uint64_t)M, (uint64_t)lda, BK, BM, f16, &ma);
     if (st != KREX_OK) return st;
-    st = make_map(b, (uint64_t)N, (uint64_t)K, (uint64_t)ldb, B_BOX_N, BK, &mb);
+    st = make_map(b, (uint64_t)N, (uint64_t)K, (uint64_t)ldb, B_BOX_N, BK, f16, &mb);
     if (st != KREX_OK) return st;
 
     static thread_local int attr_dev = -1;
@@ -1176,9 +1191,13 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
     if (attr_dev != dev) {
         KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)SMEM_BYTES));
-        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05_2sm<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)v2::Cfg<1>::SMEM_BYTES));
-        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05_2sm<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)v2::Cfg<2>::SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)v2::Cfg<1>::SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)v2::Cfg<2>::SMEM_BYTES));
         // co-resident CTA pairs; a persistent grid larger than this would only queue
         cudaLaunchConfig_t cfg = {};
@@ -1186,7 +1205,7 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         cfg.blockDim = dim3(THREADS, 1, 1);
         cfg.dynamicSmemBytes = v2::Cfg<2>::SMEM_BYTES;
         int n = 0;
-        if (cudaOccupancyMaxActiveClusters(&n, gemm_bf16_tcgen05_2sm<2>, &cfg) != cudaSuccess || n <= 0) {
+        if (cudaOccupancyMaxActiveClusters(&n, gemm_tcgen05_2sm<2, false>, &cfg) != cudaSuccess || n <= 0) {
             cudaGetLastError();
             n = sm_count() / 2;
         }
@@ -1194,12 +1213,12 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         attr_dev = dev;
     }
     const int c_vec = ((reinterpret_cast<uintptr_t>(c) & 15u) == 0) && (ldc % 8 == 0);
-    if (gemm_variant() == 2) {
+    if (gemm_variant() == 2 || f16) {  // the 1-SM form is bf16 only
         // TMA-store epilogue when C rows start on 16 bytes; else direct stores
         CUtensorMap mc;
         int c_tma = c_vec;
         if (c_tma) {
-            st = make_map(c, (uint64_t)N, (uint64_t)M, (uint64_t)ldc, v2::EPI_BOX_COLS, 32, &mc);
+            st = make_map(c, (uint64_t)N, (uint64_t)M, (uint64_t)ldc, v2::EPI_BOX_COLS, 32, f16, &mc);
             if (st != KREX_OK) return st;
         } else {
             mc = ma;  // unused
@@ -1233,16 +1252,21 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         uint32_t *ws_count =
             split_k ? reinterpret_cast<uint32_t *>(static_cast<uint8_t *>(workspace) + WS_PARTIAL_BYTES) : nullptr;
         uint32_t *ws_flag = split_k ? ws_count + WS_SLABS : nullptr;
-        if (ksub == 2)
-            gemm_bf16_tcgen05_2sm<2><<<2 * clusters, THREADS, v2::Cfg<2>::SMEM_BYTES, s>>>(
-                ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, (int)full_items, (int)items,
-                raster_group(), c_vec, c_tma, ring_stages(v2::Cfg<2>::STAGES), wait_timeout_ns(), split_k, ws_partial,
-                ws_count, ws_flag, launch_id);
+        auto go = [&](auto kernel, size_t smem, int stages) {
+            kernel<<<2 * clusters, THREADS, smem, s>>>(ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m,
+                                                       tiles_n, (int)full_items, (int)items, raster_group(), c_vec,
+                                                       c_tma, stages, wait_timeout_ns(), split_k, ws_partial,
+                                                       ws_count, ws_flag, launch_id);
+        };
+        const int st2 = ring_stages(v2::Cfg<2>::STAGES), st1 = ring_stages(v2::Cfg<1>::STAGES);
+        if (ksub == 2 && f16)
+            go(gemm_tcgen05_2sm<2, true>, v2::Cfg<2>::SMEM_BYTES, st2);
+        else if (ksub == 2)
+            go(gemm_tcgen05_2sm<2, false>, v2::Cfg<2>::SMEM_BYTES, st2);
+        else if (f16)
+            go(gemm_tcgen05_2sm<1, true>, v2::Cfg<1>::SMEM_BYTES, st1);
         else
-            gemm_bf16_tcgen05_2sm<1><<<2 * clusters, THREADS, v2::Cfg<1>::SMEM_BYTES, s>>>(
-                ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m, tiles_n, (int)full_items, (int)items,
-                raster_group(), c_vec, c_tma, ring_stages(v2::Cfg<1>::STAGES), wait_timeout_ns(), split_k, ws_partial,
-                ws_count, ws_flag, launch_id);
+            go(gemm_tcgen05_2sm<1, false>, v2::Cfg<1>::SMEM_BYTES, st1);
     } else {
         const int tiles_m = (int)((M + BM - 1) / BM), tiles_n = (int)((N + BN - 1) / BN);
         const int64_t tiles = (int64_t)tiles_m * tiles_n;

@@ -4,7 +4,7 @@ host copies of bf16 tensors as bit patterns."""
 import numpy as np
 import torch
 
-SENTINEL = {torch.bfloat16: 0x7FA5, torch.float32: 0x7FA5A5A5}
+SENTINEL = {torch.bfloat16: 0x7FA5, torch.float16: 0x7FA5, torch.float32: 0x7FA5A5A5}
 
 
 class Guarded:
@@ -16,14 +16,14 @@ class Guarded:
         self.ld = cols if ld is None else ld
         self.pad = pad_elems
         n = self.pad * 2 + max(rows * self.ld, 1)
-        itype = torch.int16 if dtype == torch.bfloat16 else torch.int32
+        itype = torch.int16 if dtype in (torch.bfloat16, torch.float16) else torch.int32
         self._sent = SENTINEL[dtype]            # positive, fits the signed type
         self.base = torch.full((n,), self._sent, dtype=itype, device="cuda").view(dtype)
         flat = self.base[self.pad:self.pad + rows * self.ld]
         self.view = flat.view(rows, self.ld)[:, :cols]
 
     def canaries_intact(self) -> bool:
-        itype = torch.int16 if self.dtype == torch.bfloat16 else torch.int32
+        itype = torch.int16 if self.dtype in (torch.bfloat16, torch.float16) else torch.int32
         raw = self.base.view(itype).cpu().numpy()
         mask = np.ones(raw.size, dtype=bool)
         for r in range(self.rows):
@@ -38,3 +38,7 @@ def bits16(t: torch.Tensor) -> np.ndarray:
 
 def to_bf16_tensor(bits: np.ndarray) -> torch.Tensor:
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def to_f16_tensor(bits: np.ndarray) -> torch.Tensor:
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.float16).cuda()

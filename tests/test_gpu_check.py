@@ -9,7 +9,7 @@ import torch
 
 import paper_2609_30057_gb300 as krex
 import inputs
-from gpu_util import Guarded, to_bf16_tensor
+from gpu_util import Guarded, to_bf16_tensor, to_f16_tensor
 from oracle import gen, ref
 
 pytestmark = pytest.mark.gpu
@@ -21,12 +21,25 @@ def scratch():
     return torch.empty(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
 
 
+class F16Bits(np.ndarray):
+    """uint16 binary16 bit patterns (plain uint16 arrays are bf16)."""
+
+
+def _f16(bits):
+    return np.asarray(bits, dtype=np.uint16).view(F16Bits)
+
+
 def _f32_of(bits_or_f32):
-    a = np.asarray(bits_or_f32)
+    a = bits_or_f32
+    if isinstance(a, F16Bits):
+        return gen.f16_to_f32(np.asarray(a).view(np.ndarray))
+    a = np.asarray(a)
     return gen.bf16_to_f32(a) if a.dtype == np.uint16 else a.astype(np.float32)
 
 
 def _dev(a):
+    if isinstance(a, F16Bits):
+        return to_f16_tensor(np.asarray(a).view(np.ndarray))
     a = np.asarray(a)
     return to_bf16_tensor(a) if a.dtype == np.uint16 else torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
@@ -106,3 +119,17 @@ def test_check_full_size(shape, pair, scratch):
     o = inputs.bf16_bits_from_f32(o32) if pair == "bf16_f32" else o32
     atol, rtol = (2.0 ** -12 * math.sqrt(shape[0]), 2.0 ** -7) if pair == "bf16_f32" else (1e-6, 0.0)
     _run(o, r32, atol, rtol, scratch)
+
+
+@pytest.mark.parametrize("n", [1, 9, 4097, 100003])
+@pytest.mark.parametrize("pair", ["f16_f32", "f16_f16", "f32_f16", "f16_bf16"])
+def test_check_f16_pairs_match_oracle(n, pair, scratch):
+    r32 = inputs.normal_f32(n + 5, (1, n))
+    o32 = inputs.perturbed(r32, n + 6, 0.3, 0.05)
+    conv = {"f16": lambda x: _f16(gen.f32_to_f16(x.ravel()).reshape(x.shape)),
+            "bf16": inputs.bf16_bits_from_f32, "f32": lambda x: x}
+    po, pr = pair.split("_")
+    o, r = conv[po](o32), conv[pr](r32)
+    for atol, rtol in ((1e-2, 1e-2), (2.0 ** -12 * 64, 2.0 ** -10), (0.0, 0.0)):
+        _run(o, r, atol, rtol, scratch)
+

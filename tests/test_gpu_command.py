@@ -71,3 +71,16 @@ def test_failing_check_skips_the_timed_loop():
     ws.cmd.rtol = 0.0
     res = ws.run()
     assert res.passed == 0 and res.n_iters == 0 and res.check.n_violations == w.M * w.N
+
+
+def test_f16_gemm_command_matches_oracle():
+    w = scaled(WORKLOADS["gemm_f16_4096"], name="gemm_f16_512", M=512, N=768, K=1024, iters=10)
+    ws = Workspace(w)
+    res = ws.run()
+    assert res.passed == 1 and res.check.n_violations == 0
+    assert res.n_iters == w.iters and res.p50_ms > 0
+    want = ref.gemm_f64(gen.uniform_f16(w.seed, 0, w.M, w.K), gen.uniform_f16(w.seed, 1, w.K, w.N), dtype="f16")
+    got = gen.f16_to_f32(bits16(ws.out)).astype(np.float64)
+    assert np.all(np.abs(got - want) <= ref.gemm_tolerance(want, w.K, dtype="f16"))
+    assert np.array_equal(bits16(ws.inputs[0]), gen.uniform_f16(w.seed, 0, w.M, w.K))
+

@@ -9,7 +9,7 @@ import pytest
 import torch
 
 import paper_2609_30057_gb300 as krex
-from gpu_util import Guarded, bits16, to_bf16_tensor
+from gpu_util import Guarded, bits16, to_bf16_tensor, to_f16_tensor
 import inputs
 from oracle import gen, ref
 
@@ -271,3 +271,103 @@ def test_2sm_ragged_edge_items_under_contention():
     want = ref.gemm_f64(gen.uniform_bf16(2064, 0, n, n), gen.uniform_bf16(2064, 1, n, n))
     ok, worst = _within_tol(bits16(c), want, n)
     assert ok, worst
+
+
+# ------------------------------------------------------------- fp16 GEMM ----
+
+def _gen16(seed, M, N, K):
+    a = torch.empty(M, K, dtype=torch.float16, device="cuda")
+    b = torch.empty(K, N, dtype=torch.float16, device="cuda")
+    krex.krex_gen_inputs(seed, 0, krex.KREX_DIST_UNIFORM_PM1, 0.0, a)
+    krex.krex_gen_inputs(seed, 1, krex.KREX_DIST_UNIFORM_PM1, 0.0, b)
+    return a, b
+
+
+def _candidate16(a, b, ws=None):
+    M, N = a.shape[0], b.shape[1]
+    c = Guarded(M, N, torch.float16)
+    if ws is None:
+        krex.krex_run_candidate(krex.KREX_OP_GEMM_F16, [a, b], c.view)
+    else:
+        krex.krex_run_candidate_ws(krex.KREX_OP_GEMM_F16, [a, b], c.view, ws)
+    torch.cuda.synchronize()
+    assert krex.krex_device_status() == 0
+    assert c.canaries_intact()
+    return c.view
+
+
+def _within_tol16(got_bits, want64, K):
+    got = gen.f16_to_f32(got_bits).astype(np.float64)
+    tol = ref.gemm_tolerance(want64, K, dtype="f16")
+    err = np.abs(got - want64)
+    return np.all(err <= tol), float(np.max(err / tol))
+
+
+@pytest.mark.parametrize("ksub", ["2", "1"])
+def test_f16_identity_and_permutation_are_exact(ksub, monkeypatch):
+    monkeypatch.setenv("KREX_GEMM_KSUB", ksub)
+    a, _ = _gen16(1, 256, 384, 384)
+    eye = to_f16_tensor(gen.f32_to_f16(inputs.identity(384).ravel()).reshape(384, 384))
+    assert np.array_equal(bits16(_candidate16(a, eye)), bits16(a))
+    p, perm = inputs.permutation_matrix(384, 9)
+    pt = to_f16_tensor(gen.f32_to_f16(p.ravel()).reshape(384, 384))
+    assert np.array_equal(bits16(_candidate16(a, pt)), bits16(a)[:, perm])
+
+
+def test_f16_small_integers_are_exact():
+    # integer products summed exactly in fp32; |C| < 2048 is exact in binary16
+    M, N, K = 256, 512, 64
+    g = inputs.rng(5)
+    a = g.integers(-4, 5, (M, K)).astype(np.float32)
+    b = g.integers(-4, 5, (K, N)).astype(np.float32)
+    ah, bh = gen.f32_to_f16(a.ravel()).reshape(M, K), gen.f32_to_f16(b.ravel()).reshape(K, N)
+    c = _candidate16(to_f16_tensor(ah), to_f16_tensor(bh))
+    want = ref.gemm_f64(ah, bh, dtype="f16")
+    assert np.array_equal(gen.f16_to_f32(bits16(c)).astype(np.float64), want)
+
+
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (100, 72, 40), (300, 1000, 520), (1024, 2048, 512),
+                                   (640, 384, 4104), (2064, 1000, 1032), (4096, 4096, 4096)])
+def test_f16_seeded_gemm_within_tolerance(M, N, K):
+    seed = 7000 + M + N + K
+    a, b = _gen16(seed, M, N, K)
+    want = ref.gemm_f64(gen.uniform_f16(seed, 0, M, K), gen.uniform_f16(seed, 1, K, N), dtype="f16")
+    for ws in (None, krex.gemm_workspace()):          # column halves / K halves in the tail
+        ok, worst = _within_tol16(bits16(_candidate16(a, b, ws)), want, K)
+        assert ok, worst
+
+
+def test_f16_large_sampled():
+    n, seed = 8192, 4
+    a, b = _gen16(seed, n, n, n)
+    c = torch.empty(n, n, dtype=torch.float16, device="cuda")
+    krex.krex_run_candidate(krex.KREX_OP_GEMM_F16, [a, b], c)
+    torch.cuda.synchronize()
+    assert krex.krex_device_status() == 0
+    i, j = ref.sample_indices(seed, 2, 4096, n, n)
+    got = bits16(c[torch.from_numpy(i).cuda(), torch.from_numpy(j).cuda()])
+    want = ref.gemm_sampled_f64(seed, n, n, n, i, j, dtype="f16")
+    ok, worst = _within_tol16(got, want, n)
+    assert ok, worst
+
+
+@pytest.mark.parametrize("M,N,K", [(256, 256, 256), (300, 1000, 520)])
+def test_f16_reference_gemm_within_fp32_bound(M, N, K):
+    seed = 88 + M
+    a, b = _gen16(seed, M, N, K)
+    r = Guarded(M, N, torch.float32)
+    krex.krex_run_reference(krex.KREX_OP_GEMM_F16, [a, b], r.view)
+    torch.cuda.synchronize()
+    assert r.canaries_intact()
+    ah, bh = gen.uniform_f16(seed, 0, M, K), gen.uniform_f16(seed, 1, K, N)
+    want = ref.gemm_f64(ah, bh, dtype="f16")
+    absab = np.abs(gen.f16_to_f32(ah).astype(np.float64)) @ np.abs(gen.f16_to_f32(bh).astype(np.float64))
+    assert np.all(np.abs(r.view.cpu().numpy() - want) <= (K + 2) * 2.0 ** -24 * absab + 1e-30)
+
+
+def test_f16_op_rejects_bf16_operands():
+    a = torch.zeros(16, 16, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(krex.KrexError, match="INVALID"):
+        krex.krex_run_candidate(krex.KREX_OP_GEMM_F16, [a, a], torch.empty(16, 16, dtype=torch.float16,
+                                                                               device="cuda"))
+

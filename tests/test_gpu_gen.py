@@ -96,3 +96,31 @@ def test_normal_softmax_input_sampled_bitexact():
     i, _ = ref.sample_indices(3, 9, 1 << 20, rows * cols, 1)
     idx = np.concatenate([i, np.arange(cols), np.arange(rows * cols - cols, rows * cols)])
     assert np.array_equal(host[idx].view(np.uint32), gen.normal_f32_at(3, 0, idx, 2.0).view(np.uint32))
+
+
+@pytest.mark.parametrize("rows,cols", SHAPES)
+def test_uniform_f16_bitexact_contiguous(rows, cols):
+    g = Guarded(rows, cols, torch.float16)
+    krex.krex_gen_inputs(7, 1, krex.KREX_DIST_UNIFORM_PM1, 0.0, g.view)
+    torch.cuda.synchronize()
+    assert np.array_equal(bits16(g.view), gen.uniform_f16(7, 1, rows, cols))
+    assert g.canaries_intact()
+
+
+@pytest.mark.parametrize("rows,cols,ld", [(5, 16, 24), (6, 7, 9)])
+def test_uniform_f16_bitexact_strided(rows, cols, ld):
+    g = Guarded(rows, cols, torch.float16, ld=ld)
+    krex.krex_gen_inputs(11, 0, krex.KREX_DIST_UNIFORM_PM1, 0.0, g.view)
+    torch.cuda.synchronize()
+    assert np.array_equal(bits16(g.view), gen.uniform_f16(11, 0, rows, cols))
+    assert g.canaries_intact()
+
+
+def test_uniform_f16_full_size_sampled():
+    # the 4096 x 4096 operand of the fp16 GEMM workload, on seeded samples
+    # (the oracle's gather form) plus the subnormal share
+    t = torch.empty(4096, 4096, dtype=torch.float16, device="cuda")
+    krex.krex_gen_inputs(2, 0, krex.KREX_DIST_UNIFORM_PM1, 0.0, t)
+    torch.cuda.synchronize()
+    idx = ref.sample_indices(2, 4, 65536, 4096 * 4096)[0]
+    assert np.array_equal(bits16(t).ravel()[idx], gen.uniform_f16_at(2, 0, idx))
