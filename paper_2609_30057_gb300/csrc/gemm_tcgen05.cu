@@ -919,10 +919,26 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                 // buffer (row = lane, 16-byte chunk j at j ^ (lane % 8)) -> one TMA store of
                 // the 32 x 64 box; two buffers per warp alternate.
                 if (row0 < M) {
+                    // The other K half's partials (split-K) are read one 64-column
+                    // chunk ahead, so their L2 round trips overlap this chunk's work
+                    // instead of adding one per 32 columns.
+                    constexpr int PC = v2::EPI_BOX_COLS;
+                    float pnext[PC];
+                    if (add) {
+#pragma unroll
+                        for (int i = 0; i < PC; ++i) pnext[i] = __ldcg(add + i * 32 + lane);
+                    }
 #pragma unroll 1
                     for (int c = 0; c < width / v2::EPI_BOX_COLS; ++c) {
                         const int col0 = n0 + c * v2::EPI_BOX_COLS;
                         if (col0 >= N) break;  // warp-uniform
+                        float pcur[PC];
+#pragma unroll
+                        for (int i = 0; i < PC; ++i) pcur[i] = pnext[i];
+                        if (add && c + 1 < width / v2::EPI_BOX_COLS) {
+#pragma unroll
+                            for (int i = 0; i < PC; ++i) pnext[i] = __ldcg(add + ((c + 1) * PC + i) * 32 + lane);
+                        }
                         uint8_t *buf = sEpi + (ew * 2 + (epi_buf & 1)) * v2::EPI_BUF_BYTES;
                         if (lane == 0) bulk_wait_group_read<1>();  // the store that used `buf` has read it
                         __syncwarp();
@@ -931,10 +947,9 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                             uint32_t v[32];
                             tmem_ld32(tbase + (uint32_t)(c * v2::EPI_BOX_COLS + h * 32), v);
                             if (add) {
-                                const float *pc = add + (c * v2::EPI_BOX_COLS + h * 32) * 32 + lane;
 #pragma unroll
                                 for (int i = 0; i < 32; ++i)
-                                    v[i] = __float_as_uint(__uint_as_float(v[i]) + __ldcg(pc + i * 32));
+                                    v[i] = __float_as_uint(__uint_as_float(v[i]) + pcur[h * 32 + i]);
                             }
 #pragma unroll
                             for (int q = 0; q < 4; ++q) {
@@ -1239,8 +1254,10 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         // K has at least two ring stages and the split tiles are the whole
         // GEMM (one partial wave); else column halves.  Measured on GB300: K
         // halves load a third less than column halves (1024 x 2048 x 8192:
-        // 8 % faster), but the partial sums' hand-over sits on the last wave's
-        // critical path (4096^3, 28 of 256 tiles split: 2 % slower).
+        // 49 -> 44 us), but the hand-over of the fp32 partials (128 KiB per CTA
+        // written, then read) sits on the last wave's critical path: at 4096^3
+        // the K halves end their MMAs 6.8 us earlier and spend about as long
+        // exchanging partials, so the multi-wave case gains nothing.
         const int ksub = stage_ksub();
         const int64_t num_kb = (((K + 63) / 64) + ksub - 1) / ksub;
         const int split_k = split && full_items == 0 && workspace && workspace_bytes >= WS_BYTES &&
