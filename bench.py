@@ -251,6 +251,14 @@ def oracle_command_cost(w, budget_s: float = 10.0):
     return total, info
 
 
+def _p95(xs) -> float:
+    """Linear-interpolation percentile 0.95 (the percentile method of the timed loop)."""
+    v = sorted(xs)
+    h = (len(v) - 1) * 0.95
+    lo = int(h)
+    return v[lo] if lo + 1 >= len(v) else v[lo] + (h - lo) * (v[lo + 1] - v[lo])
+
+
 def cpu_cores() -> int:
     return len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
 
@@ -373,15 +381,23 @@ def main():
 
     # ------------------------------------------------ roofline (GEMM kernel)
     mean_gemm_ms = statistics.fmean(gemm_ms)
-    achieved = w.flops / (mean_gemm_ms / 1e3) / 1e12
-    traffic = _ncu_traffic("gemm_tcgen05", w.name)
-    roofline = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                "frac": achieved / peaks["bf16_tflops"], "traffic": traffic,
-                "peak_kind": f"bf16 dense burst, {peaks['source']} (MEASURED_PEAKS.json)",
-                "frac_of_sustained": (achieved / peaks["bf16_tflops_sustained"]
-                                      if peaks.get("bf16_tflops_sustained") else None),
-                "kernel": "gemm_bf16_tcgen05", "launches_timed": len(gemm_ms),
-                "algorithmic_flops_per_launch": w.flops}
+    if w.is_gemm:
+        achieved = w.flops / (mean_gemm_ms / 1e3) / 1e12
+        roofline = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                    "frac": achieved / peaks["bf16_tflops"], "traffic": _ncu_traffic("gemm_tcgen05", w.name),
+                    "peak_kind": f"bf16 dense burst, {peaks['source']} (MEASURED_PEAKS.json)",
+                    "frac_of_sustained": (achieved / peaks["bf16_tflops_sustained"]
+                                          if peaks.get("bf16_tflops_sustained") else None),
+                    "kernel": "gemm_tcgen05_2sm", "launches_timed": len(gemm_ms),
+                    "algorithmic_flops_per_launch": w.flops}
+    else:
+        # the bandwidth-bound candidate: one read and one write of the matrix
+        achieved = w.candidate_bytes / (mean_gemm_ms / 1e3) / 1e9
+        roofline = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                    "frac": achieved / peaks["hbm_gbs"], "traffic": _ncu_traffic("softmax_rows", w.name),
+                    "peak_kind": f"HBM copy, {peaks['source']} (MEASURED_PEAKS.json)",
+                    "kernel": "softmax_rows_reg", "launches_timed": len(gemm_ms),
+                    "algorithmic_bytes_per_launch": w.candidate_bytes}
 
     cpu = None
     if not args.no_cpu_baseline:
@@ -393,7 +409,7 @@ def main():
     line = {
         "metric": METRIC, "value": value, "unit": "cmds/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "scaling": "weak", "vs_baseline": None, "dtype": {"bf16": "bf16", "f16": "f16"}.get(w.dtype, "f32"), "data": "synthetic",
         "config": {"workload": w.name, "M": w.M, "N": w.N, "K": w.K, "seed": w.seed, "timed_iters": w.iters,
                    "warmup_iters": w.warmup, "flush_bytes": w.flush_bytes,
                    "l2": "flushed: a flush_bytes write precedes every timed candidate iteration and region entry",
@@ -404,7 +420,9 @@ def main():
         "gpu_launches": launches,
         "clocks": cs,
         "timing_spread": {"p50_ms_median": statistics.median(p50s), "p95_ms_median": statistics.median(p95s),
-                          "p95_over_p50_minus_1": statistics.median(p95s) / statistics.median(p50s) - 1.0},
+                          "p95_over_p50_minus_1": statistics.median(p95s) / statistics.median(p50s) - 1.0,
+                          # Eq. 1 across the commands: p95 of (command median / overall median) - 1
+                          "P_across_commands": _p95([p / statistics.median(p50s) for p in p50s]) - 1.0},
         "phase_ms": dict(zip(["inputs", "reference", "candidate", "check", "timed_loop"], ph)),
         "kernels": kernels,
         "host_wall_s": wall,
