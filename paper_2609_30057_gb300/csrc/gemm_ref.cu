@@ -4,24 +4,27 @@
 // C[i,j] = sum_k A[i,k] B[k,j] with bf16 (or binary16) inputs widened exactly to fp32,
 // fp32 fused multiply-add accumulation in k order, fp32 output.
 //
-// Shared-memory tiling on the FP32 pipe: a 128x128 output tile per 256-thread
-// block, K in slices of 16 staged as fp32 in two shared-memory buffers (the
-// next slice is fetched from global memory into registers while the current
-// one is multiplied).  Each thread owns an 8x8 block made of the four 4x4
-// blocks at rows {ty*4, 64+ty*4} x cols {tx*4, 64+tx*4}, so its per-k operand
-// reads are four conflict-free 16-byte shared loads for 64 FMAs.  Any M, N, K;
-// loads outside the matrix read as zero and stores are guarded.
+// Shared-memory tiling on the FP32 pipe: a 128 x (64*NG) output tile per
+// 256-thread block, K in slices of TK staged as fp32 in two shared-memory
+// buffers (the next slice is fetched from global memory into registers while
+// the current one is multiplied).  Each thread owns an 8 x (4*NG) block made
+// of 4x4 blocks at rows {ty*4, 64+ty*4} x cols {g*64 + tx*4 : g < NG}, so its
+// per-k operand reads are conflict-free 16-byte shared loads (two for A, NG
+// for B) for 32*NG FMAs.  Any M, N, K; loads outside the matrix read as zero
+// and stores are guarded.
 #include <cuda_fp16.h>
+
+#include <cstdlib>
 
 #include "common.cuh"
 
 namespace krex {
 namespace {
 
-constexpr int TM = 128, TN = 128, TK = 16;
+constexpr int TM = 128;
 
-// 8 consecutive bf16 at (r, c..c+7) of a row-major matrix as raw 16-bit words
-// packed in a uint4, zero outside [0,R)x[0,C).
+// 8 consecutive 16-bit elements at (r, c..c+7) of a row-major matrix as raw
+// words packed in a uint4, zero outside [0,R)x[0,C).
 __device__ __forceinline__ uint4 load8(const uint16_t *__restrict__ p, int64_t ld, int64_t R, int64_t C, int64_t r,
                                        int64_t c, bool vec_ok) {
     if (vec_ok && r < R && c + 8 <= C) return __ldg(reinterpret_cast<const uint4 *>(p + r * ld + c));
@@ -48,66 +51,102 @@ __device__ __forceinline__ float hi_f32(uint32_t w) {
     return __uint_as_float(w & 0xFFFF0000u);
 }
 
-template <bool F16>
-__global__ void __launch_bounds__(256)
+// NG: 64-column groups per block (tile 128 x 64*NG); TK: K per shared slice;
+// MINB: resident blocks per SM the register budget is sized for.
+template <bool F16, int NG, int TK, int MINB>
+__global__ void __launch_bounds__(256, MINB)
 gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__restrict__ B, int64_t ldb,
               float *__restrict__ C, int64_t ldc, int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec,
               bool c_vec) {
-    __shared__ __align__(16) float As[2][TK][TM];  // As[buf][k][m]
-    __shared__ __align__(16) float Bs[2][TK][TN];  // Bs[buf][k][n]
+    constexpr int TN = 64 * NG;
+    constexpr int A_LOADS = TM * TK / 8 / 256;  // uint4 (8 elements) per thread and slice
+    constexpr int B_LOADS = TK * TN / 8 / 256;
+    static_assert(A_LOADS >= 1 && B_LOADS >= 1, "slice too small for 256 threads");
+    extern __shared__ __align__(16) float smem[];
+    float *As = smem;                  // [2][TK][TM]
+    float *Bs = smem + 2 * TK * TM;    // [2][TK][TN]
     const int t = threadIdx.x;
     const int tx = t & 15, ty = t >> 4;
     const int64_t m0 = (int64_t)blockIdx.y * TM, n0 = (int64_t)blockIdx.x * TN;
-    // load slots: A row t/2, k (t&1)*8..+7; B k-row t/16, cols (t&15)*8..+7
-    const int a_row = t >> 1, a_k = (t & 1) * 8;
-    const int b_k = t >> 4, b_n = (t & 15) * 8;
-    auto stage = [&](int nb, const uint4 &ua, const uint4 &ub) {
-        const uint32_t wa[4] = {ua.x, ua.y, ua.z, ua.w};
+    // load slots s = t + 256 i: A row s / (TK/8), k offset 8 (s % (TK/8));
+    //                           B k-row s / (TN/8), cols 8 (s % (TN/8))
+    uint4 ua[A_LOADS], ub[B_LOADS];
+    auto fetch = [&](int64_t k0) {
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            As[nb][a_k + 2 * i][a_row] = lo_f32<F16>(wa[i]);
-            As[nb][a_k + 2 * i + 1][a_row] = hi_f32<F16>(wa[i]);
+        for (int i = 0; i < A_LOADS; ++i) {
+            const int s = t + 256 * i;
+            ua[i] = load8(A, lda, M, K, m0 + s / (TK / 8), k0 + 8 * (s % (TK / 8)), a_vec);
         }
-        *reinterpret_cast<float4 *>(&Bs[nb][b_k][b_n]) =
-            make_float4(lo_f32<F16>(ub.x), hi_f32<F16>(ub.x), lo_f32<F16>(ub.y), hi_f32<F16>(ub.y));
-        *reinterpret_cast<float4 *>(&Bs[nb][b_k][b_n + 4]) =
-            make_float4(lo_f32<F16>(ub.z), hi_f32<F16>(ub.z), lo_f32<F16>(ub.w), hi_f32<F16>(ub.w));
+#pragma unroll
+        for (int i = 0; i < B_LOADS; ++i) {
+            const int s = t + 256 * i;
+            ub[i] = load8(B, ldb, K, N, k0 + s / (TN / 8), n0 + 8 * (s % (TN / 8)), b_vec);
+        }
+    };
+    auto stage = [&](int nb) {
+        float *as = As + nb * TK * TM;
+        float *bs = Bs + nb * TK * TN;
+#pragma unroll
+        for (int i = 0; i < A_LOADS; ++i) {
+            const int s = t + 256 * i;
+            const int row = s / (TK / 8), kk = 8 * (s % (TK / 8));
+            const uint32_t wa[4] = {ua[i].x, ua[i].y, ua[i].z, ua[i].w};
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                as[(kk + 2 * j) * TM + row] = lo_f32<F16>(wa[j]);
+                as[(kk + 2 * j + 1) * TM + row] = hi_f32<F16>(wa[j]);
+            }
+        }
+#pragma unroll
+        for (int i = 0; i < B_LOADS; ++i) {
+            const int s = t + 256 * i;
+            const int kr = s / (TN / 8), col = 8 * (s % (TN / 8));
+            float *dst = bs + kr * TN + col;
+            *reinterpret_cast<float4 *>(dst) =
+                make_float4(lo_f32<F16>(ub[i].x), hi_f32<F16>(ub[i].x), lo_f32<F16>(ub[i].y), hi_f32<F16>(ub[i].y));
+            *reinterpret_cast<float4 *>(dst + 4) =
+                make_float4(lo_f32<F16>(ub[i].z), hi_f32<F16>(ub[i].z), lo_f32<F16>(ub[i].w), hi_f32<F16>(ub[i].w));
+        }
     };
 
-    float acc[8][8];
+    float acc[8][4 * NG];
 #pragma unroll
     for (int i = 0; i < 8; ++i)
 #pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
+        for (int j = 0; j < 4 * NG; ++j) acc[i][j] = 0.0f;
 
-    uint4 ua = load8(A, lda, M, K, m0 + a_row, a_k, a_vec);
-    uint4 ub = load8(B, ldb, K, N, b_k, n0 + b_n, b_vec);
-    stage(0, ua, ub);
+    fetch(0);
+    stage(0);
     __syncthreads();
 
     int buf = 0;
     for (int64_t k0 = 0; k0 < K; k0 += TK) {
         const bool more = k0 + TK < K;
-        if (more) {  // fetch the next slice while this one is multiplied
-            ua = load8(A, lda, M, K, m0 + a_row, k0 + TK + a_k, a_vec);
-            ub = load8(B, ldb, K, N, k0 + TK + b_k, n0 + b_n, b_vec);
-        }
+        if (more) fetch(k0 + TK);  // the next slice comes in while this one is multiplied
+        const float *as = As + buf * TK * TM;
+        const float *bs = Bs + buf * TK * TN;
 #pragma unroll
         for (int k = 0; k < TK; ++k) {
-            const float4 a0 = *reinterpret_cast<const float4 *>(&As[buf][k][ty * 4]);
-            const float4 a1 = *reinterpret_cast<const float4 *>(&As[buf][k][64 + ty * 4]);
-            const float4 b0 = *reinterpret_cast<const float4 *>(&Bs[buf][k][tx * 4]);
-            const float4 b1 = *reinterpret_cast<const float4 *>(&Bs[buf][k][64 + tx * 4]);
+            const float4 a0 = *reinterpret_cast<const float4 *>(as + k * TM + ty * 4);
+            const float4 a1 = *reinterpret_cast<const float4 *>(as + k * TM + 64 + ty * 4);
+            float b[4 * NG];
+#pragma unroll
+            for (int g = 0; g < NG; ++g) {
+                const float4 bg = *reinterpret_cast<const float4 *>(bs + k * TN + g * 64 + tx * 4);
+                b[4 * g] = bg.x;
+                b[4 * g + 1] = bg.y;
+                b[4 * g + 2] = bg.z;
+                b[4 * g + 3] = bg.w;
+            }
             const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-            const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
 #pragma unroll
             for (int i = 0; i < 8; ++i)
 #pragma unroll
-                for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+                for (int j = 0; j < 4 * NG; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
         }
         if (more) {
             const int nb = buf ^ 1;
-            stage(nb, ua, ub);
+            stage(nb);
             __syncthreads();
             buf = nb;
         }
@@ -119,9 +158,9 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
         if (r >= M) continue;
         float *cr = C + r * ldc;
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int64_t c = n0 + h * 64 + tx * 4;
-            const float *v = &acc[i][4 * h];
+        for (int g = 0; g < NG; ++g) {
+            const int64_t c = n0 + g * 64 + tx * 4;
+            const float *v = &acc[i][4 * g];
             if (c_vec && c + 4 <= N) {
                 *reinterpret_cast<float4 *>(cr + c) = make_float4(v[0], v[1], v[2], v[3]);
             } else {
@@ -133,6 +172,47 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
     }
 }
 
+template <bool F16, int NG, int TK, int MINB>
+cudaError_t launch_cfg(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
+                       int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c_vec, cudaStream_t s) {
+    constexpr int TN = 64 * NG;
+    constexpr size_t smem = (size_t)2 * TK * (TM + TN) * sizeof(float);
+    static const cudaError_t attr = cudaFuncSetAttribute(
+        gemm_ref_simt<F16, NG, TK, MINB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (attr != cudaSuccess) return attr;
+    dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
+    gemm_ref_simt<F16, NG, TK, MINB><<<grid, 256, smem, s>>>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec);
+    return cudaGetLastError();
+}
+
+// Tiling of the reference (KREX_REF_TILE selects another for experiments):
+// 0 = 128x128, TK 16, one block per SM (143 registers); 1 = 128x256, TK 16;
+// 2 = 128x128, TK 32; 3 = 128x256, TK 32; 4 = 128x128, TK 16 with at most 128
+// registers, so two blocks share an SM.  Measured on GB300 (TFLOP/s at 4096^3
+// / 8192^3, L2 flushed): 53.3/54.5, 49.9/56.6, 50.7/51.8, 43.0/49.0,
+// 54.8/57.2, all bit-identical (each output is one k-order FMA chain); the
+// packed fp32x2 FMA form of 4 ran slower (51.6/54.0).  Default: 4.
+int ref_tile() {
+    const char *e = getenv("KREX_REF_TILE");
+    if (e) {
+        int v = atoi(e);
+        if (v >= 0 && v <= 4) return v;
+    }
+    return 4;
+}
+
+template <bool F16>
+cudaError_t launch_ref(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
+                       int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c_vec, cudaStream_t s) {
+    switch (ref_tile()) {
+    case 0: return launch_cfg<F16, 2, 16, 1>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
+    case 1: return launch_cfg<F16, 4, 16, 1>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
+    case 2: return launch_cfg<F16, 2, 32, 1>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
+    case 3: return launch_cfg<F16, 4, 32, 1>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
+    default: return launch_cfg<F16, 2, 16, 2>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_gemm_ref(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
@@ -141,12 +221,8 @@ cudaError_t launch_gemm_ref(const uint16_t *a, int64_t lda, const uint16_t *b, i
     const bool a_vec = ((reinterpret_cast<uintptr_t>(a) & 15u) == 0) && (lda % 8 == 0);
     const bool b_vec = ((reinterpret_cast<uintptr_t>(b) & 15u) == 0) && (ldb % 8 == 0);
     const bool c_vec = ((reinterpret_cast<uintptr_t>(c) & 15u) == 0) && (ldc % 4 == 0);
-    dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
-    if (f16)
-        gemm_ref_simt<true><<<grid, 256, 0, s>>>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec);
-    else
-        gemm_ref_simt<false><<<grid, 256, 0, s>>>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec);
-    return cudaGetLastError();
+    return f16 ? launch_ref<true>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s)
+               : launch_ref<false>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
 }
 
 }  // namespace krex
