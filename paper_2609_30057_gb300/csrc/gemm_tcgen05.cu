@@ -474,7 +474,7 @@ constexpr int EPI_BOX_COLS = 64;                 // TMA-store box: 64 columns x 
 constexpr int EPI_BUF_BYTES = 32 * EPI_BOX_COLS * 2;
 constexpr int EPI_BYTES = 4 * 2 * EPI_BUF_BYTES; // 4 epilogue warps x 2 buffers
 constexpr int TMEM_COLS = 2 * BN;                // two 128-lane x 256-column accumulators
-constexpr int GROUP_M = 8;                       // pair-tile rows per raster group
+constexpr int GROUP_M = 8;                       // pair-tile rows per raster group (see raster_group)
 constexpr int EPI_WARPS = 4;
 // A stage holds KSUB K sub-blocks (KSUB x 64 of K): 6 stages of 32 KiB or 3
 // of 64 KiB.  Fewer, deeper stages issue 8 MMAs per barrier wait and commit
@@ -1108,13 +1108,18 @@ int pick_pair_tile_n() {
 }
 
 // Pair-tile rows per raster group of the 2-SM kernel; KREX_GEMM_GROUP overrides.
-int raster_group() {
+// Pair-tile rows per raster group.  Measured on GB300 (TFLOP/s, group 4 vs
+// 8, L2 flushed): 3072^3 1381 vs 1325, 4096^3 1561 vs 1525, 4608^3 1579 vs
+// 1557, but 2064^3 578 vs 592, 5120^3 1616 vs 1638, 7168^3 1739 vs 1794,
+// 8192^3 1799 vs 1851: 4 for GEMMs of 1.5 to 5 waves of pair tiles, else 8.
+// KREX_GEMM_GROUP overrides it for experiments.
+int raster_group(int64_t tiles, int max_clusters) {
     const char *e = getenv("KREX_GEMM_GROUP");
     if (e) {
         int v = atoi(e);
         if (v >= 1 && v <= 64) return v;
     }
-    return v2::GROUP_M;
+    return (2 * tiles >= 3 * (int64_t)max_clusters && tiles < 5 * (int64_t)max_clusters) ? 4 : v2::GROUP_M;
 }
 
 // Column-half split of a final partial wave (on unless KREX_GEMM_TAIL_SPLIT=0).
@@ -1271,7 +1276,8 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         uint32_t *ws_flag = split_k ? ws_count + WS_SLABS : nullptr;
         auto go = [&](auto kernel, size_t smem, int stages) {
             kernel<<<2 * clusters, THREADS, smem, s>>>(ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m,
-                                                       tiles_n, (int)full_items, (int)items, raster_group(), c_vec,
+                                                       tiles_n, (int)full_items, (int)items,
+                                                       raster_group(tiles, max_clusters), c_vec,
                                                        c_tma, stages, wait_timeout_ns(), split_k, ws_partial,
                                                        ws_count, ws_flag, launch_id);
         };
