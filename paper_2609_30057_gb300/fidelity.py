@@ -135,14 +135,55 @@ def candidates(device="cuda", quick: bool = False):
     return cands
 
 
+# Variants of the tcgen05 kernel on one 4096^3 GEMM, as an agent tuning it
+# would produce: K depth per ring stage, pair-tile width, the 1-SM form, the
+# raster group and the ring depth (knob settings of gemm_tcgen05.cu).
+TILE_VARIANTS = (
+    ("sm2_k128_n256", {}),
+    ("sm2_k64_n256", {"KREX_GEMM_KSUB": "1"}),
+    ("sm2_k128_n192", {"KREX_GEMM_BN": "192"}),
+    ("sm2_k128_n128", {"KREX_GEMM_BN": "128"}),
+    ("sm2_k128_g8", {"KREX_GEMM_GROUP": "8"}),
+    ("sm2_k64_st5", {"KREX_GEMM_KSUB": "1", "KREX_GEMM_STAGES": "5"}),
+    ("sm1_n256", {"KREX_GEMM_SM": "1"}),
+)
+
+
+def tile_variant_candidates(device="cuda"):
+    """(name, op, inputs, out, env) for the kernel variants above on one
+    4096^3 GEMM; timing sets each variant's knobs in this process only, so
+    it is used where no thread of this process launches GEMMs concurrently."""
+    import torch
+    n = 4096
+    a = torch.empty(n, n, dtype=torch.bfloat16, device=device)
+    b = torch.empty(n, n, dtype=torch.bfloat16, device=device)
+    krex_gen_inputs(7, 0, 0, 0.0, a)
+    krex_gen_inputs(7, 1, 0, 0.0, b)
+    c = torch.empty(n, n, dtype=torch.bfloat16, device=device)
+    return [(f"gemm4096_{name}", KREX_OP_GEMM_BF16, [a, b], c, env) for name, env in TILE_VARIANTS]
+
+
 def time_candidates(cands, flush, iters, stream, gate=None, tenant=0, per_iter=None):
     """Median of `iters` flushed, timed iterations of each candidate (the
     command's timed loop), optionally inside a gated region.  `per_iter`, if
-    a list, receives every candidate's iteration durations."""
+    a list, receives every candidate's iteration durations.  A candidate's
+    optional fifth field is a dict of kernel knobs set while it is timed."""
+    import os
     out = []
-    for name, op, ins, o in cands:
-        d, p50, _ = krex_bench_candidate(op, ins, o, warmup=3, iters=iters, flush_scratch=flush,
-                                         flush_bytes=flush.numel(), stream=stream, gate=gate, tenant=tenant)
+    for cand in cands:
+        name, op, ins, o = cand[:4]
+        env = cand[4] if len(cand) > 4 else {}
+        saved = {k: os.environ.get(k) for k in env}
+        os.environ.update(env)
+        try:
+            d, p50, _ = krex_bench_candidate(op, ins, o, warmup=3, iters=iters, flush_scratch=flush,
+                                             flush_bytes=flush.numel(), stream=stream, gate=gate, tenant=tenant)
+        finally:
+            for k, v in saved.items():
+                if v is None:
+                    os.environ.pop(k, None)
+                else:
+                    os.environ[k] = v
         out.append(p50)
         if per_iter is not None:
             per_iter.append(list(d))
@@ -335,7 +376,9 @@ def run_xproc(tenants: int = 2, iters: int = 20, quick: bool = False, shm_dir: s
             p.start()
         stream = torch.cuda.Stream()
         flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
-        cands = candidates(quick=quick)
+        # tenants run in other processes, so the tile variants' knobs can be
+        # set in this one while they are timed
+        cands = candidates(quick=quick) + ([] if quick else tile_variant_candidates())
         t0 = time.monotonic()
         while not all(ctl[_X_BASE + 3 * i] for i in range(tenants)):
             if time.monotonic() - t0 > 120 or any(p.exitcode not in (None, 0) for p in procs):
