@@ -450,7 +450,8 @@ krex_status krex_device_status(uint32_t *code);
  * 3 nanoseconds waited; then that CTA's progress: 4 producer work item |
  * K stage << 32; 5 MMA issuer work item | K stage << 32 (0xFFFFFFFF: waiting
  * for an accumulator); 6 first epilogue warp's work item | step << 32
- * (1 waiting for an accumulator, 2 draining it, 3 released); 7 M | N << 21 |
+ * (1 waiting for an accumulator, 2 draining it, 3 released); work items
+ * count within the CTA pair's own sequence; 7 M | N << 21 |
  * K << 42 (each mod 2^21).  Read it before krex_device_status, which clears
  * both.  Synchronises the device. */
 krex_status krex_device_status_detail(uint64_t *words);

@@ -680,7 +680,8 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                       const __grid_constant__ CUtensorMap tmC, uint16_t *__restrict__ C, int64_t ldc, int M,
                       int N, int K, int bn, int tiles_m, int tiles_n, int full_items, int num_items,
                       int group_m, int c_vec, int c_tma, int stages, uint64_t timeout_ns, int split_k,
-                      float *ws_partial, uint32_t *ws_count, uint32_t *ws_flag, uint32_t launch_id) {
+                      float *ws_partial, uint32_t *ws_count, uint32_t *ws_flag, uint32_t launch_id,
+                      uint32_t wait_tag) {
     // this kernel's tile constants shadow the 1-SM ones
     using CF = v2::Cfg<KSUB>;
     constexpr int BM = v2::BM, BN = v2::BN, BK = v2::BK, STAGES = CF::STAGES;
@@ -902,7 +903,7 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                     store_c = false;
                 } else {
                     uint32_t ok = 1u;
-                    if (lane == 0) ok = flag_wait_acquire(ws_flag + sidx, launch_id, abort_flag, timeout_ns, 0x52);
+                    if (lane == 0) ok = flag_wait_acquire(ws_flag + sidx, wait_tag, abort_flag, timeout_ns, 0x52);
                     ok = __shfl_sync(0xffffffffu, ok, 0);
                     if (ok) {
                         (void)flag_load_acquire(ws_flag + sidx);  // every lane acquires the partial
@@ -1123,6 +1124,15 @@ int raster_group(int64_t tiles, int max_clusters) {
 }
 
 // Column-half split of a final partial wave (on unless KREX_GEMM_TAIL_SPLIT=0).
+// KREX_DEBUG_STALL_HANDOVER=1 (read per launch; for the failure-detection
+// test only) makes the second K half of a split tile wait for a tag that no
+// launch publishes, so its bounded wait runs out: the kernel then sets the
+// status word (0x1052), drains and returns, and the context stays usable.
+bool debug_stall_handover() {
+    const char *e = getenv("KREX_DEBUG_STALL_HANDOVER");
+    return e && e[0] == '1';
+}
+
 bool tail_split_enabled() {
     const char *e = getenv("KREX_GEMM_TAIL_SPLIT");
     return !(e && e[0] == '0');
@@ -1270,6 +1280,9 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         static std::atomic<uint32_t> launch_counter{0};
         uint32_t launch_id = launch_counter.fetch_add(1) + 1;
         if (launch_id == 0) launch_id = launch_counter.fetch_add(1) + 1;  // 0 never tags a published partial
+        // the tag the second K half waits for: this launch's, or (the failure-
+        // detection test's switch) one that no launch publishes
+        const uint32_t wait_tag = debug_stall_handover() ? (launch_id ^ 0x80000000u) : launch_id;
         float *ws_partial = split_k ? static_cast<float *>(workspace) : nullptr;
         uint32_t *ws_count =
             split_k ? reinterpret_cast<uint32_t *>(static_cast<uint8_t *>(workspace) + WS_PARTIAL_BYTES) : nullptr;
@@ -1279,7 +1292,7 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
                                                        tiles_n, (int)full_items, (int)items,
                                                        raster_group(tiles, max_clusters), c_vec,
                                                        c_tma, stages, wait_timeout_ns(), split_k, ws_partial,
-                                                       ws_count, ws_flag, launch_id);
+                                                       ws_count, ws_flag, launch_id, wait_tag);
         };
         const int st2 = ring_stages(v2::Cfg<2>::STAGES), st1 = ring_stages(v2::Cfg<1>::STAGES);
         if (ksub == 2 && f16)
