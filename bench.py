@@ -248,7 +248,13 @@ def oracle_command_cost(w, budget_s: float = 10.0):
             f"{'fp64 GEMM' if w.is_gemm else 'fp64 softmax'} on {rows} of {w.M} output rows scaled to the full "
             f"output and counted {runs}x (reference + check run + {w.warmup} warm-up + {w.iters} timed), "
             f"fp32 check on {n_chk} rows scaled; sample wall {time.perf_counter() - t0:.1f} s")
-    return total, info
+    in_bytes = (w.M * w.K + w.K * w.N) * 2 if w.is_gemm else w.M * w.N * 4
+    comp = {"gen_GB_per_s": in_bytes / t_gen / 1e9, "check_GB_per_s": w.M * w.N * (6 if w.is_gemm else 8) / t_chk / 1e9}
+    if w.is_gemm:
+        comp["gemm_fp64_GFLOP_per_s"] = 2.0 * w.M * w.N * w.K / per_full / 1e9
+    else:
+        comp["softmax_fp64_rows_per_s"] = w.M / per_full
+    return total, info, comp
 
 
 def _p95(xs) -> float:
@@ -401,8 +407,9 @@ def main():
 
     cpu = None
     if not args.no_cpu_baseline:
-        secs, info = oracle_command_cost(w)
-        cpu = {"value": 1.0 / secs, "unit": "cmds/s", "cores": cpu_cores(), "kind": "oracle", "sample": info}
+        secs, info, comp = oracle_command_cost(w)
+        cpu = {"value": 1.0 / secs, "unit": "cmds/s", "cores": cpu_cores(), "kind": "oracle", "sample": info,
+               "components": comp}
 
     cs = clocks.summary()
     ph = [statistics.fmean(p[i] for p in phases) for i in range(5)]
@@ -484,8 +491,9 @@ def reference_arm(args, rank, world):
         oracle_command_cost(w, budget)
     secs = []
     info = ""
+    comp = {}
     for _ in range(args.steps):
-        s, info = oracle_command_cost(w, budget)
+        s, info, comp = oracle_command_cost(w, budget)
         secs.append(s)
     value = args.steps / sum(secs)
     line = {"metric": METRIC, "value": value, "unit": "cmds/s", "n_gpus": world, "steps": args.steps,
@@ -495,7 +503,7 @@ def reference_arm(args, rank, world):
                        "parallelism": "host"},
             "impl": "reference",
             "cpu_baseline": {"value": value, "unit": "cmds/s", "cores": cpu_cores(), "kind": "oracle",
-                             "sample": info},
+                             "sample": info, "components": comp},
             "e2e": {"value": value, "unit": "cmds/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
 
