@@ -1,0 +1,53 @@
+"""bench.py's JSON line: the reference arm on the CPU (the oracle on the host
+cores), and our arm on the GPU, carry every key the measurement contract
+names, with consistent values."""
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+from conftest import ROOT
+
+BASE_KEYS = {"metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling",
+             "vs_baseline", "dtype", "data", "config", "e2e", "cpu_baseline"}
+
+
+def _bench(*args, timeout=600):
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), *args], capture_output=True, text=True,
+                       timeout=timeout, cwd=ROOT)
+    assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-2000:]
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def test_reference_arm_line():
+    d = _bench("--impl", "reference", "--steps", "1", "--warmup", "0", "--workload", "gemm_bf16_256")
+    assert BASE_KEYS <= set(d)
+    assert d["impl"] == "reference" and d["value"] > 0 and d["unit"] == "cmds/s" and d["higher_is_better"]
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
+    assert cb["components"]["gemm_fp64_GFLOP_per_s"] > 0
+    assert d["config"]["workload"] == "gemm_bf16_256"
+
+
+@pytest.mark.gpu
+def test_our_arm_line():
+    d = _bench("--steps", "3", "--warmup", "3", "--no-kernels")
+    assert BASE_KEYS <= set(d) and {"roofline", "gpu_launches", "clocks", "timing_spread"} <= set(d)
+    assert d["n_gpus"] == 1 and d["steps"] == 3 and d["warmup"] == 3 and d["value"] > 0
+    assert abs(d["value"] - 3 / (d["ms_per_step"] * 3 / 1e3)) < 1e-6 * d["value"]
+    r = d["roofline"]
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s" and 0 < r["frac"] < 1.2
+    assert abs(r["frac"] - r["achieved"] / r["peak"]) < 1e-9
+    e = d["e2e"]
+    assert e["value"] > 0 and e["h2d_bytes_per_step"] == 2 * 4096 * 4096 * 2
+    assert e["d2h_bytes_per_step"] >= 4096 * 4096 * 2
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] > 0
+    # launches per command: 2 fills, reference, candidate, check, entry flush, (flush + GEMM) per warm-up and
+    # timed iteration of the region
+    per_cmd = 2 + 1 + 1 + 1 + 1 + 2 * (3 + 100)
+    assert d["gpu_launches"] == 3 * per_cmd
+    assert d["clocks"]["samples"] >= 1
