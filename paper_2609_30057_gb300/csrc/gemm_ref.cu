@@ -191,7 +191,8 @@ cudaError_t launch_cfg(const uint16_t *a, int64_t lda, const uint16_t *b, int64_
 // registers, so two blocks share an SM.  Measured on GB300 (TFLOP/s at 4096^3
 // / 8192^3, L2 flushed): 53.3/54.5, 49.9/56.6, 50.7/51.8, 43.0/49.0,
 // 54.8/57.2, all bit-identical (each output is one k-order FMA chain); the
-// packed fp32x2 FMA form of 4 ran slower (51.6/54.0).  Default: 4.
+// packed fp32x2 FMA form of 4 ran slower (51.6/54.0), and so did 4 with 32-deep
+// slices (49.8/52.2).  Default: 4.
 int ref_tile() {
     const char *e = getenv("KREX_REF_TILE");
     if (e) {
