@@ -1,26 +1,32 @@
-// K4: the timed GEMM candidate, C = A B with bf16 operands, fp32 accumulation
-// in tensor memory and bf16 output (paper Section 2.1 and Figure 1a: the GEMM
-// benchmarking command whose timed loop is 8.5% of the command).
+// K4: the timed GEMM candidate, C = A B with bf16 (or IEEE binary16)
+// operands, fp32 accumulation in tensor memory and a 16-bit output rounded to
+// nearest even (paper Section 2.1 and Figure 1a: the GEMM benchmarking
+// command whose timed loop is 8.5% of the command).
 //
-// Blackwell design (sm_103a), one persistent CTA per SM:
-//   warp 0      TMA producer: cp.async.bulk.tensor loads of A (K-major, 128B
-//               swizzle) and B (N-major, 128B swizzle) into a STAGES-deep ring
-//               of shared-memory stages, completion tracked by mbarrier
-//               transaction counts.
-//   warp 1      MMA issuer: one thread issues tcgen05.mma.cta_group::1.kind::f16
-//               (M=128, N=256, K=16) into a TMEM accumulator and releases each
-//               stage with tcgen05.commit.
-//   warp 2      allocates / frees the 512 TMEM columns (two 128x256 fp32
-//               accumulators, so the epilogue of tile i overlaps the MMAs of
-//               tile i+1).
-//   warps 4-7   epilogue: tcgen05.ld 32x32b (each warp owns 32 TMEM lanes = 32
-//               rows), fp32 -> bf16 RNE, 16-byte global stores.
-// Tiles are visited in groups of GROUP_M row blocks so concurrently running
-// CTAs share A and B panels in L2.
+// Default form, gemm_tcgen05_2sm: a cluster of two CTAs (a TPC) computes a
+// 256 x bn pair tile with tcgen05.mma.cta_group::2 (M = 256, K = 16); a
+// persistent grid holds one cluster per co-resident SM pair.  Per CTA:
+//   warp 0      TMA producer: A (K-major) and its half of B (N-major) tiles,
+//               128-byte swizzle, into a ring of 128-deep K stages; both CTAs'
+//               loads complete on the leader's full barrier, on which the peer
+//               producer also arrives.
+//   warp 1      (leader only) MMA issuer: one thread, 8 MMAs per stage, each
+//               stage released to both producers by a multicast commit.
+//   warp 2      allocates / frees 512 TMEM columns: two accumulators, so the
+//               epilogue of one tile overlaps the MMAs of the next.
+//   warps 4-7   epilogue: tcgen05.ld of 32 rows each, 16-bit RNE, TMA store
+//               from 128B-swizzled staging (direct stores when C's rows are
+//               not 16-byte aligned).
+// Pair tiles run in raster groups of rows so concurrently running pairs share
+// A and B panels in L2; a final partial wave is split in two (column halves,
+// or K halves whose fp32 partials meet in a caller-provided workspace).  A
+// 1-SM form (gemm_bf16_tcgen05, cta_group::1, 128 x 256 tiles, bf16) is kept
+// for comparison.
 //
-// Every mbarrier wait is bounded (globaltimer); a wait that runs out sets a
-// shared abort flag and the device status word, every role drains what it
-// has in flight (bounded), TMEM is freed and the kernel returns.
+// Every mbarrier and flag wait is bounded (globaltimer); a wait that runs out
+// sets a shared abort flag, the device status word and a record of where each
+// role was, every role drains what it has in flight (bounded), TMEM is freed
+// and the kernel returns.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
