@@ -54,10 +54,10 @@ std::atomic<uint32_t> g_flush_value{0x5EED0001u};
 
 int sm_count() {
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return 148;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDev) return 152;
     int v = g_sm[dev].load(std::memory_order_relaxed);
     if (v <= 0) {
-        if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) v = 148;
+        if (cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || v <= 0) v = 152;
         g_sm[dev].store(v, std::memory_order_relaxed);
     }
     return v;
