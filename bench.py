@@ -154,6 +154,9 @@ def kernel_table(ws, w, peaks, stream):
     import torch
     import paper_2609_30057_gb300 as krex
     from paper_2609_30057_gb300.command import WORKLOADS, Workspace
+    if not w.is_gemm:               # the GEMM rows run at the GEMM workload's size
+        w = WORKLOADS[DEFAULT_WORKLOAD]
+        ws = Workspace(w)
     flush_t = ws.flush
     flush = lambda: krex.krex_flush_l2(flush_t, stream=stream)  # noqa: E731
     out = {}

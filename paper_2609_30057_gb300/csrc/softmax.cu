@@ -77,16 +77,17 @@ softmax_rows_reg(const float *__restrict__ x, int64_t ldx, float *__restrict__ y
         float m = -INFINITY;
 #pragma unroll
         for (int k = 0; k < VPT; ++k) m = fmaxf(m, fmaxf(fmaxf(v[k].x, v[k].y), fmaxf(v[k].z, v[k].w)));
+        // a thread whose elements are all masked (-inf) shifts by 0, so they
+        // become exp(-inf) = 0 and its sum 0, with no -inf - -inf
+        const float shift = (m == -INFINITY) ? 0.0f : m;
         float s = 0.0f;
-        if (m != -INFINITY) {
 #pragma unroll
-            for (int k = 0; k < VPT; ++k) {
-                v[k].x = expf(v[k].x - m);
-                v[k].y = expf(v[k].y - m);
-                v[k].z = expf(v[k].z - m);
-                v[k].w = expf(v[k].w - m);
-                s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
-            }
+        for (int k = 0; k < VPT; ++k) {
+            v[k].x = expf(v[k].x - shift);
+            v[k].y = expf(v[k].y - shift);
+            v[k].z = expf(v[k].z - shift);
+            v[k].w = expf(v[k].w - shift);
+            s += (v[k].x + v[k].y) + (v[k].z + v[k].w);
         }
         MS tot = block_merge<THREADS>(MS{m, s});
         float scale = (m == -INFINITY) ? 0.0f : expf(m - tot.m) / tot.s;
@@ -113,7 +114,7 @@ softmax_rows_online(const float *__restrict__ x, int64_t ldx, float *__restrict_
             if (xv > acc.m) {
                 acc.s = (acc.m == -INFINITY ? 0.0f : acc.s * expf(acc.m - xv)) + 1.0f;
                 acc.m = xv;
-            } else {
+            } else if (xv != -INFINITY) {  // a masked -inf adds 0 (and -inf - -inf would be NaN)
                 acc.s += expf(xv - acc.m);
             }
         }

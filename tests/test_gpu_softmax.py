@@ -79,3 +79,52 @@ def test_softmax_full_workload_sampled_rows():
     assert np.max(np.abs(r[st].cpu().numpy() - want)) <= ATOL
     # property at any size: every row sums to 1 within fp32 rounding
     assert torch.max(torch.abs(y.double().sum(dim=1) - 1.0)).item() < 1e-4
+
+
+# one width either side of each register-tile limit (16-byte aligned rows: the
+# vector kernels) and past the largest tile (the online kernel)
+@pytest.mark.parametrize("cols", [1020, 1028, 2044, 2052, 4092, 4100, 8188, 8196, 16380, 16388])
+def test_softmax_either_side_of_each_tile_limit(cols):
+    x = gen.normal_f32(6, cols, 3, cols, 2.0)
+    y, r = _softmax_both(x)
+    want = ref.softmax_rows_f64(x.astype(np.float64))
+    assert np.max(np.abs(y - want)) <= ATOL and np.max(np.abs(r - want)) <= ATOL
+
+
+@pytest.mark.parametrize("pad,ld", [(65, None), (64, 1026), (67, 1027)])
+def test_softmax_unaligned_layouts(pad, ld):
+    # a row base off a 16-byte boundary or an odd leading dimension rules out
+    # the vector loads; the result must not depend on which kernel ran
+    rows, cols = 5, 1024
+    x_np = gen.normal_f32(7, pad, rows, cols, 2.0)
+    x = Guarded(rows, cols, torch.float32, ld=ld, pad_elems=pad)
+    x.view.copy_(torch.from_numpy(x_np))
+    y = Guarded(rows, cols, torch.float32, ld=ld, pad_elems=pad)
+    r = Guarded(rows, cols, torch.float32, ld=ld, pad_elems=pad)
+    krex.krex_run_candidate(krex.KREX_OP_SOFTMAX_F32, [x.view], y.view)
+    krex.krex_run_reference(krex.KREX_OP_SOFTMAX_F32, [x.view], r.view)
+    torch.cuda.synchronize()
+    assert y.canaries_intact() and r.canaries_intact()
+    want = ref.softmax_rows_f64(x_np.astype(np.float64))
+    assert np.max(np.abs(y.view.cpu().numpy() - want)) <= ATOL
+    assert np.max(np.abs(r.view.cpu().numpy() - want)) <= ATOL
+
+
+@pytest.mark.parametrize("cols", [4096, 4097, 20000])
+def test_softmax_masked_entries_and_float32_extremes(cols):
+    # -inf entries (masked logits) get exactly 0, including threads whose
+    # every element is masked; +-FLT_MAX entries split the mass evenly
+    x = gen.normal_f32(8, cols, 4, cols, 2.0)
+    x[0, :-100] = -np.inf
+    x[1, 1:] = -np.inf
+    x[2, ::3] = -np.inf
+    big = np.finfo(np.float32).max
+    x[3, ::7] = big
+    x[3, 3::7] = -big
+    y, r = _softmax_both(x)
+    want = ref.softmax_rows_f64(x.astype(np.float64))
+    masked = np.isneginf(x)
+    for got in (y, r):
+        assert np.max(np.abs(got - want)) <= ATOL
+        assert np.all(got[masked] == 0.0)
+    assert y[1, 0] == 1.0

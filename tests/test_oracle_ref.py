@@ -142,6 +142,25 @@ def test_softmax_brute_force_tiny_rows():
         assert np.allclose(ref.softmax_rows_f64(x)[0], want, rtol=1e-15, atol=0)
 
 
+def test_softmax_masked_entries_are_zero_and_the_rest_renormalise():
+    # an entry of -inf (a masked logit) gets exactly 0, and the others are the
+    # softmax of the unmasked entries alone; extremes of the float32 range too
+    rng = np.random.default_rng(2)
+    x = rng.normal(0, 2, size=(3, 50))
+    keep = rng.random((3, 50)) < 0.3
+    keep[:, 0] = True
+    x[~keep] = -np.inf
+    y = ref.softmax_rows_f64(x)
+    assert np.all(y[~keep] == 0.0)
+    for r in range(3):
+        sub = x[r, keep[r]]
+        ex = [math.exp(v - max(sub)) for v in sub]
+        assert np.allclose(y[r, keep[r]], [v / math.fsum(ex) for v in ex], rtol=1e-15, atol=0)
+    big = np.float64(np.finfo(np.float32).max)
+    y = ref.softmax_rows_f64(np.array([[big, -big, big, 0.0]]))
+    assert np.array_equal(y[0], [0.5, 0.0, 0.5, 0.0])
+
+
 # ----------------------------------------------------------------- check ----
 
 def _f32(v):
