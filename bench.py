@@ -41,6 +41,12 @@ if ROOT not in sys.path:
 METRIC = "GEMM TFLOP/s & fill/flush/softmax/check GB/s vs roofline; bench cmds/s, 1 GB300"
 DEFAULT_WORKLOAD = "gemm_bf16_4096"
 SOFTMAX_WORKLOAD = "softmax_f32_65536x8192"
+# 32-bit integer-ALU operations the uniform generator's definition takes per
+# 16-bit element: per SplitMix64 draw (two elements) a 64-bit add (2) and three
+# 64-bit xor-shifts (2 funnel shifts + 2 xors each: 12); per element the 24-bit
+# field to [-1, 1) (a shift, two masks, an integer subtract: 4).  The two 64-bit
+# multiplies per draw run on the multiply-add pipe and are not counted.
+FILL_ALU_OPS_PER_ELEMENT = (2 + 12) / 2 + 4
 
 
 def _peaks():
@@ -161,7 +167,11 @@ def kernel_table(ws, w, peaks, stream):
     flush = lambda: krex.krex_flush_l2(flush_t, stream=stream)  # noqa: E731
     out = {}
 
-    def rec(name, fn, nbytes=None, flops=None, n=20, do_flush=True):
+    # integer-ALU roofline of the uniform fill: 64 ALU lanes per clock per SM
+    # at the 2070 MHz maximum SM clock (the clock the runs see under load)
+    alu_peak = torch.cuda.get_device_properties(stream.device).multi_processor_count * 64 * 2.070e9
+
+    def rec(name, fn, nbytes=None, flops=None, alu_ops=None, n=20, do_flush=True):
         for _ in range(3):
             fn()
         ms = _time_launches(fn, n, stream, flush if do_flush else None)
@@ -172,10 +182,18 @@ def kernel_table(ws, w, peaks, stream):
         if flops is not None:
             tf = flops / ms / 1e9
             e.update({"TFLOP/s": tf, "frac_bf16": tf / peaks["bf16_tflops"], "flops": flops})
+        if alu_ops is not None:
+            e.update({"bound": "alu", "alu_ops": alu_ops, "Tops/s": alu_ops / ms / 1e9,
+                      "frac_alu": alu_ops / ms * 1e3 / alu_peak})
         out[name] = e
 
     A, B = ws.inputs
-    rec("fill_uniform_bf16", lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, A, stream), nbytes=A.numel() * 2)
+    rec("fill_uniform_bf16", lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, A, stream), nbytes=A.numel() * 2,
+        alu_ops=A.numel() * FILL_ALU_OPS_PER_ELEMENT)
+    big = torch.empty(16384, 16384, dtype=torch.bfloat16, device=A.device)   # steady state, 512 MiB
+    rec("fill_uniform_bf16_16384", lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, big, stream),
+        nbytes=big.numel() * 2, alu_ops=big.numel() * FILL_ALU_OPS_PER_ELEMENT, n=10)
+    del big
     rec("flush_l2", flush, nbytes=flush_t.numel(), do_flush=False)
     rec("gemm_ref_simt", lambda: krex.krex_run_reference(w.op, ws.inputs, ws.ref, stream), flops=w.flops, n=3)
     rec("gemm_tcgen05", lambda: krex.krex_run_candidate_ws(w.op, ws.inputs, ws.out, ws.gemm_ws, stream),
@@ -197,7 +215,8 @@ def kernel_table(ws, w, peaks, stream):
     a16 = torch.empty(fw.M, fw.K, dtype=torch.float16, device=A.device)
     b16 = torch.empty(fw.K, fw.N, dtype=torch.float16, device=A.device)
     c16 = torch.empty(fw.M, fw.N, dtype=torch.float16, device=A.device)
-    rec("fill_uniform_f16", lambda: krex.krex_gen_inputs(fw.seed, 0, 0, 0.0, a16, stream), nbytes=a16.numel() * 2)
+    rec("fill_uniform_f16", lambda: krex.krex_gen_inputs(fw.seed, 0, 0, 0.0, a16, stream), nbytes=a16.numel() * 2,
+        alu_ops=a16.numel() * FILL_ALU_OPS_PER_ELEMENT)
     krex.krex_gen_inputs(fw.seed, 1, 0, 0.0, b16, stream)
     rec("gemm_tcgen05_f16", lambda: krex.krex_run_candidate_ws(fw.op, [a16, b16], c16, ws.gemm_ws, stream),
         flops=fw.flops)
