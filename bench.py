@@ -291,6 +291,20 @@ def cpu_cores() -> int:
     return len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else (os.cpu_count() or 1)
 
 
+def cpu_model() -> str:
+    """The host CPU's model name as lscpu reports it (the machine type if lscpu is missing)."""
+    import platform
+    import subprocess
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return platform.machine()
+
+
 # ------------------------------------------------------------- main ---------
 
 def main():
@@ -431,7 +445,7 @@ def main():
     if not args.no_cpu_baseline:
         secs, info, comp = oracle_command_cost(w)
         cpu = {"value": 1.0 / secs, "unit": "cmds/s", "cores": cpu_cores(), "kind": "oracle", "sample": info,
-               "components": comp}
+               "components": comp, "cpu_model": cpu_model()}
 
     cs = clocks.summary()
     ph = [statistics.fmean(p[i] for p in phases) for i in range(5)]
@@ -525,7 +539,7 @@ def reference_arm(args, rank, world):
                        "parallelism": "host"},
             "impl": "reference",
             "cpu_baseline": {"value": value, "unit": "cmds/s", "cores": cpu_cores(), "kind": "oracle",
-                             "sample": info, "components": comp},
+                             "sample": info, "components": comp, "cpu_model": cpu_model()},
             "e2e": {"value": value, "unit": "cmds/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
 

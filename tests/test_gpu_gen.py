@@ -76,15 +76,14 @@ def test_uniform_full_size_bitexact(seed, n):
         del t
 
 
-def test_uniform_16384_sampled_bitexact():
+def test_uniform_16384_full_bitexact():
+    # both operands of the 16384^3 GEMM workload, every element
     n = 16384
     t = torch.empty(n, n, dtype=torch.bfloat16, device="cuda")
-    krex.krex_gen_inputs(5, 1, krex.KREX_DIST_UNIFORM_PM1, 0.0, t)
-    torch.cuda.synchronize()
-    host = bits16(t).ravel()
-    i, j = ref.sample_indices(5, 7, 1 << 20, n * n, 1)
-    idx = np.concatenate([i, np.arange(4096), np.arange(n * n - 4096, n * n)])
-    assert np.array_equal(host[idx], gen.uniform_bf16_at(5, 1, idx))
+    for tid in (0, 1):
+        krex.krex_gen_inputs(5, tid, krex.KREX_DIST_UNIFORM_PM1, 0.0, t)
+        torch.cuda.synchronize()
+        assert np.array_equal(bits16(t), gen.uniform_bf16(5, tid, n, n))
 
 
 def test_normal_softmax_input_sampled_bitexact():
