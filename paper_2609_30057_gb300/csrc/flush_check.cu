@@ -46,6 +46,11 @@ flush_kernel(uint4 *__restrict__ p, size_t n16, uint32_t value, uint8_t *tail, s
 
 constexpr int kCheckThreads = 256;
 constexpr int kCheckMaxBlocks = 2048;
+// Resident blocks per SM the check kernels are compiled for (their register
+// budgets follow); the grid never exceeds what is resident at once, so no
+// block waits for a second wave with too few loads in flight to keep HBM busy.
+constexpr int kVecBlocksPerSM = 8;
+constexpr int kGenericBlocksPerSM = 4;
 constexpr uint32_t kCanonicalNaN = 0x7FC00000u;
 
 struct Partial {
@@ -161,7 +166,7 @@ __device__ __forceinline__ void block_reduce_publish(Acc acc, CheckScratch *sc) 
 // Contiguous fast path: 16-bit out (bf16 or binary16) vs fp32 ref, 8
 // elements per step.
 template <typename T>
-__global__ void __launch_bounds__(kCheckThreads)
+__global__ void __launch_bounds__(kCheckThreads, kVecBlocksPerSM)
 check_16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref, int64_t n8,
                  const T *out_s, const float *ref_s, int64_t n, float atol,
                  float rtol, CheckScratch *sc) {
@@ -189,7 +194,7 @@ check_16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref, 
 }
 
 // Contiguous fast path: fp32 out vs fp32 ref, 4 elements per step, 2 steps unrolled.
-__global__ void __launch_bounds__(kCheckThreads)
+__global__ void __launch_bounds__(kCheckThreads, kVecBlocksPerSM)
 check_f32_f32_vec(const float4 *__restrict__ out, const float4 *__restrict__ ref, int64_t n4,
                   const float *out_s, const float *ref_s, int64_t n, float atol, float rtol,
                   CheckScratch *sc) {
@@ -223,7 +228,7 @@ check_f32_f32_vec(const float4 *__restrict__ out, const float4 *__restrict__ ref
 
 // Any layout / dtype pair: one element per step.
 template <typename TO, typename TR>
-__global__ void __launch_bounds__(kCheckThreads)
+__global__ void __launch_bounds__(kCheckThreads, kGenericBlocksPerSM)
 check_generic(const TO *out, int64_t ldo, const TR *ref, int64_t ldr, int64_t rows,
               int64_t cols, float atol, float rtol, CheckScratch *sc) {
     Acc acc;
@@ -267,9 +272,9 @@ void launch_check_generic(const void *out, int out_dtype, int64_t ldo, const voi
         launch_generic_out<__half>(out, ldo, ref, ref_dtype, ldr, rows, cols, atol, rtol, sc, blocks, s);
 }
 
-int check_blocks(int64_t items) {
+int check_blocks(int64_t items, int blocks_per_sm) {
     int64_t b = (items + kCheckThreads - 1) / kCheckThreads;
-    int64_t cap = (int64_t)sm_count() * 8;
+    int64_t cap = (int64_t)sm_count() * blocks_per_sm;
     if (cap > kCheckMaxBlocks) cap = kCheckMaxBlocks;
     if (b > cap) b = cap;
     if (b < 1) b = 1;
@@ -304,23 +309,23 @@ cudaError_t launch_check(const void *out, int out_dtype, int64_t ldo, const void
     const bool a16 = ((reinterpret_cast<uintptr_t>(out) | reinterpret_cast<uintptr_t>(ref)) & 15u) == 0;
     if (contiguous && a16 && out_dtype == KREX_BF16 && ref_dtype == KREX_F32) {
         int64_t n8 = n / 8;
-        check_16_f32_vec<__nv_bfloat16><<<check_blocks(n8), kCheckThreads, 0, s>>>(
+        check_16_f32_vec<__nv_bfloat16><<<check_blocks(n8, kVecBlocksPerSM), kCheckThreads, 0, s>>>(
             static_cast<const uint4 *>(out), static_cast<const float4 *>(ref), n8,
             static_cast<const __nv_bfloat16 *>(out), static_cast<const float *>(ref), n, atol,
             rtol, sc);
     } else if (contiguous && a16 && out_dtype == KREX_F16 && ref_dtype == KREX_F32) {
         int64_t n8 = n / 8;
-        check_16_f32_vec<__half><<<check_blocks(n8), kCheckThreads, 0, s>>>(
+        check_16_f32_vec<__half><<<check_blocks(n8, kVecBlocksPerSM), kCheckThreads, 0, s>>>(
             static_cast<const uint4 *>(out), static_cast<const float4 *>(ref), n8,
             static_cast<const __half *>(out), static_cast<const float *>(ref), n, atol, rtol, sc);
     } else if (contiguous && a16 && out_dtype == KREX_F32 && ref_dtype == KREX_F32) {
         int64_t n4 = n / 4;
-        check_f32_f32_vec<<<check_blocks(n4 / 2), kCheckThreads, 0, s>>>(
+        check_f32_f32_vec<<<check_blocks(n4 / 2, kVecBlocksPerSM), kCheckThreads, 0, s>>>(
             static_cast<const float4 *>(out), static_cast<const float4 *>(ref), n4,
             static_cast<const float *>(out), static_cast<const float *>(ref), n, atol, rtol, sc);
     } else {
         launch_check_generic(out, out_dtype, ldo, ref, ref_dtype, ldr, rows, cols, atol, rtol, sc,
-                             check_blocks(n), s);
+                             check_blocks(n, kGenericBlocksPerSM), s);
     }
     return cudaGetLastError();
 }
