@@ -484,7 +484,9 @@ def kernel_only(args):
     krex.build()
     torch.cuda.set_device(0)
     stream = torch.cuda.current_stream()
-    name = SOFTMAX_WORKLOAD if args.kernel_only in ("softmax", "fill_normal") else args.workload
+    name = args.workload
+    if args.kernel_only in ("softmax", "fill_normal") and WORKLOADS[name].is_gemm:
+        name = SOFTMAX_WORKLOAD
     w = WORKLOADS[name]
     ws = Workspace(w)
     k = args.kernel_only

@@ -2,8 +2,9 @@
 
 A workload is one benchmarking command of the paper's Section 2.1 (generate
 seeded inputs, run the reference, run the candidate once, check it, then time
-it in a flushed warm-up + timed loop).  The five workloads below are named by
-what they are; sizes, seeds and iteration counts are part of the workload.
+it in a flushed warm-up + timed loop).  The workloads below are named by
+what they are; sizes, seeds and iteration counts are part of the workload
+(the last one is a smaller softmax for full ncu captures).
 
 PyTorch only allocates the buffers; ``run`` is a single ``krex_command_run``
 call into the library.
@@ -81,6 +82,10 @@ WORKLOADS = {
                               flush_bytes=256 * MiB),
     "gemm_bf16_16384": Workload("gemm_bf16_16384", KREX_OP_GEMM_BF16, 16384, 16384, 16384, seed=5, iters=20,
                                 flush_bytes=256 * MiB, oracle_samples=4096, repeat=32),
+    # a quarter of the softmax workload's rows (512 MiB in, 512 MiB out, still
+    # four times L2): the size at which its kernels are profiled in full
+    "softmax_f32_16384x8192": Workload("softmax_f32_16384x8192", KREX_OP_SOFTMAX_F32, 16384, 8192, 0, seed=3,
+                                       iters=100, flush_bytes=256 * MiB, oracle_samples=4096),
 }
 
 
