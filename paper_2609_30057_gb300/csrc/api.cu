@@ -589,6 +589,14 @@ krex_status krex_bench_candidate(int32_t op, const krex_buf *in, int32_t n_in, k
     return krex_region_end(r, durations_ms, iters, nullptr, p50_ms, p95_ms);
 }
 
+// Host <-> device copy of `rows` rows of `width` bytes: one linear copy when
+// the rows are packed on both sides, else a 2-D copy.
+static cudaError_t copy_rows(void *dst, size_t dpitch, const void *src, size_t spitch, size_t width, size_t rows,
+                             cudaMemcpyKind kind, cudaStream_t s) {
+    if (dpitch == width && spitch == width) return cudaMemcpyAsync(dst, src, width * rows, kind, s);
+    return cudaMemcpy2DAsync(dst, dpitch, src, spitch, width, rows, kind, s);
+}
+
 krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *bufs, const void *const *host_in,
                              void *host_out, float *durations_ms, krex_command_result *result,
                              krex_stream_t stream) {
@@ -622,8 +630,8 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
         const krex_buf &b = bufs->in[i];
         if (host_in && host_in[i]) {
             const size_t es = elem_size(b.dtype);
-            KREX_CUDA_TRY(cudaMemcpy2DAsync(b.ptr, (size_t)b.ld * es, host_in[i], (size_t)b.cols * es,
-                                            (size_t)b.cols * es, (size_t)b.rows, cudaMemcpyHostToDevice, s));
+            KREX_CUDA_TRY(copy_rows(b.ptr, (size_t)b.ld * es, host_in[i], (size_t)b.cols * es, (size_t)b.cols * es,
+                                    (size_t)b.rows, cudaMemcpyHostToDevice, s));
         } else {
             st = is_gemm(op)
                      ? krex_gen_inputs(cmd->seed, (uint32_t)i, KREX_DIST_UNIFORM_PM1, 0.0f, b, stream)
@@ -672,8 +680,8 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
     if (host_out) {
         const krex_buf &b = bufs->out;
         const size_t es = elem_size(b.dtype);
-        KREX_CUDA_TRY(cudaMemcpy2DAsync(host_out, (size_t)b.cols * es, b.ptr, (size_t)b.ld * es, (size_t)b.cols * es,
-                                        (size_t)b.rows, cudaMemcpyDeviceToHost, s));
+        KREX_CUDA_TRY(copy_rows(host_out, (size_t)b.cols * es, b.ptr, (size_t)b.ld * es, (size_t)b.cols * es,
+                                (size_t)b.rows, cudaMemcpyDeviceToHost, s));
         KREX_CUDA_TRY(cudaStreamSynchronize(s));
     }
     result->launches = (int32_t)(g_launches.load() - launches0);
