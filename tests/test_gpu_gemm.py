@@ -154,6 +154,45 @@ def test_k_zero_gives_zero_and_empty_is_noop(variant):
                             torch.empty(0, 8, dtype=torch.bfloat16, device="cuda"))
 
 
+@pytest.mark.parametrize("lda_pad,ldb_pad", [(8, 0), (0, 16), (24, 40)])
+def test_input_row_strides(lda_pad, ldb_pad, variant):
+    # A and B as views into wider rows whose padding holds NaN: a kernel that
+    # read past a row's K (A) or N (B) elements would put NaN into C.  The
+    # reference GEMM gets the same strided operands.
+    M, N, K = 300, 1000, 520
+    seed = 4100 + lda_pad + ldb_pad
+    nan16 = 0x7FC0
+    abase = torch.full((M, K + lda_pad), nan16, dtype=torch.int16, device="cuda").view(torch.bfloat16)
+    bbase = torch.full((K, N + ldb_pad), nan16, dtype=torch.int16, device="cuda").view(torch.bfloat16)
+    a, b = abase[:, :K], bbase[:, :N]
+    krex.krex_gen_inputs(seed, 0, krex.KREX_DIST_UNIFORM_PM1, 0.0, a)
+    krex.krex_gen_inputs(seed, 1, krex.KREX_DIST_UNIFORM_PM1, 0.0, b)
+    c = Guarded(M, N, torch.bfloat16)
+    r = Guarded(M, N, torch.float32)
+    krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [a, b], c.view)
+    krex.krex_run_reference(krex.KREX_OP_GEMM_BF16, [a, b], r.view)
+    torch.cuda.synchronize()
+    assert krex.krex_device_status() == 0
+    assert c.canaries_intact() and r.canaries_intact()
+    want = ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N))
+    ok, worst = _within_tol(bits16(c.view), want, K)
+    assert ok, worst
+    ok, worst = _within_tol(bits16(r.view.to(torch.bfloat16)), want, K)
+    assert ok, worst
+
+
+def test_unaligned_input_strides_are_rejected():
+    # TMA rows must start on 16 bytes: lda or ldb not a multiple of 8 elements
+    a = torch.zeros(64, 72, dtype=torch.bfloat16, device="cuda")[:, :64]
+    b = torch.zeros(64, 68, dtype=torch.bfloat16, device="cuda")[:, :64]
+    c = torch.empty(64, 64, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(krex.KrexError, match="UNSUPPORTED"):
+        krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [a[:, :60], b[:60]], c)   # K = 60
+    a2 = torch.zeros(64 * 68, dtype=torch.bfloat16, device="cuda").view(64, 68)[:, :64]   # lda = 68
+    with pytest.raises(krex.KrexError, match="UNSUPPORTED"):
+        krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [a2, b], c)                # ldb = 68 too
+
+
 def test_unsupported_shapes_are_rejected():
     a = torch.zeros(16, 12, dtype=torch.bfloat16, device="cuda")
     b = torch.zeros(12, 16, dtype=torch.bfloat16, device="cuda")
