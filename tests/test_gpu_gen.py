@@ -123,3 +123,14 @@ def test_uniform_f16_full_size_sampled():
     torch.cuda.synchronize()
     idx = ref.sample_indices(2, 4, 65536, 4096 * 4096)[0]
     assert np.array_equal(bits16(t).ravel()[idx], gen.uniform_f16_at(2, 0, idx))
+
+
+@pytest.mark.parametrize("rows,cols", [(0, 16), (4, 0), (0, 0)])
+@pytest.mark.parametrize("dtype,dist", [(torch.bfloat16, krex.KREX_DIST_UNIFORM_PM1),
+                                        (torch.float16, krex.KREX_DIST_UNIFORM_PM1),
+                                        (torch.float32, krex.KREX_DIST_NORMAL)])
+def test_empty_buffers_are_noops(rows, cols, dtype, dist):
+    g = Guarded(rows, cols, dtype, ld=max(cols, 8))
+    krex.krex_gen_inputs(1, 0, dist, 2.0, g.view)
+    torch.cuda.synchronize()
+    assert g.canaries_intact()

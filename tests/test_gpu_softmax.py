@@ -128,3 +128,13 @@ def test_softmax_masked_entries_and_float32_extremes(cols):
         assert np.max(np.abs(got - want)) <= ATOL
         assert np.all(got[masked] == 0.0)
     assert y[1, 0] == 1.0
+
+
+@pytest.mark.parametrize("rows,cols", [(0, 16), (4, 0), (0, 0)])
+def test_softmax_empty_is_noop(rows, cols):
+    x = Guarded(rows, cols, torch.float32, ld=max(cols, 8))
+    y = Guarded(rows, cols, torch.float32, ld=max(cols, 8))
+    krex.krex_run_candidate(krex.KREX_OP_SOFTMAX_F32, [x.view], y.view)
+    krex.krex_run_reference(krex.KREX_OP_SOFTMAX_F32, [x.view], y.view)
+    torch.cuda.synchronize()
+    assert x.canaries_intact() and y.canaries_intact()
