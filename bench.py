@@ -442,7 +442,7 @@ def main():
                     "algorithmic_bytes_per_launch": w.candidate_bytes}
 
     cpu = None
-    if not args.no_cpu_baseline:
+    if not args.no_cpu_baseline and world == 1:   # the host baseline is a single-GPU figure
         secs, info, comp = oracle_command_cost(w)
         cpu = {"value": 1.0 / secs, "unit": "cmds/s", "cores": cpu_cores(), "kind": "oracle", "sample": info,
                "components": comp, "cpu_model": cpu_model()}
