@@ -1139,6 +1139,19 @@ bool debug_stall_handover() {
     return e && e[0] == '1';
 }
 
+// K halves for a single partial wave (when a workspace is given): "auto"
+// (K >= kSplitKMinK), or KREX_GEMM_SPLIT_K=1 (whenever the shape allows: the
+// tests use it to exercise the hand-over on small shapes) / =0 (never).
+// Measured on GB300 (L2 flushed): the hand-over of the fp32 partials costs
+// about 4-6 us, so below K = 4096 column halves win (256^3: 10.2 against
+// 16.4 us; 1024^3: 14.3 against 18.5 us), while 1024 x 2048 x 8192 gains 8 %.
+constexpr int64_t kSplitKMinK = 4096;
+int split_k_mode() {
+    const char *e = getenv("KREX_GEMM_SPLIT_K");
+    if (e && (e[0] == '0' || e[0] == '1')) return e[0] - '0';
+    return -1;
+}
+
 bool tail_split_enabled() {
     const char *e = getenv("KREX_GEMM_TAIL_SPLIT");
     return !(e && e[0] == '0');
@@ -1272,8 +1285,9 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         const int64_t items = split ? tiles + rem : tiles;
         const int clusters = (int)(items < max_clusters ? items : max_clusters);
         // K halves (full-width MMAs) when a zero-initialised workspace is given,
-        // K has at least two ring stages and the split tiles are the whole
-        // GEMM (one partial wave); else column halves.  Measured on GB300: K
+        // K has at least two ring stages and is long enough (split_k_mode), and
+        // the split tiles are the whole GEMM (one partial wave); else column
+        // halves.  Measured on GB300: K
         // halves load a third less than column halves (1024 x 2048 x 8192:
         // 49 -> 44 us), but the hand-over of the fp32 partials (128 KiB per CTA
         // written, then read) sits on the last wave's critical path: at 4096^3
@@ -1281,8 +1295,10 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         // exchanging partials, so the multi-wave case gains nothing.
         const int ksub = stage_ksub();
         const int64_t num_kb = (((K + 63) / 64) + ksub - 1) / ksub;
+        const int sk_mode = split_k_mode();
+        const bool k_worth_it = sk_mode == 1 || (sk_mode < 0 && K >= kSplitKMinK);
         const int split_k = split && full_items == 0 && workspace && workspace_bytes >= WS_BYTES &&
-                            rem <= WS_SLOTS && num_kb >= 2 && clusters >= 2;
+                            rem <= WS_SLOTS && num_kb >= 2 && clusters >= 2 && k_worth_it;
         static std::atomic<uint32_t> launch_counter{0};
         uint32_t launch_id = launch_counter.fetch_add(1) + 1;
         if (launch_id == 0) launch_id = launch_counter.fetch_add(1) + 1;  // 0 never tags a published partial

@@ -25,6 +25,7 @@ import paper_2609_30057_gb300 as krex
 from oracle import gen, ref
 krex.build()
 M, N, K = 1024, 2048, 512            # one partial wave: K halves through the workspace
+os.environ["KREX_GEMM_SPLIT_K"] = "1"  # (at this K only when asked for)
 a = torch.empty(M, K, dtype=torch.bfloat16, device="cuda")
 b = torch.empty(K, N, dtype=torch.bfloat16, device="cuda")
 krex.krex_gen_inputs(31, 0, 0, 0.0, a)

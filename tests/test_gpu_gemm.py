@@ -249,6 +249,7 @@ def test_2sm_split_k_tail(M, N, K, ksub, monkeypatch):
     # reset themselves, the flags are tagged per launch)
     monkeypatch.setenv("KREX_GEMM_SM", "2")
     monkeypatch.setenv("KREX_GEMM_KSUB", ksub)
+    monkeypatch.setenv("KREX_GEMM_SPLIT_K", "1")   # the hand-over at every K, not only where it pays
     seed = 6000 + M + N + K
     a, b = _gen(seed, M, N, K)
     ws = krex.gemm_workspace()
@@ -266,9 +267,10 @@ def test_2sm_split_k_tail(M, N, K, ksub, monkeypatch):
         assert torch.count_nonzero(counters).item() == 0  # every arrival counter back at 0
 
 
-def test_split_k_matches_column_split_closely():
+def test_split_k_matches_column_split_closely(monkeypatch):
     # K halves and column halves sum the same products in different orders:
     # both within tolerance, and equal in most elements
+    monkeypatch.setenv("KREX_GEMM_SPLIT_K", "1")
     M, N, K = 1536, 1536, 3072
     a, b = _gen(2, M, N, K)
     c0 = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
@@ -367,7 +369,8 @@ def test_f16_small_integers_are_exact():
 
 @pytest.mark.parametrize("M,N,K", [(128, 256, 64), (100, 72, 40), (300, 1000, 520), (1024, 2048, 512),
                                    (640, 384, 4104), (2064, 1000, 1032), (4096, 4096, 4096)])
-def test_f16_seeded_gemm_within_tolerance(M, N, K):
+def test_f16_seeded_gemm_within_tolerance(M, N, K, monkeypatch):
+    monkeypatch.setenv("KREX_GEMM_SPLIT_K", "1")
     seed = 7000 + M + N + K
     a, b = _gen16(seed, M, N, K)
     want = ref.gemm_f64(gen.uniform_f16(seed, 0, M, K), gen.uniform_f16(seed, 1, K, N), dtype="f16")
