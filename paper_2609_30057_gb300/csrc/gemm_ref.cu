@@ -11,7 +11,8 @@
 // of 4x4 blocks at rows {ty*4, 64+ty*4} x cols {g*64 + tx*4 : g < NG}, so its
 // per-k operand reads are conflict-free 16-byte shared loads (two for A, NG
 // for B) for 32*NG FMAs.  Any M, N, K; loads outside the matrix read as zero
-// and stores are guarded.
+// and stores are guarded.  GEMMs of a few tiles use a one-output-per-thread
+// kernel instead, with the same k-order chains (identical bits).
 #include <cuda_fp16.h>
 
 #include <cstdlib>
@@ -172,6 +173,44 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
     }
 }
 
+// Small GEMMs (a few 128x128 tiles would leave most SMs idle): one output per
+// thread, 16x16 outputs per 256-thread block, K in 16-deep shared slices padded
+// with zeros like the large tiling's, so each output is the same k-order FMA
+// chain and both give identical bits.
+template <bool F16>
+__device__ __forceinline__ float widen16(const uint16_t *p, int64_t i) {
+    const uint32_t w = p[i];
+    if constexpr (F16) return __half2float(__ushort_as_half((unsigned short)w));
+    return __uint_as_float(w << 16);
+}
+
+template <bool F16>
+__global__ void __launch_bounds__(256)
+gemm_ref_small(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__restrict__ B, int64_t ldb,
+               float *__restrict__ C, int64_t ldc, int64_t M, int64_t N, int64_t K) {
+    __shared__ float As[16][17], Bs[16][17];
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    const int64_t row = (int64_t)blockIdx.y * 16 + ty, col = (int64_t)blockIdx.x * 16 + tx;
+    float acc = 0.0f;
+    for (int64_t k0 = 0; k0 < K; k0 += 16) {
+        As[ty][tx] = (row < M && k0 + tx < K) ? widen16<F16>(A, row * lda + k0 + tx) : 0.0f;
+        Bs[ty][tx] = (k0 + ty < K && col < N) ? widen16<F16>(B, (k0 + ty) * ldb + col) : 0.0f;
+        __syncthreads();
+#pragma unroll
+        for (int k = 0; k < 16; ++k) acc = fmaf(As[ty][k], Bs[k][tx], acc);
+        __syncthreads();
+    }
+    if (row < M && col < N) C[row * ldc + col] = acc;
+}
+
+template <bool F16>
+cudaError_t launch_small(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
+                         int64_t M, int64_t N, int64_t K, cudaStream_t s) {
+    dim3 grid((unsigned)((N + 15) / 16), (unsigned)((M + 15) / 16));
+    gemm_ref_small<F16><<<grid, 256, 0, s>>>(a, lda, b, ldb, c, ldc, M, N, K);
+    return cudaGetLastError();
+}
+
 template <bool F16, int NG, int TK, int MINB>
 cudaError_t launch_cfg(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
                        int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c_vec, cudaStream_t s) {
@@ -192,24 +231,27 @@ cudaError_t launch_cfg(const uint16_t *a, int64_t lda, const uint16_t *b, int64_
 // / 8192^3, L2 flushed): 53.3/54.5, 49.9/56.6, 50.7/51.8, 43.0/49.0,
 // 54.8/57.2, all bit-identical (each output is one k-order FMA chain); the
 // packed fp32x2 FMA form of 4 ran slower (51.6/54.0), and so did 4 with 32-deep
-// slices (49.8/52.2).  Default: 4.
-int ref_tile() {
+// slices (49.8/52.2).  Default: 4, or 5 (the one-output-per-thread kernel)
+// when the GEMM has at most 16 tiles of 128x128 (L2 flushed: 256^3 30 -> 18
+// us, 512^3 53 -> 47 us; at 768^3, 36 tiles, the tiled form is faster).
+int ref_tile(int64_t M, int64_t N) {
     const char *e = getenv("KREX_REF_TILE");
     if (e) {
         int v = atoi(e);
-        if (v >= 0 && v <= 4) return v;
+        if (v >= 0 && v <= 5) return v;
     }
-    return 4;
+    return ((M + 127) / 128) * ((N + 127) / 128) <= 16 ? 5 : 4;
 }
 
 template <bool F16>
 cudaError_t launch_ref(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
                        int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c_vec, cudaStream_t s) {
-    switch (ref_tile()) {
+    switch (ref_tile(M, N)) {
     case 0: return launch_cfg<F16, 2, 16, 1>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
     case 1: return launch_cfg<F16, 4, 16, 1>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
     case 2: return launch_cfg<F16, 2, 32, 1>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
     case 3: return launch_cfg<F16, 4, 32, 1>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
+    case 5: return launch_small<F16>(a, lda, b, ldb, c, ldc, M, N, K, s);
     default: return launch_cfg<F16, 2, 16, 2>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
     }
 }

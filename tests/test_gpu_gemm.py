@@ -415,18 +415,21 @@ def test_f16_op_rejects_bf16_operands():
 
 
 
-@pytest.mark.parametrize("tile", ["0", "1", "2", "3", "4"])
-def test_reference_tilings_are_bit_identical(tile, monkeypatch):
+@pytest.mark.parametrize("f16", [False, True], ids=["bf16", "f16"])
+@pytest.mark.parametrize("tile", ["0", "1", "2", "3", "4", "5"])
+def test_reference_tilings_are_bit_identical(tile, f16, monkeypatch):
     # every output of the reference is one fp32 FMA chain in k order, so the
-    # tiling must not change a bit (ragged shape: partial tiles in M, N, K)
+    # tiling (5: one output per thread, the small-GEMM form) must not change a
+    # bit (ragged shape: partial tiles in M, N, K)
     M, N, K = 300, 1000, 520
-    a, b = _gen(99, M, N, K)
+    a, b = _gen16(99, M, N, K) if f16 else _gen(99, M, N, K)
+    op = krex.KREX_OP_GEMM_F16 if f16 else krex.KREX_OP_GEMM_BF16
     r0 = torch.empty(M, N, dtype=torch.float32, device="cuda")
     monkeypatch.setenv("KREX_REF_TILE", "0")
-    krex.krex_run_reference(krex.KREX_OP_GEMM_BF16, [a, b], r0)
+    krex.krex_run_reference(op, [a, b], r0)
     r = Guarded(M, N, torch.float32)
     monkeypatch.setenv("KREX_REF_TILE", tile)
-    krex.krex_run_reference(krex.KREX_OP_GEMM_BF16, [a, b], r.view)
+    krex.krex_run_reference(op, [a, b], r.view)
     torch.cuda.synchronize()
     assert r.canaries_intact()
     assert torch.equal(r.view.contiguous().view(torch.int32), r0.view(torch.int32))
