@@ -421,7 +421,9 @@ typedef struct {
     double p50_ms, p95_ms;     /* of the timed iterations */
     int32_t launches;          /* kernels this command launched */
     int32_t reserved;
-    double phase_ms[5];        /* host wall time: inputs, reference, candidate, check, timed loop */
+    double phase_ms[5];        /* inputs, reference, candidate, check: device time between CUDA
+                                  events (the four run back to back; the check's ends when its
+                                  verdict is on the host); timed loop: host wall time */
 } krex_command_result;
 
 /* Run one command.  host_in (may be NULL): if given, host_in[i] (pinned host

@@ -624,8 +624,22 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
         return std::chrono::duration<double, std::milli>(clk::now() - t).count();
     };
 
+    // Phases 1-4 run back to back on the stream and are timed with events
+    // between them (a host synchronisation per phase would add an idle gap to
+    // each); the check ends by reading its verdict back to the host, and its
+    // phase ends with an event recorded after that.  The timed loop is host
+    // wall time.
+    int dev = 0;
+    KREX_CUDA_TRY(cudaGetDevice(&dev));
+    std::vector<cudaEvent_t> pev;
+    KREX_CUDA_TRY(event_pool().take(dev, 5, pev));
+    struct GiveBack {
+        int dev;
+        std::vector<cudaEvent_t> &ev;
+        ~GiveBack() { event_pool().give(dev, ev); }
+    } give_back{dev, pev};
+    KREX_CUDA_TRY(cudaEventRecord(pev[0], s));
     // 1) inputs: generated on the device, or copied from the caller's host buffers
-    auto t = clk::now();
     for (int i = 0; i < n_in; ++i) {
         const krex_buf &b = bufs->in[i];
         if (host_in && host_in[i]) {
@@ -639,27 +653,27 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
             if (st) return st;
         }
     }
-    KREX_CUDA_TRY(cudaStreamSynchronize(s));
-    result->phase_ms[0] = ms_since(t);
+    KREX_CUDA_TRY(cudaEventRecord(pev[1], s));
     // 2) reference
-    t = clk::now();
     if ((st = do_reference(op, bufs->in, bufs->ref, s))) return st;
-    KREX_CUDA_TRY(cudaStreamSynchronize(s));
-    result->phase_ms[1] = ms_since(t);
+    KREX_CUDA_TRY(cudaEventRecord(pev[2], s));
     // 3) candidate once, for the check
-    t = clk::now();
     if ((st = do_candidate(op, bufs->in, bufs->out, s, bufs->gemm_workspace, bufs->gemm_workspace_bytes))) return st;
-    KREX_CUDA_TRY(cudaStreamSynchronize(s));
-    result->phase_ms[2] = ms_since(t);
-    // 4) check
-    t = clk::now();
+    KREX_CUDA_TRY(cudaEventRecord(pev[3], s));
+    // 4) check (synchronous: every earlier phase has completed when it returns)
     if ((st = krex_check(bufs->out, bufs->ref, cmd->atol, cmd->rtol, bufs->check_scratch, bufs->check_scratch_bytes,
                          &result->check, stream)))
         return st;
-    result->phase_ms[3] = ms_since(t);
+    KREX_CUDA_TRY(cudaEventRecord(pev[4], s));
+    KREX_CUDA_TRY(cudaEventSynchronize(pev[4]));
+    for (int i = 0; i < 4; ++i) {
+        float ms = 0.0f;
+        KREX_CUDA_TRY(cudaEventElapsedTime(&ms, pev[i], pev[i + 1]));
+        result->phase_ms[i] = ms;
+    }
     result->passed = result->check.n_violations == 0;
     // 5) timed loop inside a critical region (skipped when the check failed)
-    t = clk::now();
+    const auto t = clk::now();
     result->p50_ms = result->p95_ms = NAN;
     if (result->passed) {
         krex_region_opts o;

@@ -2,6 +2,7 @@
 reference, candidate, check, timed loop — on small and full workloads, with
 device-generated and host-supplied inputs."""
 import ctypes
+import time
 
 import numpy as np
 import pytest
@@ -84,3 +85,20 @@ def test_f16_gemm_command_matches_oracle():
     assert np.all(np.abs(got - want) <= ref.gemm_tolerance(want, w.K, dtype="f16"))
     assert np.array_equal(bits16(ws.inputs[0]), gen.uniform_f16(w.seed, 0, w.M, w.K))
 
+
+
+def test_phase_times_are_positive_and_within_the_command():
+    # inputs, reference, candidate and check are timed between CUDA events on
+    # the command's stream, the timed loop on the host clock: every phase is
+    # positive and together they fit inside the command's wall time
+    w = WORKLOADS["gemm_bf16_256"]
+    ws = Workspace(w)
+    ws.run()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    r = ws.run()
+    torch.cuda.synchronize()
+    wall_ms = (time.perf_counter() - t0) * 1e3
+    ph = list(r.phase_ms)
+    assert all(p > 0 for p in ph), ph
+    assert sum(ph) <= wall_ms * 1.02 + 0.02, (ph, wall_ms)
