@@ -10,11 +10,16 @@ iterations each preceded by an L2-flush write).  Every step is one
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
   python bench.py --impl reference ...   # the CPU oracle, timed on host cores
 
-The JSON line carries: value (commands/s, device-timed with inputs resident),
-e2e (the same metric with host-resident inputs and outputs copied inside the
-timed region), roofline (the GEMM kernel, from the per-iteration CUDA events
-of the commands' timed loops), kernels (each kernel of the path timed alone
-with CUDA events), cpu_baseline (the oracle on a bounded sample), clocks.
+The default workload is the 16384^3 GEMM command, 32 commands per
+measurement.  The JSON line carries: value (commands/s, device-timed with
+inputs resident), e2e (the same metric with host-resident inputs and outputs
+copied inside the timed region), roofline (the tcgen05 GEMM candidate, from
+the per-iteration CUDA events of the commands' timed loops),
+roofline_reference (the CUDA-core reference GEMM on the FP32 FMA pipe),
+configs (one sub-record per workload of the configuration list: commands/s,
+the candidate's roofline, p50/p95, P across commands), kernels (each kernel
+of the path timed alone with CUDA events), cpu_baseline (the oracle on a
+bounded sample, measured), clocks.
 Under torchrun (N > 1) every rank runs independent commands on its own GPU
 (replicas; no data-path collective) and rank 0 reports the aggregate.
 """
@@ -22,16 +27,13 @@ from __future__ import annotations
 
 import argparse
 import csv
-import ctypes
 import hashlib
 import io
 import json
-import math
 import os
 import statistics
 import subprocess
 import sys
-import threading
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -39,14 +41,24 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "GEMM TFLOP/s & fill/flush/softmax/check GB/s vs roofline; bench cmds/s, 1 GB300"
-DEFAULT_WORKLOAD = "gemm_bf16_4096"
+# the headline: the 16384^3 GEMM command, repeated 32 times to report commands/s
+DEFAULT_WORKLOAD = "gemm_bf16_16384"
+# every workload of the configuration list, each measured as a sub-record, with
+# the number of commands timed for it
+CONFIG_WORKLOADS = {"gemm_bf16_256": 32, "gemm_bf16_4096": 20, "softmax_f32_65536x8192": 10,
+                    "gemm_bf16_8192": 8, "gemm_bf16_16384": 32}
 SOFTMAX_WORKLOAD = "softmax_f32_65536x8192"
+SMALL_GEMM_WORKLOAD = "gemm_bf16_4096"
 # 32-bit integer-ALU operations the uniform generator's definition takes per
 # 16-bit element: per SplitMix64 draw (two elements) a 64-bit add (2) and three
 # 64-bit xor-shifts (2 funnel shifts + 2 xors each: 12); per element the 24-bit
 # field to [-1, 1) (a shift, two masks, an integer subtract: 4).  The two 64-bit
-# multiplies per draw run on the multiply-add pipe and are not counted.
+# multiplies per draw (3 multiply-adds each) run on the multiply-add pipe and
+# are counted separately (FILL_IMAD_OPS_PER_ELEMENT).
 FILL_ALU_OPS_PER_ELEMENT = (2 + 12) / 2 + 4
+FILL_IMAD_OPS_PER_ELEMENT = (2 * 3) / 2
+# FP32 fused multiply-add lanes per SM (the CUDA-core reference GEMM's pipe)
+FMA_LANES_PER_SM = 128
 
 
 def _peaks():
@@ -154,129 +166,189 @@ def _time_launches(fn, n, stream, flush=None):
     return statistics.fmean(a.elapsed_time(b) for a, b in evs)
 
 
-def kernel_table(ws, w, peaks, stream):
+def kernel_table(peaks, stream, gemm_names=(DEFAULT_WORKLOAD, SMALL_GEMM_WORKLOAD)):
     """Each kernel of the path timed alone (after warm-up, L2 flushed before
-    every launch), with its algorithmic bytes or flops per launch."""
+    every launch), with its algorithmic bytes or flops per launch: the GEMM
+    path's kernels at the sizes of `gemm_names`, the softmax path's at its
+    workload's size."""
     import torch
     import paper_2609_30057_gb300 as krex
     from paper_2609_30057_gb300.command import WORKLOADS, Workspace
-    if not w.is_gemm:               # the GEMM rows run at the GEMM workload's size
-        w = WORKLOADS[DEFAULT_WORKLOAD]
-        ws = Workspace(w)
-    flush_t = ws.flush
-    flush = lambda: krex.krex_flush_l2(flush_t, stream=stream)  # noqa: E731
     out = {}
-
+    dev = torch.cuda.current_device()
+    n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
     # integer-ALU roofline of the uniform fill: 64 ALU lanes per clock per SM
     # at the 2070 MHz maximum SM clock (the clock the runs see under load)
-    alu_peak = torch.cuda.get_device_properties(stream.device).multi_processor_count * 64 * 2.070e9
+    alu_peak = n_sm * 64 * 2.070e9
 
-    def rec(name, fn, nbytes=None, flops=None, alu_ops=None, n=20, do_flush=True):
+    def rec(name, fn, flush, nbytes=None, flops=None, alu_ops=None, n=20, fma_peak=None):
         for _ in range(3):
             fn()
-        ms = _time_launches(fn, n, stream, flush if do_flush else None)
-        e = {"ms": ms}
+        ms = _time_launches(fn, n, stream, flush)
+        e = {"ms": ms, "launches": n}
         if nbytes is not None:
             gbs = nbytes / ms / 1e6
             e.update({"GB/s": gbs, "frac_hbm": gbs / peaks["hbm_gbs"], "bytes": nbytes})
         if flops is not None:
             tf = flops / ms / 1e9
-            e.update({"TFLOP/s": tf, "frac_bf16": tf / peaks["bf16_tflops"], "flops": flops})
+            e.update({"TFLOP/s": tf, "flops": flops})
+            if fma_peak is None:
+                e["frac_bf16"] = tf / peaks["bf16_tflops"]
+            else:
+                e.update({"bound": "fp32 fma", "frac_fma": tf * 1e12 / fma_peak})
         if alu_ops is not None:
             e.update({"bound": "alu", "alu_ops": alu_ops, "Tops/s": alu_ops / ms / 1e9,
                       "frac_alu": alu_ops / ms * 1e3 / alu_peak})
         out[name] = e
 
-    A, B = ws.inputs
-    rec("fill_uniform_bf16", lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, A, stream), nbytes=A.numel() * 2,
-        alu_ops=A.numel() * FILL_ALU_OPS_PER_ELEMENT)
-    big = torch.empty(16384, 16384, dtype=torch.bfloat16, device=A.device)   # steady state, 512 MiB
-    rec("fill_uniform_bf16_16384", lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, big, stream),
-        nbytes=big.numel() * 2, alu_ops=big.numel() * FILL_ALU_OPS_PER_ELEMENT, n=10)
-    del big
-    rec("flush_l2", flush, nbytes=flush_t.numel(), do_flush=False)
-    rec("gemm_ref_simt", lambda: krex.krex_run_reference(w.op, ws.inputs, ws.ref, stream), flops=w.flops, n=3)
-    rec("gemm_tcgen05", lambda: krex.krex_run_candidate_ws(w.op, ws.inputs, ws.out, ws.gemm_ws, stream),
-        flops=w.flops)
-    scratch = ws.check_scratch
-    rec("check_bf16_f32", lambda: krex.krex_check_launch(ws.out, ws.ref, w.atol, w.rtol, scratch, stream),
-        nbytes=ws.out.numel() * 6, n=10)
+    for gname in gemm_names:
+        w = WORKLOADS[gname]
+        ws = Workspace(w)
+        sfx = f"@{w.M}"
+        flush = lambda ws=ws: krex.krex_flush_l2(ws.flush, stream=stream)  # noqa: E731
+        A, B = ws.inputs
+        rec("fill_uniform_bf16" + sfx, lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, A, stream), flush,
+            nbytes=A.numel() * 2, alu_ops=A.numel() * FILL_ALU_OPS_PER_ELEMENT, n=10)
+        krex.krex_gen_inputs(w.seed, 1, 0, 0.0, B, stream)
+        if gname == gemm_names[0]:
+            rec("flush_l2", flush, None, nbytes=ws.flush.numel())
+        rec("gemm_ref_simt" + sfx, lambda: krex.krex_run_reference(w.op, ws.inputs, ws.ref, stream), flush,
+            flops=w.flops, n=2 if w.M >= 16384 else 3, fma_peak=n_sm * FMA_LANES_PER_SM * 2 * 2.070e9)
+        rec("gemm_tcgen05" + sfx, lambda: krex.krex_run_candidate_ws(w.op, ws.inputs, ws.out, ws.gemm_ws, stream),
+            flush, flops=w.flops, n=10 if w.M >= 16384 else 20)
+        rec("check_bf16_f32" + sfx,
+            lambda: krex.krex_check_launch(ws.out, ws.ref, w.atol, w.rtol, ws.check_scratch, stream), flush,
+            nbytes=ws.out.numel() * 6, n=10)
+        del ws, A, B
+        torch.cuda.empty_cache()
     # the bandwidth-bound candidate at its own workload size
     sw = WORKLOADS[SOFTMAX_WORKLOAD]
-    x = torch.empty(sw.M, sw.N, dtype=torch.float32, device=A.device)
-    y = torch.empty_like(x)
-    rec("fill_normal_f32", lambda: krex.krex_gen_inputs(sw.seed, 0, 1, sw.sigma, x, stream), nbytes=x.numel() * 4,
-        n=10)
-    rec("softmax_f32", lambda: krex.krex_run_candidate(1, [x], y, stream), nbytes=x.numel() * 8, n=10)
-    rec("check_f32_f32", lambda: krex.krex_check_launch(y, x, 1e-6, 0.0, scratch, stream), nbytes=x.numel() * 8, n=5)
-    del x, y
-    # the fp16 form of the GEMM candidate at the same size
+    sws = Workspace(sw)
+    flush = lambda: krex.krex_flush_l2(sws.flush, stream=stream)  # noqa: E731
+    x, y = sws.inputs[0], sws.out
+    rec("fill_normal_f32", lambda: krex.krex_gen_inputs(sw.seed, 0, 1, sw.sigma, x, stream), flush,
+        nbytes=x.numel() * 4, n=10)
+    rec("softmax_f32", lambda: krex.krex_run_candidate(1, [x], y, stream), flush, nbytes=x.numel() * 8, n=10)
+    rec("check_f32_f32", lambda: krex.krex_check_launch(y, x, 1e-6, 0.0, sws.check_scratch, stream), flush,
+        nbytes=x.numel() * 8, n=5)
+    del sws, x, y
+    # the fp16 form of the GEMM candidate at 4096^3
     fw = WORKLOADS["gemm_f16_4096"]
-    a16 = torch.empty(fw.M, fw.K, dtype=torch.float16, device=A.device)
-    b16 = torch.empty(fw.K, fw.N, dtype=torch.float16, device=A.device)
-    c16 = torch.empty(fw.M, fw.N, dtype=torch.float16, device=A.device)
-    rec("fill_uniform_f16", lambda: krex.krex_gen_inputs(fw.seed, 0, 0, 0.0, a16, stream), nbytes=a16.numel() * 2,
-        alu_ops=a16.numel() * FILL_ALU_OPS_PER_ELEMENT)
+    fws = Workspace(fw)
+    flush = lambda: krex.krex_flush_l2(fws.flush, stream=stream)  # noqa: E731
+    a16, b16 = fws.inputs
+    rec("fill_uniform_f16@4096", lambda: krex.krex_gen_inputs(fw.seed, 0, 0, 0.0, a16, stream), flush,
+        nbytes=a16.numel() * 2, alu_ops=a16.numel() * FILL_ALU_OPS_PER_ELEMENT)
     krex.krex_gen_inputs(fw.seed, 1, 0, 0.0, b16, stream)
-    rec("gemm_tcgen05_f16", lambda: krex.krex_run_candidate_ws(fw.op, [a16, b16], c16, ws.gemm_ws, stream),
-        flops=fw.flops)
-    del a16, b16, c16
+    rec("gemm_tcgen05_f16@4096", lambda: krex.krex_run_candidate_ws(fw.op, fws.inputs, fws.out, fws.gemm_ws, stream),
+        flush, flops=fw.flops)
+    del fws, a16, b16
     torch.cuda.empty_cache()
     return out
 
 
 # ---------------------------------------------------------- CPU oracle ------
 
-def oracle_command_cost(w, budget_s: float = 10.0):
-    """Seconds one benchmarking command of workload `w` takes when the oracle
-    does its arithmetic on the host: generate the inputs, the GEMM once for the
-    reference and once per candidate run (1 + warm-up + iters), the check.
-    Bounded sample: the GEMM is timed on a block of output rows and scaled by
-    M / rows; generation and the check run in full.  Returns (seconds, info)."""
+def _oracle_block(w):
+    """The block of one workload's output that one oracle step computes:
+    (rows, cols) of C for a GEMM (cols = N for the small GEMM, whose whole
+    command is one step), rows for the softmax."""
+    if w.is_gemm:
+        if w.M * w.N <= 256 * 256:
+            return w.M, w.N
+        return 256, 256
+    return 128, w.N
+
+
+def oracle_command_fraction(w, step: int):
+    """One step of the oracle as a benchmarking command's program on the host:
+    the work of a block of the command's output, executed in full.  For block
+    b of C (r rows, c columns): generate the r rows of A and c columns of B the
+    block needs; compute the block with the oracle's fp64 GEMM once for the
+    reference, once for the candidate's checked run and once per warm-up and
+    timed candidate run; check the block (fp32, oracle check).  The softmax
+    does the same on r rows.  The block is a fraction f = r*c / (M*N) of the
+    command's output; the step's generation covers more than f of the inputs
+    (whole operand rows and columns), so f / seconds understates the oracle's
+    command rate.  Blocks walk the output in order with `step`.
+    Returns (f, seconds, description)."""
     import numpy as np
     from oracle import gen, ref
+    r, c = _oracle_block(w)
+    runs = 1 + 1 + w.warmup + w.iters
     t0 = time.perf_counter()
     if w.is_gemm:
-        a = gen.uniform(w.dtype, w.seed, 0, w.M, w.K)
-        b = gen.uniform(w.dtype, w.seed, 1, w.K, w.N)
+        nbr, nbc = w.M // r, w.N // c
+        br, bc = (step // max(1, nbc)) % max(1, nbr), step % max(1, nbc)
+        r0, c0 = br * r, bc * c
+        kk = np.arange(w.K, dtype=np.int64)
+        a_idx = (r0 + np.arange(r, dtype=np.int64))[:, None] * w.K + kk[None, :]
+        b_idx = kk[:, None] * w.N + (c0 + np.arange(c, dtype=np.int64))[None, :]
+        a = gen.uniform_at(w.dtype, w.seed, 0, a_idx.ravel()).reshape(r, w.K)
+        b = gen.uniform_at(w.dtype, w.seed, 1, b_idx.ravel()).reshape(w.K, c)
+        for _ in range(runs):
+            blk = ref.gemm_f64(a, b, dtype=w.dtype)
+        what = f"a {r}x{c} block of C (K = {w.K}): {r} rows of A and {c} columns of B generated"
     else:
-        x = gen.normal_f32(w.seed, 0, min(w.M, 2048), w.N, w.sigma)
-    t_gen = time.perf_counter() - t0
-    if not w.is_gemm:
-        t_gen *= w.M / min(w.M, 2048)
-    rows = 0
-    t_work = 0.0
-    reps = 0
-    tb = time.perf_counter()
-    block = 64 if w.is_gemm else 256
-    while time.perf_counter() - tb < budget_s * 0.6 and rows < w.M:
-        t1 = time.perf_counter()
-        if w.is_gemm:
-            c = ref.gemm_f64(a[rows % w.M:rows % w.M + block], b, dtype=w.dtype)
-        else:
-            c = ref.softmax_rows_f64(x[:block].astype(np.float64))
-        t_work += time.perf_counter() - t1
-        rows += block
-        reps += 1
-    per_full = t_work * (w.M / rows)
-    t1 = time.perf_counter()
-    n_chk = min(w.M, 2048)
-    o32 = c[:1].astype(np.float32).repeat(n_chk, axis=0)
-    ref.check_f32(o32, o32, w.atol, w.rtol)
-    t_chk = (time.perf_counter() - t1) * (w.M / n_chk)
-    runs = 1 + 1 + w.warmup + w.iters
-    total = t_gen + runs * per_full + t_chk
-    info = (f"oracle command of {w.name}: input generation in full (single thread), "
-            f"{'fp64 GEMM' if w.is_gemm else 'fp64 softmax'} on {rows} of {w.M} output rows scaled to the full "
-            f"output and counted {runs}x (reference + check run + {w.warmup} warm-up + {w.iters} timed), "
-            f"fp32 check on {n_chk} rows scaled; sample wall {time.perf_counter() - t0:.1f} s")
-    in_bytes = (w.M * w.K + w.K * w.N) * 2 if w.is_gemm else w.M * w.N * 4
-    comp = {"gen_GB_per_s": in_bytes / t_gen / 1e9, "check_GB_per_s": w.M * w.N * (6 if w.is_gemm else 8) / t_chk / 1e9}
-    if w.is_gemm:
-        comp["gemm_fp64_GFLOP_per_s"] = 2.0 * w.M * w.N * w.K / per_full / 1e9
-    else:
-        comp["softmax_fp64_rows_per_s"] = w.M / per_full
-    return total, info, comp
+        r0 = (step * r) % w.M
+        x = gen.normal_f32_at(w.seed, 0, (r0 * w.N + np.arange(r * w.N, dtype=np.int64)), w.sigma).reshape(r, w.N)
+        for _ in range(runs):
+            blk = ref.softmax_rows_f64(x.astype(np.float64))
+        what = f"{r} rows of {w.N} generated"
+    b32 = blk.astype(np.float32)
+    ref.check_f32(b32, b32, w.atol, w.rtol)
+    secs = time.perf_counter() - t0
+    frac = (r * c) / (w.M * w.N)
+    info = (f"{what}, computed {runs} times in fp64 (reference + checked run + {w.warmup} warm-up + {w.iters} "
+            f"timed) and checked in fp32; a fraction {frac:.3g} of one command's output, executed in full")
+    return frac, secs, info
+
+
+def oracle_rate(w, budget_s: float, first_step: int = 0):
+    """Commands/s of the oracle over consecutive steps until `budget_s` of
+    host time has passed (at least one step): total fraction / total time."""
+    f_tot = t_tot = 0.0
+    step = first_step
+    info = ""
+    while True:
+        f, t, info = oracle_command_fraction(w, step)
+        f_tot += f
+        t_tot += t
+        step += 1
+        if t_tot >= budget_s:
+            break
+    return f_tot / t_tot, step - first_step, t_tot, info
+
+
+def oracle_full_command(w):
+    """The oracle running one whole command of a small workload, unextrapolated:
+    generate A and B, the fp64 GEMM for the reference, the checked run, the
+    warm-up and the timed runs, the fp32 check.  Returns seconds."""
+    from oracle import gen, ref
+    t0 = time.perf_counter()
+    a = gen.uniform(w.dtype, w.seed, 0, w.M, w.K)
+    b = gen.uniform(w.dtype, w.seed, 1, w.K, w.N)
+    for _ in range(1 + 1 + w.warmup + w.iters):
+        c = ref.gemm_f64(a, b, dtype=w.dtype)
+    c32 = c.astype("float32")
+    ref.check_f32(c32, c32, w.atol, w.rtol)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline_record(w, budget_s: float = 12.0):
+    """The oracle as it stands on the host cores (a bounded sample of the
+    workload), plus one whole small command timed in full."""
+    from paper_2609_30057_gb300.command import WORKLOADS
+    rate, steps, secs, info = oracle_rate(w, budget_s)
+    small = WORKLOADS["gemm_bf16_256"]
+    full_s = oracle_full_command(small)
+    return {"value": rate, "unit": "cmds/s", "cores": cpu_cores(), "kind": "oracle",
+            "sample": (f"{steps} oracle steps of {w.name}, {secs:.1f} s of host time measured; each step: {info}; "
+                       f"value = fractions of a command executed / measured seconds"),
+            "measured_wall_s": secs, "steps": steps,
+            "threads": "fp64 GEMM through numpy's BLAS on all host cores; generation and check single-threaded",
+            "cpu_model": cpu_model(),
+            "full_command_unextrapolated": {"workload": small.name, "seconds": full_s, "cmds_per_s": 1.0 / full_s}}
 
 
 def _p95(xs) -> float:
@@ -305,16 +377,120 @@ def cpu_model() -> str:
     return platform.machine()
 
 
+def workload_config(w, world: int) -> dict:
+    """The `config` object of a JSON line (the same keys for both arms)."""
+    return {"workload": w.name, "M": w.M, "N": w.N, "K": w.K, "seed": w.seed, "timed_iters": w.iters,
+            "warmup_iters": w.warmup, "flush_bytes": w.flush_bytes, "commands_per_measurement": w.repeat,
+            "l2": "flushed: a flush_bytes write precedes every timed candidate iteration and region entry",
+            "parallelism": f"replicas{world}"}
+
+
 # ------------------------------------------------------------- main ---------
+
+def candidate_roofline(w, mean_ms: float, peaks) -> dict:
+    """The candidate kernel's roofline from its mean CUDA-event duration."""
+    if w.is_gemm:
+        achieved = w.flops / (mean_ms / 1e3) / 1e12
+        return {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
+                "frac": achieved / peaks["bf16_tflops"], "traffic": _ncu_traffic("gemm_tcgen05", w.name),
+                "peak_kind": f"bf16 dense burst, {peaks['source']} (MEASURED_PEAKS.json)",
+                "frac_of_sustained": (achieved / peaks["bf16_tflops_sustained"]
+                                      if peaks.get("bf16_tflops_sustained") else None),
+                "kernel": "gemm_tcgen05_2sm", "algorithmic_flops_per_launch": w.flops}
+    # the bandwidth-bound candidate: one read and one write of the matrix
+    achieved = w.candidate_bytes / (mean_ms / 1e3) / 1e9
+    return {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": achieved / peaks["hbm_gbs"], "traffic": _ncu_traffic("softmax_rows", w.name),
+            "peak_kind": f"HBM copy, {peaks['source']} (MEASURED_PEAKS.json)",
+            "kernel": "softmax_rows_reg", "algorithmic_bytes_per_launch": w.candidate_bytes}
+
+
+def reference_roofline(w, mean_ms: float, n_sm: int, sm_mhz) -> dict | None:
+    """The CUDA-core reference GEMM on the FP32 fused multiply-add pipe: peak =
+    SMs x 128 FMA lanes x 2 flops x clock (the 2070 MHz maximum; also at the
+    median SM clock sampled during the run)."""
+    if not w.is_gemm:
+        return None
+    achieved = w.flops / (mean_ms / 1e3) / 1e12
+    peak = n_sm * FMA_LANES_PER_SM * 2 * 2.070e9 / 1e12
+    r = {"bound": "alu", "pipe": "fp32 fma", "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
+         "frac": achieved / peak, "traffic": _ncu_traffic("gemm_ref_simt", w.name),
+         "peak_kind": f"derived: {n_sm} SMs x {FMA_LANES_PER_SM} FP32 FMA lanes x 2 flops x 2070 MHz",
+         "kernel": "gemm_ref_simt", "algorithmic_flops_per_launch": w.flops, "ms_per_launch": mean_ms}
+    if sm_mhz:
+        r["frac_at_sampled_clock"] = achieved / (peak * sm_mhz / 2070.0)
+    return r
+
+
+def measure_commands(ws, n: int, stream):
+    """n back-to-back commands timed with CUDA events on `stream`; returns
+    (elapsed ms, candidate durations, p50s, p95s, phases)."""
+    import torch
+    cand, p50s, p95s, phases = [], [], [], []
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(n):
+        r = ws.run()
+        if not r.passed:
+            raise SystemExit(f"{ws.w.name}: check failed: {r.check.n_violations} violations")
+        cand.extend(ws.durations[: r.n_iters])
+        p50s.append(r.p50_ms)
+        p95s.append(r.p95_ms)
+        phases.append(list(r.phase_ms))
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    return ev0.elapsed_time(ev1), cand, p50s, p95s, phases
+
+
+def spread(p50s, p95s) -> dict:
+    m50 = statistics.median(p50s)
+    return {"p50_ms_median": m50, "p95_ms_median": statistics.median(p95s),
+            "p95_over_p50_minus_1": statistics.median(p95s) / m50 - 1.0,
+            # Eq. 1 across the commands: p95 of (command median / overall median) - 1
+            "P_across_commands": _p95([p / m50 for p in p50s]) - 1.0}
+
+
+def config_records(names, peaks, stream, n_sm, skip=()):
+    """One sub-record per workload of the configuration list: commands/s,
+    the candidate's roofline, p50/p95 and P across commands."""
+    import torch
+    from paper_2609_30057_gb300.command import WORKLOADS, Workspace
+    out = {}
+    for name in names:
+        if name in skip:
+            continue
+        w = WORKLOADS[name]
+        n = CONFIG_WORKLOADS[name]
+        ws = Workspace(w)
+        for _ in range(2):
+            ws.run()
+        torch.cuda.synchronize()
+        ms, cand, p50s, p95s, phases = measure_commands(ws, n, stream)
+        ph = [statistics.fmean(p[i] for p in phases) for i in range(5)]
+        rl = candidate_roofline(w, statistics.fmean(cand), peaks)
+        rec = {"commands": n, "cmds_per_s": n / (ms / 1e3), "ms_per_command": ms / n,
+               "candidate": {k: rl[k] for k in ("kernel", "achieved", "unit", "peak", "frac")},
+               "phase_ms": dict(zip(["inputs", "reference", "candidate", "check", "timed_loop"], ph))}
+        rr = reference_roofline(w, ph[1], n_sm, None)
+        if rr:
+            rec["reference"] = {k: rr[k] for k in ("kernel", "achieved", "unit", "peak", "frac")}
+        rec.update(spread(p50s, p95s))
+        out[name] = rec
+        del ws
+        torch.cuda.empty_cache()
+    return out
+
 
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="commands timed (default: the workload's commands per measurement, else 20)")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-kernels", action="store_true", help="skip the per-kernel table")
+    ap.add_argument("--no-configs", action="store_true", help="skip the per-configuration sub-records")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--kernel-only", default=None,
@@ -324,16 +500,20 @@ def main():
     args = ap.parse_args()
 
     from paper_2609_30057_gb300 import replicas
+    from paper_2609_30057_gb300.command import WORKLOADS
     rank, world, local_rank = replicas.rank_world()
+    w = WORKLOADS[args.workload]
+    if args.steps is None:
+        args.steps = w.repeat if w.repeat > 1 else 20
 
     if args.impl == "reference":
-        return reference_arm(args, rank, world)
+        return reference_arm(args, w, rank, world)
     if args.kernel_only:
         return kernel_only(args)
 
     import torch
     import paper_2609_30057_gb300 as krex
-    from paper_2609_30057_gb300.command import WORKLOADS, Workspace
+    from paper_2609_30057_gb300.command import Workspace
 
     torch.cuda.set_device(local_rank)
     dist = None
@@ -345,10 +525,10 @@ def main():
     if world > 1:
         dist.barrier()
 
-    w = WORKLOADS[args.workload]
     peaks = _peaks()
     ws = Workspace(w)
     stream = torch.cuda.current_stream()
+    n_sm = torch.cuda.get_device_properties(local_rank).multi_processor_count
 
     def barrier():
         replicas.barrier(dist)
@@ -359,25 +539,13 @@ def main():
             raise SystemExit(f"check failed during warm-up: {r.check.n_violations} violations")
 
     # ------------------------------------------------ timed region (value)
-    gemm_ms, p50s, p95s, phases = [], [], [], []
     clocks = ClockSampler(torch.cuda.current_device())
     barrier()
     torch.cuda.synchronize()
     launches0 = krex.krex_launch_count()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with clocks:
-        ev0.record(stream)
         t0 = time.perf_counter()
-        for _ in range(args.steps):
-            r = ws.run()
-            if not r.passed:
-                raise SystemExit(f"check failed: {r.check.n_violations} violations")
-            gemm_ms.extend(ws.durations[: r.n_iters])
-            p50s.append(r.p50_ms)
-            p95s.append(r.p95_ms)
-            phases.append(list(r.phase_ms))
-        ev1.record(stream)
-        torch.cuda.synchronize()
+        elapsed, cand_ms, p50s, p95s, phases = measure_commands(ws, args.steps, stream)
         wall = time.perf_counter() - t0
     barrier()
     launches = int(replicas.sum_over_ranks(dist, krex.krex_launch_count() - launches0, device="cuda"))
@@ -385,7 +553,7 @@ def main():
     status = krex.krex_device_status()
     if status:
         raise SystemExit(f"a kernel reported device status {status:#x} during the timed region")
-    elapsed_ms = replicas.max_over_ranks(dist, ev0.elapsed_time(ev1), device="cuda")
+    elapsed_ms = replicas.max_over_ranks(dist, elapsed, device="cuda")
     value = replicas.aggregate_throughput(args.steps, world, elapsed_ms / 1e3)
 
     # ------------------------------------------------ e2e (host buffers)
@@ -396,7 +564,7 @@ def main():
             h.copy_(t)
         host_out = torch.empty(ws.out.shape, dtype=ws.out.dtype).pin_memory()
         ptrs = [h.data_ptr() for h in host_in]
-        for _ in range(max(1, args.warmup)):
+        for _ in range(max(1, min(args.warmup, 2))):
             ws.run(host_in=ptrs, host_out=host_out.data_ptr())
         barrier()
         torch.cuda.synchronize()
@@ -413,60 +581,61 @@ def main():
         e2e = {"value": replicas.aggregate_throughput(args.steps, world, te_ms / 1e3), "unit": "cmds/s",
                "h2d_bytes_per_step": sum(h.numel() * h.element_size() for h in host_in),
                "d2h_bytes_per_step": host_out.numel() * host_out.element_size() + 16}
+        del host_in, host_out
 
-    kernels = None if args.no_kernels or rank != 0 else kernel_table(ws, w, peaks, stream)
+    cs = clocks.summary()
+    ph = [statistics.fmean(p[i] for p in phases) for i in range(5)]
+    headline = {"commands": args.steps, "cmds_per_s": args.steps / (elapsed / 1e3),
+                "ms_per_command": elapsed / args.steps}
+    rl_c = candidate_roofline(w, statistics.fmean(cand_ms), peaks)
+    rl_c["launches_timed"] = len(cand_ms)
+    rl_r = reference_roofline(w, ph[1], n_sm, cs.get("sm_mhz") if cs else None)
+    if rl_r:
+        rl_r["launches_timed"] = len(phases)
+    del ws
+    torch.cuda.empty_cache()
+
+    configs = None
+    kernels = None
+    if rank == 0:
+        if not args.no_configs:
+            configs = config_records(list(CONFIG_WORKLOADS), peaks, stream, n_sm, skip=(w.name,))
+            hl = dict(headline)
+            hl["candidate"] = {k: rl_c[k] for k in ("kernel", "achieved", "unit", "peak", "frac")}
+            if rl_r:
+                hl["reference"] = {k: rl_r[k] for k in ("kernel", "achieved", "unit", "peak", "frac")}
+            hl["phase_ms"] = dict(zip(["inputs", "reference", "candidate", "check", "timed_loop"], ph))
+            hl.update(spread(p50s, p95s))
+            configs[w.name] = {"headline": True, **hl}
+        if not args.no_kernels:
+            gnames = (w.name, SMALL_GEMM_WORKLOAD) if w.is_gemm and w.name != SMALL_GEMM_WORKLOAD \
+                else (SMALL_GEMM_WORKLOAD,)
+            kernels = kernel_table(peaks, stream, gnames)
 
     if rank != 0:
         if dist is not None:
             dist.destroy_process_group()
         return
 
-    # ------------------------------------------------ roofline (GEMM kernel)
-    mean_gemm_ms = statistics.fmean(gemm_ms)
-    if w.is_gemm:
-        achieved = w.flops / (mean_gemm_ms / 1e3) / 1e12
-        roofline = {"bound": "tensor", "achieved": achieved, "peak": peaks["bf16_tflops"], "unit": "TFLOP/s",
-                    "frac": achieved / peaks["bf16_tflops"], "traffic": _ncu_traffic("gemm_tcgen05", w.name),
-                    "peak_kind": f"bf16 dense burst, {peaks['source']} (MEASURED_PEAKS.json)",
-                    "frac_of_sustained": (achieved / peaks["bf16_tflops_sustained"]
-                                          if peaks.get("bf16_tflops_sustained") else None),
-                    "kernel": "gemm_tcgen05_2sm", "launches_timed": len(gemm_ms),
-                    "algorithmic_flops_per_launch": w.flops}
-    else:
-        # the bandwidth-bound candidate: one read and one write of the matrix
-        achieved = w.candidate_bytes / (mean_gemm_ms / 1e3) / 1e9
-        roofline = {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                    "frac": achieved / peaks["hbm_gbs"], "traffic": _ncu_traffic("softmax_rows", w.name),
-                    "peak_kind": f"HBM copy, {peaks['source']} (MEASURED_PEAKS.json)",
-                    "kernel": "softmax_rows_reg", "launches_timed": len(gemm_ms),
-                    "algorithmic_bytes_per_launch": w.candidate_bytes}
-
     cpu = None
     if not args.no_cpu_baseline and world == 1:   # the host baseline is a single-GPU figure
-        secs, info, comp = oracle_command_cost(w)
-        cpu = {"value": 1.0 / secs, "unit": "cmds/s", "cores": cpu_cores(), "kind": "oracle", "sample": info,
-               "components": comp, "cpu_model": cpu_model()}
+        cpu = cpu_baseline_record(w)
 
-    cs = clocks.summary()
-    ph = [statistics.fmean(p[i] for p in phases) for i in range(5)]
     line = {
         "metric": METRIC, "value": value, "unit": "cmds/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": {"bf16": "bf16", "f16": "f16"}.get(w.dtype, "f32"), "data": "synthetic",
-        "config": {"workload": w.name, "M": w.M, "N": w.N, "K": w.K, "seed": w.seed, "timed_iters": w.iters,
-                   "warmup_iters": w.warmup, "flush_bytes": w.flush_bytes,
-                   "l2": "flushed: a flush_bytes write precedes every timed candidate iteration and region entry",
-                   "parallelism": f"replicas{world}"},
-        "roofline": roofline,
+        "scaling": "weak", "vs_baseline": None, "dtype": {"bf16": "bf16", "f16": "f16"}.get(w.dtype, "f32"),
+        "data": "synthetic",
+        "config": workload_config(w, world),
+        "roofline": rl_c,
+        "roofline_reference": rl_r,
         "cpu_baseline": cpu,
         "e2e": e2e,
         "gpu_launches": launches,
         "clocks": cs,
-        "timing_spread": {"p50_ms_median": statistics.median(p50s), "p95_ms_median": statistics.median(p95s),
-                          "p95_over_p50_minus_1": statistics.median(p95s) / statistics.median(p50s) - 1.0,
-                          # Eq. 1 across the commands: p95 of (command median / overall median) - 1
-                          "P_across_commands": _p95([p / statistics.median(p50s) for p in p50s]) - 1.0},
+        "timing_spread": spread(p50s, p95s),
         "phase_ms": dict(zip(["inputs", "reference", "candidate", "check", "timed_loop"], ph)),
+        "configs": configs,
         "kernels": kernels,
         "host_wall_s": wall,
     }
@@ -517,31 +686,34 @@ def kernel_only(args):
     print(json.dumps({"kernel_only": k, "workload": w.name, "launches": args.launches}))
 
 
-def reference_arm(args, rank, world):
-    """The oracle as the reference arm: each step is one bounded-sample oracle
-    command on the host cores; rank 0 alone runs it."""
+def reference_arm(args, w, rank, world):
+    """The oracle as the reference arm: each step executes a block of one
+    command of the workload in full on the host cores (oracle_command_fraction);
+    value = fractions of a command executed / measured seconds.  Rank 0 alone
+    runs it."""
     if rank != 0:
         return
-    from paper_2609_30057_gb300.command import WORKLOADS
-    w = WORKLOADS[args.workload]
-    budget = max(1.0, min(10.0, 150.0 / max(1, args.steps + args.warmup)))
-    for _ in range(args.warmup):
-        oracle_command_cost(w, budget)
-    secs = []
+    for i in range(args.warmup):
+        oracle_command_fraction(w, i)
+    fr, secs = [], []
     info = ""
-    comp = {}
-    for _ in range(args.steps):
-        s, info, comp = oracle_command_cost(w, budget)
-        secs.append(s)
-    value = args.steps / sum(secs)
+    for i in range(args.steps):
+        f, t, info = oracle_command_fraction(w, args.warmup + i)
+        fr.append(f)
+        secs.append(t)
+    value = sum(fr) / sum(secs)
     line = {"metric": METRIC, "value": value, "unit": "cmds/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * sum(secs) / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": w.name, "M": w.M, "N": w.N, "K": w.K, "seed": w.seed, "timed_iters": w.iters,
-                       "parallelism": "host"},
+            "config": workload_config(w, world),
             "impl": "reference",
             "cpu_baseline": {"value": value, "unit": "cmds/s", "cores": cpu_cores(), "kind": "oracle",
-                             "sample": info, "components": comp, "cpu_model": cpu_model()},
+                             "sample": f"each step: {info}; value = fractions of a command executed / measured "
+                                       f"seconds",
+                             "measured_wall_s": sum(secs), "fraction_per_step": fr[0],
+                             "threads": "fp64 GEMM through numpy's BLAS on all host cores; generation and check "
+                                        "single-threaded",
+                             "cpu_model": cpu_model()},
             "e2e": {"value": value, "unit": "cmds/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
 

@@ -189,9 +189,16 @@ def kendall_tau_b(x, y) -> float:
 # --------------------------------------------------------------- samples ----
 
 def sample_indices(seed: int, tensor_id: int, n_samples: int, M: int, N: int = 1):
-    """Seeded output sample: z_s = draw(key(seed, tensor_id), s);
+    """Seeded output sample (reading R12 of the workloads: which elements of a
+    large output the oracle recomputes): the draws of the stream keyed by
+    key(seed, tensor_id), each mapped to a position by sample_indices_from_key."""
+    return sample_indices_from_key(gen.stream_key(seed, tensor_id), n_samples, M, N)
+
+
+def sample_indices_from_key(key: int, n_samples: int, M: int, N: int = 1):
+    """Sample s of an M x N output: z_s = draw(key, s);
     i = z_s mod M, j = (z_s >> 32) mod N (duplicates allowed)."""
-    z = gen.draws(gen.stream_key(seed, tensor_id), 0, n_samples)
+    z = gen.draws(key, 0, n_samples)
     i = (z % np.uint64(M)).astype(np.int64)
     j = ((z >> np.uint64(32)) % np.uint64(N)).astype(np.int64)
     return i, j

@@ -79,6 +79,7 @@ SIGNATURES = {
     "krex_flush_l2": (_i32, [_vp, _sz, _vp]),
     "krex_l2_bytes": (_i32, [_P(_sz)]),
     "krex_check_scratch_bytes": (_sz, []),
+    "krex_check_scratch_init": (_i32, [_vp, _sz, _vp]),
     "krex_check": (_i32, [krex_buf, krex_buf, _f32, _f32, _vp, _sz, _P(krex_check_result), _vp]),
     "krex_check_launch": (_i32, [krex_buf, krex_buf, _f32, _f32, _vp, _sz, _vp]),
     "krex_check_fetch": (_i32, [_vp, _P(krex_check_result), _vp]),
@@ -250,6 +251,19 @@ def krex_l2_bytes() -> int:
 
 def krex_check_scratch_bytes() -> int:
     return int(lib().krex_check_scratch_bytes())
+
+
+def krex_check_scratch_init(scratch, stream=None):
+    """Zero a check scratch's header once before its first check."""
+    ptr = scratch if isinstance(scratch, int) else scratch.data_ptr()
+    nbytes = krex_check_scratch_bytes() if isinstance(scratch, int) else scratch.numel() * scratch.element_size()
+    _ok(lib().krex_check_scratch_init(ptr, nbytes, _stream(stream)), "krex_check_scratch_init")
+
+
+def check_scratch(device="cuda"):
+    """A check scratch buffer ready for use (zero-filled, torch-allocated)."""
+    import torch
+    return torch.zeros(krex_check_scratch_bytes(), dtype=torch.uint8, device=device)
 
 
 def krex_check(out, ref, atol: float, rtol: float, scratch, stream=None):

@@ -110,7 +110,7 @@ class Workspace:
             self.out = torch.empty(w.M, w.N, dtype=f32, device=device)
         self.ref = torch.empty(w.M, w.N, dtype=f32, device=device)
         self.flush = torch.empty(max(w.flush_bytes, 16), dtype=torch.uint8, device=device)
-        self.check_scratch = torch.empty(krex_check_scratch_bytes(), dtype=torch.uint8, device=device)
+        self.check_scratch = torch.zeros(krex_check_scratch_bytes(), dtype=torch.uint8, device=device)
         # the GEMM's split-K meeting place: zero-filled once, left ready by every call
         self.gemm_ws = (torch.zeros(krex_gemm_workspace_bytes(), dtype=torch.uint8, device=device)
                         if w.is_gemm else None)

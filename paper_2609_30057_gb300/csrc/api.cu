@@ -42,6 +42,8 @@ static krex_status ok() {
     return KREX_OK;
 }
 
+krex_status ok_status() { return ok(); }
+
 // ------------------------------------------------------- device properties --
 
 namespace {
@@ -103,7 +105,7 @@ static int32_t op_dtype(int32_t op) {
     return op == KREX_OP_GEMM_BF16 ? KREX_BF16 : (op == KREX_OP_GEMM_F16 ? KREX_F16 : KREX_F32);
 }
 
-static krex_status check_buf(const krex_buf &b, const char *name) {
+krex_status check_buf(const krex_buf &b, const char *name) {
     if (elem_size(b.dtype) == 0) return set_error(KREX_ERR_INVALID, "%s: bad dtype %d", name, b.dtype);
     if (b.rows < 0 || b.cols < 0) return set_error(KREX_ERR_INVALID, "%s: negative shape", name);
     if (b.rows > 0 && b.ld < b.cols) return set_error(KREX_ERR_INVALID, "%s: ld %lld < cols %lld", name,
@@ -412,11 +414,18 @@ krex_status krex_check_launch(krex_buf out, krex_buf ref, float atol, float rtol
 
 krex_status krex_check_fetch(const void *dev_scratch, krex_check_result *host_result, krex_stream_t stream) {
     if (!dev_scratch || !host_result) return set_error(KREX_ERR_INVALID, "check_fetch: null argument");
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     krex_check_result r;
-    KREX_CUDA_TRY(cudaMemcpyAsync(&r, dev_scratch, sizeof(r), cudaMemcpyDeviceToHost, s));
-    KREX_CUDA_TRY(cudaStreamSynchronize(s));
+    krex_status st = read_check_header(dev_scratch, &r, reinterpret_cast<cudaStream_t>(stream));
+    if (st) return st;
     *host_result = r;
+    return ok();
+}
+
+krex_status krex_check_scratch_init(void *dev_scratch, size_t scratch_bytes, krex_stream_t stream) {
+    if (!dev_scratch || scratch_bytes < check_scratch_bytes())
+        return set_error(KREX_ERR_INVALID, "check scratch needs %zu bytes", check_scratch_bytes());
+    if (!aligned16(dev_scratch)) return set_error(KREX_ERR_UNSUPPORTED, "check scratch must be 16-byte aligned");
+    KREX_CUDA_TRY(init_check_scratch(dev_scratch, reinterpret_cast<cudaStream_t>(stream)));
     return ok();
 }
 

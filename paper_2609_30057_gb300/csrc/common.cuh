@@ -2,6 +2,7 @@
 // Not part of the public ABI (see include/krex.h).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -24,8 +25,14 @@ cudaError_t launch_fill_normal_f32(uint64_t key, float sigma, float *out, int64_
                                    int64_t cols, int64_t ld, cudaStream_t s);
 // K3: grid-stride writer of `bytes` bytes of `value`.
 cudaError_t launch_flush(void *p, size_t bytes, uint32_t value, cudaStream_t s);
-// K6: compare-and-reduce; result (16 bytes) lands in scratch.
+// K6: compare-and-reduce; result (16 bytes) lands in scratch, whose 32-byte
+// header must be zero before its first use and is left ready by every call.
 size_t check_scratch_bytes();
+size_t check_header_bytes();
+cudaError_t init_check_scratch(void *scratch, cudaStream_t s);
+// Copy the result of the last check on `scratch` to *r (synchronises s);
+// KREX_ERR_STATE if the header shows the scratch was not ready on entry.
+krex_status read_check_header(const void *scratch, krex_check_result *r, cudaStream_t s);
 cudaError_t launch_check(const void *out, int out_dtype, int64_t ldo, const void *ref,
                          int ref_dtype, int64_t ldr, int64_t rows, int64_t cols, float atol,
                          float rtol, void *scratch, cudaStream_t s);
@@ -56,6 +63,11 @@ void note_launches(int n);
 // ---- errors -----------------------------------------------------------------
 krex_status set_error(krex_status st, const char *fmt, ...);
 krex_status cuda_error(cudaError_t e, const char *what);
+// KREX_OK, clearing the calling thread's last error string.
+krex_status ok_status();
+// Validation of a caller's buffer descriptor (dtype, shape, stride, pointer);
+// sets the error string and returns KREX_ERR_INVALID on a bad one.
+krex_status check_buf(const krex_buf &b, const char *name);
 
 }  // namespace krex
 

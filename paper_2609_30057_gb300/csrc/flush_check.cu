@@ -11,14 +11,24 @@
 // non-negative floats; a NaN dominates and is reported as the canonical quiet
 // NaN 0x7FC00000).  Warp reduction with __reduce_max_sync/__reduce_add_sync,
 // one partial per block in scratch, one atomic ticket per block; the last
-// block to take a ticket combines the partials and re-arms the ticket.  Max
-// and count are exact, so the result does not depend on the launch shape.
+// block to take a ticket combines the partials, writes the result, re-arms
+// the ticket and marks the call done.  Max and count are exact, so the result
+// does not depend on the launch shape.
+//
+// The scratch header is zeroed once (by the caller or krex_check_scratch_init)
+// and every call leaves it ready for the next, so a check is one launch with
+// no reset in front of it.  Block 0 clears the done word at its start; a
+// scratch whose ticket was not zero on entry ends with done = 0 (no block saw
+// itself last) or a non-zero ticket (a block saw itself last too early), and
+// the host's fetch reports that instead of a result.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
 #include <type_traits>
 
 #include <mutex>
+
+#include <string.h>
 
 #include "common.cuh"
 
@@ -59,13 +69,16 @@ struct Partial {
     unsigned long long count;
 };
 
-// Scratch layout (device, caller-owned).
+// Scratch layout (device, caller-owned).  Header: 32 bytes.
 struct CheckScratch {
     Partial result;          // final {max_bits, count}
-    unsigned int ticket;     // blocks that have published a partial
-    unsigned int pad[3];
+    unsigned int ticket;     // blocks that have published a partial; 0 between calls
+    unsigned int done;       // 1 once the last block has written result
+    unsigned int pad[2];
     Partial partial[kCheckMaxBlocks];
 };
+constexpr size_t kCheckHeaderBytes = offsetof(CheckScratch, partial);
+static_assert(kCheckHeaderBytes == 32, "check scratch header is 32 bytes");
 
 __device__ __forceinline__ float widen(const __nv_bfloat16 *p, int64_t i) {
     return __uint_as_float((uint32_t)(*reinterpret_cast<const uint16_t *>(p + i)) << 16);
@@ -160,6 +173,17 @@ __device__ __forceinline__ void block_reduce_publish(Acc acc, CheckScratch *sc) 
         sc->result.pad = 0;
         sc->result.count = fc;
         sc->ticket = 0;  // re-arm for the next call
+        __threadfence();
+        sc->done = 1u;
+    }
+}
+
+// Block 0 clears the done word before any block can take the last ticket
+// (its own ticket comes after this store and a fence).
+__device__ __forceinline__ void clear_done(CheckScratch *sc) {
+    if (blockIdx.x == 0 && threadIdx.x == 0) {
+        sc->done = 0u;
+        __threadfence();
     }
 }
 
@@ -171,6 +195,7 @@ check_16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref, 
                  const T *out_s, const float *ref_s, int64_t n, float atol,
                  float rtol, CheckScratch *sc) {
     Acc acc;
+    clear_done(sc);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < n8; g += stride) {
         uint4 o = __ldcs(out + g);
@@ -199,6 +224,7 @@ check_f32_f32_vec(const float4 *__restrict__ out, const float4 *__restrict__ ref
                   const float *out_s, const float *ref_s, int64_t n, float atol, float rtol,
                   CheckScratch *sc) {
     Acc acc;
+    clear_done(sc);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     for (; g + stride < n4; g += 2 * stride) {
@@ -232,6 +258,7 @@ __global__ void __launch_bounds__(kCheckThreads, kGenericBlocksPerSM)
 check_generic(const TO *out, int64_t ldo, const TR *ref, int64_t ldr, int64_t rows,
               int64_t cols, float atol, float rtol, CheckScratch *sc) {
     Acc acc;
+    clear_done(sc);
     const int64_t n = rows * cols;
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += stride) {
@@ -285,6 +312,29 @@ int check_blocks(int64_t items, int blocks_per_sm) {
 
 size_t check_scratch_bytes() { return sizeof(CheckScratch); }
 
+size_t check_header_bytes() { return kCheckHeaderBytes; }
+
+cudaError_t init_check_scratch(void *scratch, cudaStream_t s) {
+    return cudaMemsetAsync(scratch, 0, kCheckHeaderBytes, s);
+}
+
+krex_status read_check_header(const void *scratch, krex_check_result *r, cudaStream_t s) {
+    CheckScratch h;
+    cudaError_t e = cudaMemcpyAsync(&h, scratch, kCheckHeaderBytes, cudaMemcpyDeviceToHost, s);
+    if (e != cudaSuccess) return cuda_error(e, "cudaMemcpyAsync (check result)");
+    e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_error(e, "cudaStreamSynchronize (check result)");
+    if (h.done != 1u || h.ticket != 0u)
+        return set_error(KREX_ERR_STATE,
+                         "check scratch was not ready (done %u, ticket %u): zero its first %zu bytes once before "
+                         "its first check (krex_check_scratch_init)",
+                         h.done, h.ticket, kCheckHeaderBytes);
+    memcpy(&r->max_abs_err, &h.result.max_bits, sizeof(float));
+    r->reserved = 0;
+    r->n_violations = h.result.count;
+    return KREX_OK;
+}
+
 cudaError_t launch_flush(void *p, size_t bytes, uint32_t value, cudaStream_t s) {
     if (bytes == 0) return cudaSuccess;
     size_t n16 = bytes / 16, ntail = bytes % 16;
@@ -301,9 +351,6 @@ cudaError_t launch_check(const void *out, int out_dtype, int64_t ldo, const void
                          int ref_dtype, int64_t ldr, int64_t rows, int64_t cols, float atol,
                          float rtol, void *scratch, cudaStream_t s) {
     CheckScratch *sc = static_cast<CheckScratch *>(scratch);
-    // zero the result and the ticket: the scratch contents on entry do not matter
-    cudaError_t e = cudaMemsetAsync(sc, 0, offsetof(CheckScratch, partial), s);
-    if (e != cudaSuccess) return e;
     const int64_t n = rows * cols;
     const bool contiguous = (ldo == cols && ldr == cols) || rows <= 1;
     const bool a16 = ((reinterpret_cast<uintptr_t>(out) | reinterpret_cast<uintptr_t>(ref)) & 15u) == 0;
@@ -342,59 +389,106 @@ cudaError_t launch_check(const void *out, int out_dtype, int64_t ldo, const void
 // measurement around them.  The scratch is a fixed static device array that
 // each GPU loading this library keeps until the process exits.
 
-// Capacity: the check's 16-byte result/ticket header plus one 16-byte partial
-// for each of its at most 2048 blocks (32,800 bytes), rounded up.
+// Capacity: the check's 32-byte header (result, ticket, done word, padding)
+// plus one 16-byte partial for each of its at most 2048 blocks (32,800 bytes),
+// rounded up to a multiple of 256.
 #define KREX_CHECK_NOALLOC_SCRATCH_BYTES 33024
 static __device__ __align__(256) unsigned char g_check_noalloc_scratch[KREX_CHECK_NOALLOC_SCRATCH_BYTES];
+static_assert(sizeof(krex::CheckScratch) <= KREX_CHECK_NOALLOC_SCRATCH_BYTES,
+              "the static check scratch must hold the check's scratch layout");
 
 namespace krex {
 namespace {
+
+typedef CUresult (*PfnCtxGetCurrent)(CUcontext *);
+typedef CUresult (*PfnCtxGetId)(CUcontext, unsigned long long *);
+
+// The driver's cuCtxGetCurrent / cuCtxGetId through the runtime's entry-point
+// query (the library links no driver library).
+void driver_ctx_fns(PfnCtxGetCurrent *get_current, PfnCtxGetId *get_id) {
+    static PfnCtxGetCurrent gc = nullptr;
+    static PfnCtxGetId gi = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            gc = reinterpret_cast<PfnCtxGetCurrent>(p);
+        p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            gi = reinterpret_cast<PfnCtxGetId>(p);
+    });
+    *get_current = gc;
+    *get_id = gi;
+}
+
+// Where the static array lives, per device ordinal, and in which context:
+// a context that is destroyed and created again (a device reset, a new
+// primary context) reloads the module and may move the array, so the address
+// is resolved again whenever the current context's id differs.
+struct NoallocSlot {
+    unsigned long long ctx_id = 0;
+    void *addr = nullptr;
+};
 std::mutex g_noalloc_mu;
-void *g_noalloc_addr[64];  // device address of the array, per device ordinal
+NoallocSlot g_noalloc[64];
+
 }  // namespace
 }  // namespace krex
 
 extern "C" krex_status krex_check_noalloc(krex_buf out, krex_buf ref, float atol, float rtol,
                                           krex_check_result *host_result, krex_stream_t stream) {
     using namespace krex;
-    auto bad_buf = [](const krex_buf &b) {
-        return (b.dtype != KREX_BF16 && b.dtype != KREX_F32 && b.dtype != KREX_F16) || b.rows < 0 || b.cols < 0 ||
-               (b.rows > 0 && b.ld < b.cols) || (b.rows * b.cols > 0 && b.ptr == nullptr);
-    };
-    if (bad_buf(out) || bad_buf(ref)) return set_error(KREX_ERR_INVALID, "check_noalloc: bad out or ref buffer");
+    krex_status st;
+    if ((st = check_buf(out, "check_noalloc: out")) || (st = check_buf(ref, "check_noalloc: ref"))) return st;
     if (out.rows != ref.rows || out.cols != ref.cols)
         return set_error(KREX_ERR_INVALID, "check_noalloc: out and ref shapes differ");
     if (!host_result) return set_error(KREX_ERR_INVALID, "check_noalloc: host_result is null");
-    const size_t need = check_scratch_bytes();
-    if (need > (size_t)KREX_CHECK_NOALLOC_SCRATCH_BYTES)
-        return set_error(KREX_ERR_UNSUPPORTED, "check_noalloc: needs %zu bytes of scratch, the static array holds %d",
-                         need, KREX_CHECK_NOALLOC_SCRATCH_BYTES);
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return cuda_error(e, "cudaGetDevice");
     if (dev < 0 || dev >= 64) return set_error(KREX_ERR_UNSUPPORTED, "check_noalloc: device ordinal %d >= 64", dev);
+    PfnCtxGetCurrent get_current = nullptr;
+    PfnCtxGetId get_id = nullptr;
+    driver_ctx_fns(&get_current, &get_id);
+    if (!get_current || !get_id)
+        return set_error(KREX_ERR_CUDA, "check_noalloc: the driver offers no cuCtxGetCurrent / cuCtxGetId");
+    CUcontext ctx = nullptr;
+    if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) {
+        // no context bound to this thread yet: bind the device's primary one
+        e = cudaSetDevice(dev);
+        if (e != cudaSuccess) return cuda_error(e, "cudaSetDevice (check_noalloc)");
+        if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr)
+            return set_error(KREX_ERR_CUDA, "check_noalloc: no current context on device %d", dev);
+    }
+    unsigned long long ctx_id = 0;
+    if (get_id(ctx, &ctx_id) != CUDA_SUCCESS)
+        return set_error(KREX_ERR_CUDA, "check_noalloc: cuCtxGetId failed");
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     void *scratch = nullptr;
     {
-        // first call on a device: resolve the array's device address there
+        // set-up, once per device and context: resolve the array's device
+        // address in that context and zero the check's header there
         std::lock_guard<std::mutex> lk(g_noalloc_mu);
-        if (!g_noalloc_addr[dev]) {
+        NoallocSlot &slot = g_noalloc[dev];
+        if (slot.addr == nullptr || slot.ctx_id != ctx_id) {
             void *p = nullptr;
             e = cudaGetSymbolAddress(&p, g_check_noalloc_scratch);
             if (e != cudaSuccess) return cuda_error(e, "cudaGetSymbolAddress (check_noalloc scratch)");
-            g_noalloc_addr[dev] = p;
+            e = init_check_scratch(p, s);
+            if (e != cudaSuccess) return cuda_error(e, "cudaMemsetAsync (check_noalloc scratch header)");
+            slot.addr = p;
+            slot.ctx_id = ctx_id;
         }
-        scratch = g_noalloc_addr[dev];
+        scratch = slot.addr;
     }
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    // launch_check clears the result and ticket in the array before the kernel
     e = launch_check(out.ptr, out.dtype, out.ld, ref.ptr, ref.dtype, ref.ld, out.rows, out.cols, atol, rtol, scratch, s);
     if (e != cudaSuccess) return cuda_error(e, "check_noalloc launch");
     note_launches(1);
     krex_check_result r;
-    e = cudaMemcpyAsync(&r, scratch, sizeof(r), cudaMemcpyDeviceToHost, s);
-    if (e != cudaSuccess) return cuda_error(e, "cudaMemcpyAsync (check_noalloc result)");
-    e = cudaStreamSynchronize(s);
-    if (e != cudaSuccess) return cuda_error(e, "cudaStreamSynchronize (check_noalloc)");
+    if ((st = read_check_header(scratch, &r, s))) return st;
     *host_result = r;
-    return KREX_OK;
+    return ok_status();
 }

@@ -28,19 +28,36 @@ def test_reference_arm_line():
     assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == d["value"] and cb["cores"] >= 1 and cb["sample"]
-    assert cb["components"]["gemm_fp64_GFLOP_per_s"] > 0
+    # measured, not extrapolated: the small command is one whole command per step
+    assert cb["fraction_per_step"] == 1.0
+    assert abs(d["value"] - 1e3 / d["ms_per_step"]) < 1e-9 * d["value"]
+    assert abs(cb["measured_wall_s"] - d["ms_per_step"] / 1e3) < 1e-9
     assert d["config"]["workload"] == "gemm_bf16_256"
+
+
+def test_reference_arm_config_keys_match_our_arm():
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2609_30057_gb300.command import WORKLOADS
+    d = _bench("--impl", "reference", "--steps", "2", "--warmup", "1", "--workload", "gemm_bf16_4096")
+    assert d["config"] == bench.workload_config(WORKLOADS["gemm_bf16_4096"], 1)
+    f = d["cpu_baseline"]["fraction_per_step"]
+    assert f == (256 * 256) / (4096 * 4096)
+    # value = fractions executed / measured time, and the steps' time is real
+    assert abs(d["value"] - 2 * f / (d["ms_per_step"] * 2 / 1e3)) < 1e-9 * d["value"]
 
 
 @pytest.mark.gpu
 def test_our_arm_line():
-    d = _bench("--steps", "3", "--warmup", "3", "--no-kernels")
+    d = _bench("--steps", "3", "--warmup", "3", "--no-kernels", "--no-configs", "--workload", "gemm_bf16_4096")
     assert BASE_KEYS <= set(d) and {"roofline", "gpu_launches", "clocks", "timing_spread"} <= set(d)
     assert d["n_gpus"] == 1 and d["steps"] == 3 and d["warmup"] == 3 and d["value"] > 0
     assert abs(d["value"] - 3 / (d["ms_per_step"] * 3 / 1e3)) < 1e-6 * d["value"]
     r = d["roofline"]
     assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s" and 0 < r["frac"] < 1.2
     assert abs(r["frac"] - r["achieved"] / r["peak"]) < 1e-9
+    rr = d["roofline_reference"]
+    assert rr["bound"] == "alu" and rr["kernel"] == "gemm_ref_simt" and 0 < rr["frac"] < 1.05
     e = d["e2e"]
     assert e["value"] > 0 and e["h2d_bytes_per_step"] == 2 * 4096 * 4096 * 2
     assert e["d2h_bytes_per_step"] >= 4096 * 4096 * 2

@@ -18,7 +18,7 @@ pytestmark = pytest.mark.gpu
 @pytest.fixture(scope="module")
 def scratch():
     krex.build()
-    return torch.empty(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
+    return torch.zeros(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
 
 
 class F16Bits(np.ndarray):
@@ -133,3 +133,28 @@ def test_check_f16_pairs_match_oracle(n, pair, scratch):
     for atol, rtol in ((1e-2, 1e-2), (2.0 ** -12 * 64, 2.0 ** -10), (0.0, 0.0)):
         _run(o, r, atol, rtol, scratch)
 
+
+
+@pytest.mark.parametrize("fill", [0xFF, 0x01])
+def test_scratch_that_was_never_zeroed_is_reported_then_initialised(fill):
+    # A scratch whose header was not zeroed (ticket 0xFFFFFFFF: no block sees
+    # itself last; ticket 0x01010101: a block would see itself last too early
+    # or never) gives STATE, never a result; after krex_check_scratch_init the
+    # same buffer gives the oracle's result, and keeps doing so call after call.
+    o = inputs.normal_f32(51, (300, 517))
+    r = inputs.perturbed(o, 52, 0.2, 1e-3)
+    bad = torch.full((krex.krex_check_scratch_bytes(),), fill, dtype=torch.uint8, device="cuda")
+    with pytest.raises(RuntimeError, match="not ready"):
+        krex.krex_check(_dev(o), _dev(r), 1e-4, 0.0, bad)
+    krex.krex_check_scratch_init(bad)
+    for _ in range(3):
+        _run(o, r, 1e-4, 0.0, bad)
+
+
+def test_scratch_init_rejects_small_or_unaligned_buffers():
+    lib = krex.lib()
+    buf = torch.zeros(krex.krex_check_scratch_bytes() + 16, dtype=torch.uint8, device="cuda")
+    assert lib.krex_check_scratch_init(buf.data_ptr(), 16, None) == krex.KREX_ERR_INVALID
+    assert lib.krex_check_scratch_init(buf.data_ptr() + 8, krex.krex_check_scratch_bytes(),
+                                       None) == krex.KREX_ERR_UNSUPPORTED
+    assert lib.krex_check_scratch_init(None, krex.krex_check_scratch_bytes(), None) == krex.KREX_ERR_INVALID

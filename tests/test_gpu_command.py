@@ -34,9 +34,13 @@ def test_gemm_256_command_matches_oracle():
     want = ref.gemm_f64(gen.uniform_bf16(w.seed, 0, w.M, w.K), gen.uniform_bf16(w.seed, 1, w.K, w.N))
     got = gen.bf16_to_f32(bits16(ws.out)).astype(np.float64)
     assert np.all(np.abs(got - want) <= ref.gemm_tolerance(want, w.K))
-    # the check's result equals the oracle's check of the same two device outputs
-    # recomputed from oracle inputs: C within tolerance of fp64 means ref fp32 too
+    # the device reference is within the fp32 summation bound of fp64
     assert np.max(np.abs(ws.ref.cpu().numpy() - want)) < 1e-4
+    # the command's verdict is the oracle's check of the two downloaded
+    # outputs, bit for bit (count and max error)
+    mx, nv = ref.check_f32(got.astype(np.float32), ws.ref.cpu().numpy(), w.atol, w.rtol)
+    assert int(res.check.n_violations) == nv == 0
+    assert ref.check_bits(res.check.max_abs_err) == ref.check_bits(mx)
 
 
 def test_command_with_host_buffers_equals_device_generated():
@@ -102,3 +106,52 @@ def test_phase_times_are_positive_and_within_the_command():
     ph = list(r.phase_ms)
     assert all(p > 0 for p in ph), ph
     assert sum(ph) <= wall_ms * 1.02 + 0.02, (ph, wall_ms)
+
+
+def test_failing_command_verdict_equals_the_oracle_check():
+    # a tolerance that part of the output fails: the device verdict (count and
+    # max error) equals the oracle's check of the downloaded buffers exactly
+    w = scaled(WORKLOADS["gemm_bf16_256"], M=384, N=640, K=512, iters=3)
+    ws = Workspace(w)
+    ws.cmd.atol = 2.0 ** -9
+    ws.cmd.rtol = 2.0 ** -9
+    res = ws.run()
+    out = gen.bf16_to_f32(bits16(ws.out))
+    r32 = ws.ref.cpu().numpy()
+    mx, nv = ref.check_f32(out, r32, 2.0 ** -9, 2.0 ** -9)
+    assert 0 < nv < w.M * w.N
+    assert int(res.check.n_violations) == nv and res.passed == 0 and res.n_iters == 0
+    assert ref.check_bits(res.check.max_abs_err) == ref.check_bits(mx)
+
+
+def test_gemm_16384_command_against_the_oracle():
+    # the 16384^3 command (its own seed, flush and tolerance; two timed
+    # iterations instead of twenty to keep the test short): inputs on oracle
+    # samples, the candidate and the reference on 4096 oracle-sampled outputs,
+    # and the verdict equal to the oracle's check of the downloaded buffers
+    w = scaled(WORKLOADS["gemm_bf16_16384"], iters=2)
+    ws = Workspace(w)
+    res = ws.run()
+    assert res.passed == 1 and res.n_iters == 2 and krex.krex_device_status() == 0
+    n = w.M
+    i, j = ref.sample_indices(w.seed, 2, 4096, n, n)
+    want = ref.gemm_sampled_f64(w.seed, n, n, n, i, j)
+    ti, tj = torch.from_numpy(i).cuda(), torch.from_numpy(j).cuda()
+    got = gen.bf16_to_f32(bits16(ws.out[ti, tj])).astype(np.float64)
+    assert np.all(np.abs(got - want) <= ref.gemm_tolerance(want, n))
+    # the device reference: within the fp32 recursive-summation bound
+    # K 2^-24 sum_k |a_ik b_kj| of fp64 (first 512 samples)
+    r = ws.ref[ti, tj].cpu().numpy().astype(np.float64)
+    kk = np.arange(n, dtype=np.int64)
+    for s_ in range(512):
+        ra = np.abs(gen.widen("bf16", gen.uniform_at("bf16", w.seed, 0, i[s_] * n + kk)).astype(np.float64))
+        cb = np.abs(gen.widen("bf16", gen.uniform_at("bf16", w.seed, 1, kk * n + j[s_])).astype(np.float64))
+        assert abs(r[s_] - want[s_]) <= n * 2.0 ** -24 * float(ra @ cb), s_
+    # inputs: sampled elements of A and B are the oracle's draws, bit for bit
+    k = torch.from_numpy((i * 7 + 3) % n).cuda()
+    assert np.array_equal(bits16(ws.inputs[0][ti, k]), gen.uniform_at("bf16", w.seed, 0, i * n + (i * 7 + 3) % n))
+    assert np.array_equal(bits16(ws.inputs[1][k, tj]), gen.uniform_at("bf16", w.seed, 1, ((i * 7 + 3) % n) * n + j))
+    # the verdict over all 2^28 outputs: the oracle's check of the downloaded buffers
+    mx, nv = ref.check_f32(gen.bf16_to_f32(bits16(ws.out)), ws.ref.cpu().numpy(), w.atol, w.rtol)
+    assert nv == 0 == int(res.check.n_violations)
+    assert ref.check_bits(res.check.max_abs_err) == ref.check_bits(mx)

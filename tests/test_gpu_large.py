@@ -57,7 +57,7 @@ def test_normal_fill_beyond_2_32_elements():
 
 
 def test_check_counts_exactly_beyond_2_32_elements():
-    scratch = torch.empty(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
+    scratch = torch.zeros(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
     r = torch.zeros(ROWS, COLS, dtype=torch.float32, device="cuda")
     o = torch.zeros(ROWS, COLS, dtype=torch.bfloat16, device="cuda")
     planted = torch.tensor([5, BEYOND - 1, BEYOND, BEYOND + 12345, N - 1], device="cuda")

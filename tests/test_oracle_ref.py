@@ -102,6 +102,61 @@ def test_sample_indices_in_range_and_seeded():
     assert len(set(zip(i.tolist(), j.tolist()))) > 4000
 
 
+def test_sample_indices_hand_worked_from_published_draws():
+    # (key, s, z_s, M, N, i, j) read off the published SplitMix64 outputs by hand
+    rows = [ln.split() for ln in read_golden("sample_indices.txt")]
+    for key, s, z_hex, M, N, i_want, j_want in rows:
+        key, s, M, N = int(key), int(s), int(M), int(N)
+        z = gen.draws(key, s, 1)
+        assert int(z[0]) == int(z_hex, 16)
+        i, j = ref.sample_indices_from_key(key, s + 1, M, N)
+        assert (int(i[s]), int(j[s])) == (int(i_want), int(j_want)), (key, s, M, N)
+
+
+def test_sample_indices_use_the_stream_of_seed_and_tensor():
+    # the seeded form is the key form on key(seed, tensor): the published
+    # vector's entry t is stream_key(1234567, t), whose stream starts with
+    # draw(stream_key(1234567, t), 0)
+    for seed, tid in ((4, 2), (5, 2), (3, 3)):
+        key = int(gen.stream_key(seed, tid))
+        a = ref.sample_indices(seed, tid, 64, 16384, 16384)
+        b = ref.sample_indices_from_key(key, 64, 16384, 16384)
+        assert all(np.array_equal(x, y) for x, y in zip(a, b))
+        z = gen.draws(key, 0, 1)
+        assert int(a[0][0]) == int(z[0]) % 16384 and int(a[1][0]) == (int(z[0]) >> 32) % 16384
+
+
+def test_gemm_tolerance_hand_worked_fixture():
+    # bound = rtol |c| + 2^-12 sqrt(K), worked by hand for the workloads' K
+    for dtype, K, c, atol, rtol, bound in (ln.split() for ln in read_golden("gemm_tolerance.txt")):
+        K, c, bound = int(K), float(c), float(bound)
+        got = ref.gemm_tolerance(np.array([c]), K, dtype=dtype)
+        assert got.shape == (1,) and float(got[0]) == bound, (dtype, K, c)
+        assert ref.GEMM_RTOL[dtype] == float(rtol)
+        assert float(ref.gemm_tolerance(np.array([0.0]), K, dtype=dtype)[0]) == float(atol)
+
+
+def test_workload_tolerances_are_the_oracle_bound():
+    # the product's per-workload atol / rtol (passed to the device check) are
+    # the same bound the oracle accepts with: exactly for the K of the fixture,
+    # and atol^2 = 2^-24 K for every other K
+    from paper_2609_30057_gb300.command import WORKLOADS
+    fixture = {(d, int(K)): (float(a), float(r)) for d, K, _, a, r, _ in
+               (ln.split() for ln in read_golden("gemm_tolerance.txt"))}
+    seen = 0
+    for w in WORKLOADS.values():
+        if not w.is_gemm:
+            assert (w.atol, w.rtol) == (ref.SOFTMAX_ATOL, 0.0)
+            continue
+        assert w.rtol == ref.GEMM_RTOL[w.dtype]
+        if (w.dtype, w.K) in fixture:
+            assert (w.atol, w.rtol) == fixture[(w.dtype, w.K)]
+            seen += 1
+        assert math.isclose((w.atol * 2 ** 12) ** 2, w.K, rel_tol=1e-15)
+        assert w.atol == float(ref.gemm_tolerance(np.array([0.0]), w.K, dtype=w.dtype)[0])
+    assert seen >= 4
+
+
 # --------------------------------------------------------------- softmax ----
 
 def test_softmax_hand_worked_fixture():

@@ -47,15 +47,35 @@ def _call_noalloc(lib, out, ref_t, atol, rtol):
 def test_noalloc_check_matches_scratch_check_on_two_calls_in_a_row():
     krex.build()
     lib = krex.lib()
-    scratch = torch.empty(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
+    scratch = torch.zeros(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
     for name, out, ref_t, atol, rtol in _cases():
         want = krex.krex_check(out, ref_t, atol, rtol, scratch)
         first = _call_noalloc(lib, out, ref_t, atol, rtol)
         second = _call_noalloc(lib, out, ref_t, atol, rtol)
+        # and the oracle's check of the same two buffers, bit for bit
+        o32 = out.float().cpu().numpy() if out.dtype == torch.bfloat16 else out.cpu().numpy()
+        oracle = ref.check_f32(o32, ref_t.cpu().numpy(), atol, rtol)
         for got in (first, second):
-            assert got[1] == want[1], name
-            assert ref.check_bits(got[0]) == ref.check_bits(want[0]), name
+            assert got[1] == want[1] == oracle[1], name
+            assert ref.check_bits(got[0]) == ref.check_bits(want[0]) == ref.check_bits(oracle[0]), name
         assert want[1] > 0, name        # every case has violations to count
+
+
+def test_noalloc_check_takes_no_device_memory():
+    # after a first call (the set-up), a call leaves the device's free memory
+    # exactly as it was: nothing is allocated, not even by the driver
+    lib = krex.lib()
+    o = torch.from_numpy(inputs.normal_f32(37, (1024, 1024))).cuda().half()
+    r = torch.from_numpy(inputs.normal_f32(38, (1024, 1024))).cuda()
+    _call_noalloc(lib, o, r, 1e-3, 1e-3)
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    got = _call_noalloc(lib, o, r, 1e-3, 1e-3)
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert free1 == free0
+    want = ref.check_f32(o.float().cpu().numpy(), r.cpu().numpy(), 1e-3, 1e-3)
+    assert got[1] == want[1] and ref.check_bits(got[0]) == ref.check_bits(want[0])
 
 
 def test_noalloc_check_rejects_bad_arguments():
@@ -65,3 +85,9 @@ def test_noalloc_check_rejects_bad_arguments():
     b = krex.krex_buf(16, krex.KREX_F32, 0, 4, 5, 5)
     assert lib.krex_check_noalloc(a, b, 0.0, 0.0, ctypes.byref(res), None) == krex.KREX_ERR_INVALID
     assert lib.krex_check_noalloc(a, a, 0.0, 0.0, None, None) == krex.KREX_ERR_INVALID
+    # a row stride past 2^40 elements is rejected, as krex_check rejects it
+    huge = krex.krex_buf(16, krex.KREX_F32, 0, 4, 4, (1 << 40) + 8)
+    assert lib.krex_check_noalloc(huge, huge, 0.0, 0.0, ctypes.byref(res), None) == krex.KREX_ERR_INVALID
+    scratch = torch.zeros(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
+    assert lib.krex_check(huge, huge, 0.0, 0.0, scratch.data_ptr(), scratch.numel(), ctypes.byref(res),
+                          None) == krex.KREX_ERR_INVALID
