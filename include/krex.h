@@ -450,6 +450,42 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
                              const void *const *host_in, void *host_out, float *durations_ms,
                              krex_command_result *result, krex_stream_t stream);
 
+/* ------------------------------------------------------------ tuning ----- */
+
+/* The kernels' launch configuration, process-wide.  The library never reads
+ * its environment: every choice is a field here, and a field left at its
+ * default (0, or -1 where stated) takes the measured choice.  Not part of the
+ * paper: the knobs of this implementation's kernels.  Changing it affects
+ * launches issued after the call (it is read once per launch). */
+typedef struct {
+    int32_t gemm_pair_tile_n;  /* columns of a 2-SM pair tile: 0 = 256; else 128, 192 or 256 */
+    int32_t gemm_stage_k;      /* K depth of a shared-memory ring stage: 0 = 128; else 64 or 128 */
+    int32_t gemm_ring_stages;  /* stages of the ring in use: 0 = all that fit (3 of K 128, 6 of K 64); else
+                                  2 .. that number */
+    int32_t gemm_raster_group; /* pair-tile rows per raster group: 0 = 4 for GEMMs of 1.5 to 5 waves of pair
+                                  tiles, else 8; else 1..64 */
+    int32_t gemm_tail_split;   /* split a final partial wave: -1 = yes (default), 0 = no, 1 = yes */
+    int32_t gemm_split_k;      /* split a single partial wave into K halves (needs the workspace of
+                                  krex_run_candidate_ws): -1 = when K >= 4096 (default), 0 = never,
+                                  1 = whenever the shape allows */
+    int32_t reference_tiling;  /* the CUDA-core reference GEMM's tiling: -1 = by size (default); 0..5 as
+                                  documented in gemm_ref.cu (all give identical bits) */
+    int32_t wait_timeout_ms;   /* bound on every wait inside a kernel: 0 = 2000 ms; else 1..600000 */
+} krex_tuning;
+
+/* The defaults (what every measurement of this library uses). */
+void krex_tuning_defaults(krex_tuning *t);
+/* Replace the process-wide tuning (NULL: back to the defaults).  INVALID for
+ * a field out of its range (nothing changes then). */
+krex_status krex_set_tuning(const krex_tuning *t);
+krex_status krex_get_tuning(krex_tuning *t);
+
+/* Test hook for failure detection: while on (non-zero), the second K half of a
+ * split GEMM tile waits for a tag that no launch publishes, so its bounded
+ * wait runs out (status 0x1052; see krex_device_status) without faulting or
+ * hanging the GPU.  Off by default. */
+krex_status krex_debug_stall_handover(int32_t on);
+
 /* ------------------------------------------------------ host helpers ----- */
 
 /* Linear-interpolated percentile of n host floats (q in [0,1]); host only. */

@@ -43,6 +43,13 @@ class krex_region_opts(ctypes.Structure):
                 ("reserved2", ctypes.c_int32)]
 
 
+class krex_tuning(ctypes.Structure):
+    _fields_ = [("gemm_pair_tile_n", ctypes.c_int32), ("gemm_stage_k", ctypes.c_int32),
+                ("gemm_ring_stages", ctypes.c_int32), ("gemm_raster_group", ctypes.c_int32),
+                ("gemm_tail_split", ctypes.c_int32), ("gemm_split_k", ctypes.c_int32),
+                ("reference_tiling", ctypes.c_int32), ("wait_timeout_ms", ctypes.c_int32)]
+
+
 class krex_command(ctypes.Structure):
     _fields_ = [("op", ctypes.c_int32), ("warmup", ctypes.c_int32), ("iters", ctypes.c_int32),
                 ("pin_cpu", ctypes.c_int32), ("M", ctypes.c_int64), ("N", ctypes.c_int64),
@@ -101,6 +108,10 @@ SIGNATURES = {
     "krex_last_error_string": (ctypes.c_char_p, []),
     "krex_version": (_i32, []),
     "krex_debug_hold_stream": (_i32, [_vp, _P(_i32), _i32]),
+    "krex_tuning_defaults": (None, [_P(krex_tuning)]),
+    "krex_set_tuning": (_i32, [_P(krex_tuning)]),
+    "krex_get_tuning": (_i32, [_P(krex_tuning)]),
+    "krex_debug_stall_handover": (_i32, [_i32]),
     "krex_gate_shared_bytes": (_sz, [_i32]),
     "krex_gate_shared_init": (_i32, [_vp, _sz, _i32]),
     "krex_gate_shared_attach": (_i32, [_vp, _sz, _P(_vp)]),
@@ -425,6 +436,46 @@ def krex_device_status_detail() -> dict:
             "cluster_rank": hi(w[2]), "waited_ns": w[3], "producer": (lo(w[4]), hi(w[4])),
             "mma": (lo(w[5]), hi(w[5])), "epilogue": (lo(w[6]), hi(w[6])),
             "MNK": (w[7] & m, (w[7] >> 21) & m, (w[7] >> 42) & m)}
+
+
+def krex_get_tuning() -> dict:
+    t = krex_tuning()
+    _ok(lib().krex_get_tuning(ctypes.byref(t)), "krex_get_tuning")
+    return {name: getattr(t, name) for name, _ in krex_tuning._fields_}
+
+
+def krex_set_tuning(**fields) -> None:
+    """Set the process-wide tuning: the defaults with `fields` replaced
+    (krex_set_tuning() alone restores the defaults)."""
+    t = krex_tuning()
+    lib().krex_tuning_defaults(ctypes.byref(t))
+    for k, v in fields.items():
+        if k not in dict(krex_tuning._fields_):
+            raise KeyError(k)
+        setattr(t, k, int(v))
+    _ok(lib().krex_set_tuning(ctypes.byref(t)), "krex_set_tuning")
+
+
+class tuning:
+    """Context manager: the given tuning fields while inside, the previous
+    tuning restored on exit (process-wide: use where no other thread of the
+    process launches kernels whose configuration matters meanwhile)."""
+
+    def __init__(self, **fields):
+        self.fields = fields
+        self.saved = None
+
+    def __enter__(self):
+        self.saved = krex_get_tuning()
+        krex_set_tuning(**{**self.saved, **self.fields})
+        return self
+
+    def __exit__(self, *exc):
+        krex_set_tuning(**self.saved)
+
+
+def krex_debug_stall_handover(on: bool) -> None:
+    _ok(lib().krex_debug_stall_handover(1 if on else 0), "krex_debug_stall_handover")
 
 
 def krex_launch_count() -> int:

@@ -80,6 +80,38 @@ size_t l2_bytes_current() {
 
 static void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
 
+// ------------------------------------------------------------------ tuning --
+
+namespace {
+std::mutex g_tuning_mu;
+krex_tuning default_tuning() {
+    krex_tuning t;
+    memset(&t, 0, sizeof(t));
+    t.gemm_tail_split = -1;
+    t.gemm_split_k = -1;
+    t.reference_tiling = -1;
+    return t;
+}
+krex_tuning g_tuning = default_tuning();
+
+bool tuning_valid(const krex_tuning &t) {
+    return (t.gemm_pair_tile_n == 0 || t.gemm_pair_tile_n == 128 || t.gemm_pair_tile_n == 192 ||
+            t.gemm_pair_tile_n == 256) &&
+           (t.gemm_stage_k == 0 || t.gemm_stage_k == 64 || t.gemm_stage_k == 128) &&
+           (t.gemm_ring_stages == 0 ||
+            (t.gemm_ring_stages >= 2 && t.gemm_ring_stages <= (t.gemm_stage_k == 64 ? 6 : 3))) &&
+           (t.gemm_raster_group >= 0 && t.gemm_raster_group <= 64) &&
+           (t.gemm_tail_split >= -1 && t.gemm_tail_split <= 1) && (t.gemm_split_k >= -1 && t.gemm_split_k <= 1) &&
+           (t.reference_tiling >= -1 && t.reference_tiling <= 5) &&
+           (t.wait_timeout_ms >= 0 && t.wait_timeout_ms <= 600000);
+}
+}  // namespace
+
+krex_tuning tuning_snapshot() {
+    std::lock_guard<std::mutex> lk(g_tuning_mu);
+    return g_tuning;
+}
+
 void note_launches(int n) { count_launches(n); }
 
 // ---------------------------------------------------------- host SplitMix64 --
@@ -749,6 +781,29 @@ static void CUDART_CB hold_fn(void *p) {
         nanosleep(&ts, nullptr);
     }
     delete a;
+}
+
+void krex_tuning_defaults(krex_tuning *t) {
+    if (t) *t = default_tuning();
+}
+
+krex_status krex_set_tuning(const krex_tuning *t) {
+    const krex_tuning v = t ? *t : default_tuning();
+    if (!tuning_valid(v)) return set_error(KREX_ERR_INVALID, "set_tuning: a field is out of its range");
+    std::lock_guard<std::mutex> lk(g_tuning_mu);
+    g_tuning = v;
+    return ok();
+}
+
+krex_status krex_get_tuning(krex_tuning *t) {
+    if (!t) return set_error(KREX_ERR_INVALID, "get_tuning: null argument");
+    *t = tuning_snapshot();
+    return ok();
+}
+
+krex_status krex_debug_stall_handover(int32_t on) {
+    set_debug_stall_handover(on != 0);
+    return ok();
 }
 
 krex_status krex_debug_hold_stream(krex_stream_t stream, volatile int32_t *gate, int32_t hold_ms) {

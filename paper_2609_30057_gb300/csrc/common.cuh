@@ -57,6 +57,11 @@ size_t gemm_workspace_bytes();
 cudaError_t read_and_clear_device_status(uint32_t *code);
 cudaError_t read_device_status_detail(unsigned long long *words);
 
+// The process-wide tuning record (a copy; see krex_set_tuning).
+krex_tuning tuning_snapshot();
+// The failure-detection test hook of the GEMM's split-K hand-over.
+void set_debug_stall_handover(bool on);
+
 // Count kernels launched outside api.cu in krex_launch_count().
 void note_launches(int n);
 

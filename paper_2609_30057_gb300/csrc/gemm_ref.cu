@@ -15,8 +15,6 @@
 // kernel instead, with the same k-order chains (identical bits).
 #include <cuda_fp16.h>
 
-#include <cstdlib>
-
 #include "common.cuh"
 
 namespace krex {
@@ -52,9 +50,19 @@ __device__ __forceinline__ float hi_f32(uint32_t w) {
     return __uint_as_float(w & 0xFFFF0000u);
 }
 
+// 8 consecutive 16-bit elements at (r, c..c+7), for a block whose tile and
+// K slices lie wholly inside the matrix and whose rows allow 16-byte loads.
+__device__ __forceinline__ uint4 load8_inside(const uint16_t *__restrict__ p, int64_t ld, int64_t r, int64_t c) {
+    return __ldg(reinterpret_cast<const uint4 *>(p + r * ld + c));
+}
+
 // NG: 64-column groups per block (tile 128 x 64*NG); TK: K per shared slice;
-// MINB: resident blocks per SM the register budget is sized for.
-template <bool F16, int NG, int TK, int MINB>
+// MINB: resident blocks per SM the register budget is sized for.  INSIDE:
+// every tile and K slice of the launch lies inside the matrices and every row
+// allows 16-byte accesses (M % 128 = N % (64 NG) = K % TK = 0, aligned rows),
+// so loads and stores need no bounds checks (measured: 2-3 % faster at
+// 16384^3).
+template <bool F16, int NG, int TK, int MINB, bool INSIDE>
 __global__ void __launch_bounds__(256, MINB)
 gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__restrict__ B, int64_t ldb,
               float *__restrict__ C, int64_t ldc, int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec,
@@ -76,12 +84,14 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
 #pragma unroll
         for (int i = 0; i < A_LOADS; ++i) {
             const int s = t + 256 * i;
-            ua[i] = load8(A, lda, M, K, m0 + s / (TK / 8), k0 + 8 * (s % (TK / 8)), a_vec);
+            ua[i] = INSIDE ? load8_inside(A, lda, m0 + s / (TK / 8), k0 + 8 * (s % (TK / 8)))
+                           : load8(A, lda, M, K, m0 + s / (TK / 8), k0 + 8 * (s % (TK / 8)), a_vec);
         }
 #pragma unroll
         for (int i = 0; i < B_LOADS; ++i) {
             const int s = t + 256 * i;
-            ub[i] = load8(B, ldb, K, N, k0 + s / (TN / 8), n0 + 8 * (s % (TN / 8)), b_vec);
+            ub[i] = INSIDE ? load8_inside(B, ldb, k0 + s / (TN / 8), n0 + 8 * (s % (TN / 8)))
+                           : load8(B, ldb, K, N, k0 + s / (TN / 8), n0 + 8 * (s % (TN / 8)), b_vec);
         }
     };
     auto stage = [&](int nb) {
@@ -140,10 +150,12 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
                 b[4 * g + 3] = bg.w;
             }
             const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+            // column-major sweep of the outer product (each b[j] held across
+            // the eight rows): measured 2-5 % faster than row-major on GB300
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
+            for (int j = 0; j < 4 * NG; ++j)
 #pragma unroll
-                for (int j = 0; j < 4 * NG; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+                for (int i = 0; i < 8; ++i) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
         }
         if (more) {
             const int nb = buf ^ 1;
@@ -156,13 +168,13 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
         const int64_t r = m0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + (i - 4));
-        if (r >= M) continue;
+        if (!INSIDE && r >= M) continue;
         float *cr = C + r * ldc;
 #pragma unroll
         for (int g = 0; g < NG; ++g) {
             const int64_t c = n0 + g * 64 + tx * 4;
             const float *v = &acc[i][4 * g];
-            if (c_vec && c + 4 <= N) {
+            if (INSIDE || (c_vec && c + 4 <= N)) {
                 *reinterpret_cast<float4 *>(cr + c) = make_float4(v[0], v[1], v[2], v[3]);
             } else {
 #pragma unroll
@@ -211,35 +223,44 @@ cudaError_t launch_small(const uint16_t *a, int64_t lda, const uint16_t *b, int6
     return cudaGetLastError();
 }
 
-template <bool F16, int NG, int TK, int MINB>
-cudaError_t launch_cfg(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
-                       int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c_vec, cudaStream_t s) {
+template <bool F16, int NG, int TK, int MINB, bool INSIDE>
+cudaError_t launch_cfg_as(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
+                          int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c_vec, cudaStream_t s) {
     constexpr int TN = 64 * NG;
     constexpr size_t smem = (size_t)2 * TK * (TM + TN) * sizeof(float);
     static const cudaError_t attr = cudaFuncSetAttribute(
-        gemm_ref_simt<F16, NG, TK, MINB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        gemm_ref_simt<F16, NG, TK, MINB, INSIDE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (attr != cudaSuccess) return attr;
     dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
-    gemm_ref_simt<F16, NG, TK, MINB><<<grid, 256, smem, s>>>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec);
+    gemm_ref_simt<F16, NG, TK, MINB, INSIDE><<<grid, 256, smem, s>>>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec,
+                                                                     c_vec);
     return cudaGetLastError();
 }
 
-// Tiling of the reference (KREX_REF_TILE selects another for experiments):
-// 0 = 128x128, TK 16, one block per SM (143 registers); 1 = 128x256, TK 16;
-// 2 = 128x128, TK 32; 3 = 128x256, TK 32; 4 = 128x128, TK 16 with at most 128
-// registers, so two blocks share an SM.  Measured on GB300 (TFLOP/s at 4096^3
-// / 8192^3, L2 flushed): 53.3/54.5, 49.9/56.6, 50.7/51.8, 43.0/49.0,
-// 54.8/57.2, all bit-identical (each output is one k-order FMA chain); the
-// packed fp32x2 FMA form of 4 ran slower (51.6/54.0), and so did 4 with 32-deep
-// slices (49.8/52.2).  Default: 4, or 5 (the one-output-per-thread kernel)
-// when the GEMM has at most 16 tiles of 128x128 (L2 flushed: 256^3 30 -> 18
-// us, 512^3 53 -> 47 us; at 768^3, 36 tiles, the tiled form is faster).
+template <bool F16, int NG, int TK, int MINB>
+cudaError_t launch_cfg(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
+                       int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c_vec, cudaStream_t s) {
+    const bool inside = M % TM == 0 && N % (64 * NG) == 0 && K % TK == 0 && a_vec && b_vec && c_vec;
+    return inside ? launch_cfg_as<F16, NG, TK, MINB, true>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s)
+                  : launch_cfg_as<F16, NG, TK, MINB, false>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
+}
+
+// Tiling of the reference (the tuning record's reference_tiling selects another
+// for comparisons): 0 = 128x128, TK 16, one block per SM (143 registers); 1 =
+// 128x256, TK 16; 2 = 128x128, TK 32; 3 = 128x256, TK 32; 4 = 128x128, TK 16
+// with at most 128 registers, so two blocks share an SM.  Measured on GB300
+// (TFLOP/s at 4096^3 / 8192^3, L2 flushed, before the column-major sweep and
+// the unchecked form): 53.3/54.5, 49.9/56.6, 50.7/51.8, 43.0/49.0, 54.8/57.2,
+// all bit-identical (each output is one k-order FMA chain).  Also measured and
+// dropped: packed fp32x2 FMAs (with duplicated or diagonally paired operands:
+// 47-55 at 16384^3), 32-deep slices with two blocks per SM, per-thread tiles of
+// 4x16, 16x4, 8x16 and 16x8 (54-59 at 16384^3).  Default: 4, or 5 (the
+// one-output-per-thread kernel) when the GEMM has at most 16 tiles of 128x128
+// (L2 flushed: 256^3 30 -> 18 us, 512^3 53 -> 47 us; at 768^3, 36 tiles, the
+// tiled form is faster).
 int ref_tile(int64_t M, int64_t N) {
-    const char *e = getenv("KREX_REF_TILE");
-    if (e) {
-        int v = atoi(e);
-        if (v >= 0 && v <= 5) return v;
-    }
+    const int v = tuning_snapshot().reference_tiling;
+    if (v >= 0 && v <= 5) return v;
     return ((M + 127) / 128) * ((N + 127) / 128) <= 16 ? 5 : 4;
 }
 

@@ -19,9 +19,10 @@
 //               not 16-byte aligned).
 // Pair tiles run in raster groups of rows so concurrently running pairs share
 // A and B panels in L2; a final partial wave is split in two (column halves,
-// or K halves whose fp32 partials meet in a caller-provided workspace).  A
-// 1-SM form (gemm_bf16_tcgen05, cta_group::1, 128 x 256 tiles, bf16) is kept
-// for comparison.
+// or K halves whose fp32 partials meet in a caller-provided workspace).  The
+// launch configuration (pair-tile width, stage depth, ring depth, raster
+// group, tail split, split-K policy, wait bound) comes from the library's
+// tuning record (krex_set_tuning); its defaults are the measured choices.
 //
 // Every mbarrier and flag wait is bounded (globaltimer); a wait that runs out
 // sets a shared abort flag, the device status word and a record of where each
@@ -47,26 +48,11 @@ __device__ unsigned long long g_gemm_diag[8];
 
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64;
-constexpr int STAGES = 4;
-constexpr int A_STAGE_BYTES = BM * BK * 2;          // 16 KiB
+// TMA boxes shared by the host-side tensor maps: A boxes of BK x BM (K-major),
+// B boxes of B_BOX_N x BK (N-major); 256 threads per CTA.
+constexpr int BM = 128, BK = 64;
 constexpr int B_BOX_N = 64;                         // 64 bf16 = 128-byte swizzle span
-constexpr int B_BOXES = BN / B_BOX_N;               // 4 boxes per stage
-constexpr int B_BOX_BYTES = BK * B_BOX_N * 2;       // 8 KiB
-constexpr int B_STAGE_BYTES = BK * BN * 2;          // 32 KiB
-constexpr int TMEM_COLS = 2 * BN;                   // 512
 constexpr int THREADS = 256;
-constexpr int GROUP_M = 16;
-constexpr int EPI_THREADS = 128;
-constexpr int NUM_BARS = 2 * STAGES + 4 + 1;        // full, empty, tmem_full[2], tmem_empty[2], mma_done
-constexpr size_t SMEM_BYTES = 1024 /*align slack*/ + (size_t)STAGES * (A_STAGE_BYTES + B_STAGE_BYTES) +
-                              NUM_BARS * 8 + 48;
-
-// Instruction descriptor, kind::f16: D fp32 (bits 4-5 = 1), A bf16 (bits 7-9 =
-// 1), B bf16 (bits 10-12 = 1), A K-major (bit 15 = 0), B MN-major (bit 16 = 1),
-// N >> 3 in bits 17-22, M >> 4 in bits 24-28.
-constexpr uint32_t IDESC = (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | (1u << 16) |
-                           ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
 
 // Shared-memory matrix descriptor: start >> 4 (bits 0-13), leading byte
 // offset >> 4 (16-29), stride byte offset >> 4 (32-45), version 1 (46-47),
@@ -216,22 +202,6 @@ __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                         uint32_t accumulate) {
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(IDESC), "r"(accumulate)
-        : "memory");
-}
-
-__device__ __forceinline__ void mma_commit(uint32_t bar) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-        : "memory");
-}
-
 // 32 consecutive fp32 columns of this warp's 32 TMEM lanes (thread t <-> lane base+t).
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile(
@@ -247,209 +217,6 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-__device__ __forceinline__ void tile_coords(int tile, int tiles_m, int tiles_n, int &mb, int &nb) {
-    const int per_group = GROUP_M * tiles_n;
-    const int g = tile / per_group;
-    const int first_m = g * GROUP_M;
-    const int gsize = min(tiles_m - first_m, GROUP_M);
-    const int in_g = tile - g * per_group;
-    mb = first_m + in_g % gsize;
-    nb = in_g / gsize;
-}
-
-__global__ void __launch_bounds__(THREADS, 1)
-gemm_bf16_tcgen05(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                  uint16_t *__restrict__ C, int64_t ldc, int M, int N, int K, int tiles_m,
-                  int tiles_n, int c_vec, uint64_t timeout_ns) {
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                                ~uintptr_t(1023));
-    uint8_t *sA = smem;
-    uint8_t *sB = smem + STAGES * A_STAGE_BYTES;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(sB + STAGES * B_STAGE_BYTES);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + NUM_BARS);
-    volatile uint32_t *abort_flag = tmem_slot + 1;
-
-    const uint32_t bar0 = smem_u32(bars);
-    auto full_bar = [&](int s) { return bar0 + 8u * s; };
-    auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
-    auto tfull_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + a); };
-    auto tempty_bar = [&](int a) { return bar0 + 8u * (2 * STAGES + 2 + a); };
-    const uint32_t mma_done_bar = bar0 + 8u * (2 * STAGES + 4);
-
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int num_tiles = tiles_m * tiles_n;
-    const int num_kb = (K + BK - 1) / BK;
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(full_bar(s), 1);
-            mbar_init(empty_bar(s), 1);
-        }
-        for (int a = 0; a < 2; ++a) {
-            mbar_init(tfull_bar(a), 1);
-            mbar_init(tempty_bar(a), EPI_THREADS);
-        }
-        mbar_init(mma_done_bar, 1);
-        for (int i = 0; i < PROG_WORDS; ++i) abort_flag[i] = 0u;
-        abort_flag[7] = (uint32_t)M;
-        abort_flag[8] = (uint32_t)N;
-        abort_flag[9] = (uint32_t)K;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmA)) : "memory");
-        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tmB)) : "memory");
-    }
-    if (warp == 2) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         smem_u32(tmem_slot)),
-                     "r"(TMEM_COLS)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem_base = *tmem_slot;
-
-    if (warp == 0 && lane == 0) {
-        // ------------------------------------------------------ TMA producer
-        int stage = 0;
-        uint32_t phase = 0;
-        int filled = 0;  // total stage fills issued
-        bool ok = true;
-        for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x) {
-            int mb, nb;
-            tile_coords(tile, tiles_m, tiles_n, mb, nb);
-            const int n0 = nb * BN;
-            const int nbox = min(B_BOXES, (N - n0 + B_BOX_N - 1) / B_BOX_N);  // boxes inside N
-            const uint32_t bytes = A_STAGE_BYTES + nbox * B_BOX_BYTES;
-            for (int kb = 0; kb < num_kb; ++kb) {
-                if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, timeout_ns, 0x01)) {
-                    ok = false;
-                    break;
-                }
-                mbar_expect_tx(full_bar(stage), bytes);
-                tma_load_2d(smem_u32(sA + stage * A_STAGE_BYTES), &tmA, full_bar(stage), kb * BK,
-                            mb * BM);
-                for (int j = 0; j < nbox; ++j)
-                    tma_load_2d(smem_u32(sB + stage * B_STAGE_BYTES + j * B_BOX_BYTES), &tmB,
-                                full_bar(stage), n0 + j * B_BOX_N, kb * BK);
-                ++filled;
-                if (++stage == STAGES) {
-                    stage = 0;
-                    phase ^= 1u;
-                }
-            }
-        }
-        if (!ok) {
-            // let the loads already issued land before shared memory is released
-            const int last = filled < STAGES ? filled : STAGES;
-            for (int i = 1; i <= last; ++i) {
-                const int f = filled - i;
-                mbar_wait(full_bar(f % STAGES), (uint32_t)((f / STAGES) & 1), abort_flag,
-                          10000000ull, 0x02, true);
-            }
-        }
-    } else if (warp == 1 && lane == 0) {
-        // --------------------------------------------------------- MMA issuer
-        int stage = 0;
-        uint32_t phase = 0;
-        bool ok = true;
-        int local = 0;
-        for (int tile = blockIdx.x; ok && tile < num_tiles; tile += gridDim.x, ++local) {
-            const int acc = local & 1;
-            const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
-            if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, timeout_ns, 0x11)) {
-                ok = false;
-                break;
-            }
-            tc_fence_after();
-            const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
-            for (int kb = 0; kb < num_kb; ++kb) {
-                if (!mbar_wait(full_bar(stage), phase, abort_flag, timeout_ns, 0x12)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint64_t adesc = sdesc_sw128(smem_u32(sA + stage * A_STAGE_BYTES), 16, 1024);
-                const uint64_t bdesc =
-                    sdesc_sw128(smem_u32(sB + stage * B_STAGE_BYTES), B_BOX_BYTES, 1024);
-#pragma unroll
-                for (int k = 0; k < BK / 16; ++k) {
-                    // A: +32 bytes along K inside the 128B swizzle row; B: +2 core
-                    // groups of 8 K-rows (2 x 1024 bytes) per K=16 step.
-                    mma_bf16(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(128 * k),
-                             (kb | k) != 0 ? 1u : 0u);
-                }
-                mma_commit(empty_bar(stage));
-                if (++stage == STAGES) {
-                    stage = 0;
-                    phase ^= 1u;
-                }
-            }
-            if (ok) mma_commit(tfull_bar(acc));
-        }
-        // all MMAs issued by this thread complete before TMEM can be freed
-        mma_commit(mma_done_bar);
-        mbar_wait(mma_done_bar, 0u, abort_flag, 10000000ull, 0x13, true);
-    } else if (warp >= 4) {
-        // ----------------------------------------------------------- epilogue
-        const int ew = warp - 4;  // TMEM lanes [32*ew, 32*ew+32)
-        int local = 0;
-        for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x, ++local) {
-            int mb, nb;
-            tile_coords(tile, tiles_m, tiles_n, mb, nb);
-            const int acc = local & 1;
-            const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
-            // every lane waits; the vote keeps the warp converged (all lanes load
-            // or none) for the .sync.aligned TMEM loads even if a wait runs out
-            const bool waited = mbar_wait(tfull_bar(acc), acc_phase, abort_flag, timeout_ns, 0x21);
-            if (!__all_sync(0xffffffffu, waited)) break;
-            tc_fence_after();
-            const int row = mb * BM + ew * 32 + lane;
-            const int n0 = nb * BN;
-            uint16_t *crow = C + (int64_t)row * ldc;
-#pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
-                const int col0 = n0 + c * 32;
-                if (col0 >= N) break;  // warp-uniform
-                uint32_t v[32];
-                tmem_ld32(tmem_base + ((uint32_t)(ew * 32) << 16) + (uint32_t)(acc * BN + c * 32), v);
-                if (row < M) {
-                    uint32_t p[16];
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) {
-                        __nv_bfloat162 h =
-                            __floats2bfloat162_rn(__uint_as_float(v[2 * i]), __uint_as_float(v[2 * i + 1]));
-                        p[i] = *reinterpret_cast<uint32_t *>(&h);
-                    }
-                    if (c_vec && col0 + 32 <= N) {
-                        uint4 *dst = reinterpret_cast<uint4 *>(crow + col0);
-                        dst[0] = make_uint4(p[0], p[1], p[2], p[3]);
-                        dst[1] = make_uint4(p[4], p[5], p[6], p[7]);
-                        dst[2] = make_uint4(p[8], p[9], p[10], p[11]);
-                        dst[3] = make_uint4(p[12], p[13], p[14], p[15]);
-                    } else {
-                        for (int i = 0; i < 32 && col0 + i < N; ++i)
-                            crow[col0 + i] = (uint16_t)((i & 1) ? (p[i >> 1] >> 16) : (p[i >> 1] & 0xFFFFu));
-                    }
-                }
-            }
-            tc_fence_before();
-            mbar_arrive(tempty_bar(acc));
-        }
-    }
-
-    // ---------------------------------------------------------------- teardown
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 2) {
-        tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_base),
-                     "r"(TMEM_COLS)
-                     : "memory");
-    }
-}
 
 // ===================================================== 2-SM (cta_group::2) form
 //
@@ -458,7 +225,7 @@ gemm_bf16_tcgen05(const __grid_constant__ CUtensorMap tmA, const __grid_constant
 // A tile and columns [128r, 128r+128) of the B tile in its own shared memory,
 // and its own TMEM holds its 128 rows of the 256-column accumulator.  Per SM
 // a stage is 32 KiB (A 128x64 + half of B 64x128), so six stages fit and the
-// L2 -> SM traffic per flop is two thirds of the 1-SM form.
+// L2 -> SM traffic per flop is two thirds of a one-SM 128 x 256 tile's.
 //   - both CTAs' TMA loads complete on the leader CTA's (rank 0) full barrier
 //     (.cta_group::2 lets the barrier live in the peer CTA);
 //   - the leader's MMA thread releases a stage in both CTAs and publishes an
@@ -688,7 +455,7 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                       int group_m, int c_vec, int c_tma, int stages, uint64_t timeout_ns, int split_k,
                       float *ws_partial, uint32_t *ws_count, uint32_t *ws_flag, uint32_t launch_id,
                       uint32_t wait_tag) {
-    // this kernel's tile constants shadow the 1-SM ones
+    // the pair kernel's tile constants (the file-level BM, BK serve the host's tensor maps)
     using CF = v2::Cfg<KSUB>;
     constexpr int BM = v2::BM, BN = v2::BN, BK = v2::BK, STAGES = CF::STAGES;
     constexpr int A_STAGE_BYTES = CF::A_STAGE_BYTES, B_STAGE_BYTES = CF::B_STAGE_BYTES;
@@ -1101,96 +868,50 @@ krex_status make_map(const void *ptr, uint64_t inner, uint64_t outer, uint64_t l
     return KREX_OK;
 }
 
-// Pair-tile width for the 2-SM kernel.  Measured on GB300, a tcgen05.mma of
-// N = 224 or 192 costs about as much time as N = 256, so narrower tiles only
-// add waves: 256 everywhere.  KREX_GEMM_BN (128, 192 or 256: the epilogue
-// stores 64-column boxes) overrides it for experiments and tests.
-int pick_pair_tile_n() {
-    const char *e = getenv("KREX_GEMM_BN");
-    if (e) {
-        int v = atoi(e);
-        if (v >= 128 && v <= 256 && v % 64 == 0) return v;
-    }
-    return 256;
-}
+// Launch configuration of the 2-SM kernel, from the library's tuning record
+// (krex_get_tuning_internal); a field at its default takes the measured
+// choice documented beside it.
+//
+// Pair-tile width: measured on GB300, a tcgen05.mma of N = 224 or 192 costs
+// about as much time as N = 256, so narrower tiles only add waves: 256
+// unless set (128, 192 or 256: the epilogue stores 64-column boxes).
+int pick_pair_tile_n(const krex_tuning &t) { return t.gemm_pair_tile_n ? t.gemm_pair_tile_n : 256; }
 
-// Pair-tile rows per raster group of the 2-SM kernel; KREX_GEMM_GROUP overrides.
 // Pair-tile rows per raster group.  Measured on GB300 (TFLOP/s, group 4 vs
 // 8, L2 flushed): 3072^3 1381 vs 1325, 4096^3 1561 vs 1525, 4608^3 1579 vs
 // 1557, but 2064^3 578 vs 592, 5120^3 1616 vs 1638, 7168^3 1739 vs 1794,
 // 8192^3 1799 vs 1851: 4 for GEMMs of 1.5 to 5 waves of pair tiles, else 8.
-// KREX_GEMM_GROUP overrides it for experiments.
-int raster_group(int64_t tiles, int max_clusters) {
-    const char *e = getenv("KREX_GEMM_GROUP");
-    if (e) {
-        int v = atoi(e);
-        if (v >= 1 && v <= 64) return v;
-    }
+int raster_group(const krex_tuning &t, int64_t tiles, int max_clusters) {
+    if (t.gemm_raster_group) return t.gemm_raster_group;
     return (2 * tiles >= 3 * (int64_t)max_clusters && tiles < 5 * (int64_t)max_clusters) ? 4 : v2::GROUP_M;
 }
 
-// Column-half split of a final partial wave (on unless KREX_GEMM_TAIL_SPLIT=0).
-// KREX_DEBUG_STALL_HANDOVER=1 (read per launch; for the failure-detection
-// test only) makes the second K half of a split tile wait for a tag that no
-// launch publishes, so its bounded wait runs out: the kernel then sets the
-// status word (0x1052), drains and returns, and the context stays usable.
-bool debug_stall_handover() {
-    const char *e = getenv("KREX_DEBUG_STALL_HANDOVER");
-    return e && e[0] == '1';
-}
-
-// K halves for a single partial wave (when a workspace is given): "auto"
-// (K >= kSplitKMinK), or KREX_GEMM_SPLIT_K=1 (whenever the shape allows: the
-// tests use it to exercise the hand-over on small shapes) / =0 (never).
-// Measured on GB300 (L2 flushed): the hand-over of the fp32 partials costs
-// about 4-6 us, so below K = 4096 column halves win (256^3: 10.2 against
-// 16.4 us; 1024^3: 14.3 against 18.5 us), while 1024 x 2048 x 8192 gains 8 %.
+// K halves for a single partial wave (when a workspace is given): by default
+// when K >= kSplitKMinK; the tuning record can force them whenever the shape
+// allows (the tests use that to exercise the hand-over on small shapes) or
+// switch them off.  Measured on GB300 (L2 flushed): the hand-over of the fp32
+// partials costs about 4-6 us, so below K = 4096 column halves win (256^3:
+// 10.2 against 16.4 us; 1024^3: 14.3 against 18.5 us), while 1024 x 2048 x
+// 8192 gains 8 %.
 constexpr int64_t kSplitKMinK = 4096;
-int split_k_mode() {
-    const char *e = getenv("KREX_GEMM_SPLIT_K");
-    if (e && (e[0] == '0' || e[0] == '1')) return e[0] - '0';
-    return -1;
+
+// Stages of the shared-memory ring in use (at most `max_stages`).
+int ring_stages(const krex_tuning &t, int max_stages) {
+    return t.gemm_ring_stages ? t.gemm_ring_stages : max_stages;
 }
 
-bool tail_split_enabled() {
-    const char *e = getenv("KREX_GEMM_TAIL_SPLIT");
-    return !(e && e[0] == '0');
-}
+// K sub-blocks (of 64) per ring stage: 2 = three 64 KiB stages (default),
+// 1 = six 32 KiB stages.
+int stage_ksub(const krex_tuning &t) { return t.gemm_stage_k == 64 ? 1 : 2; }
 
-// Stages of the 2-SM kernel's shared-memory ring in use (at most `max_stages`);
-// KREX_GEMM_STAGES overrides.
-int ring_stages(int max_stages) {
-    const char *e = getenv("KREX_GEMM_STAGES");
-    if (e) {
-        int v = atoi(e);
-        if (v >= 2 && v <= max_stages) return v;
-    }
-    return max_stages;
-}
+// The second K half of a split tile waits for a tag that no launch publishes
+// while this is set (krex_debug_stall_handover; the failure-detection test
+// only), so its bounded wait runs out: the kernel then sets the status word
+// (0x1052), drains and returns, and the context stays usable.
+std::atomic<int> g_debug_stall_handover{0};
 
-// K sub-blocks (of 64) per ring stage of the 2-SM kernel: 2 = three 64 KiB
-// stages, 1 = six 32 KiB stages; KREX_GEMM_KSUB overrides.
-int stage_ksub() {
-    const char *e = getenv("KREX_GEMM_KSUB");
-    if (e && (e[0] == '1' || e[0] == '2')) return e[0] - '0';
-    return 2;
-}
-
-// 2 = the 2-SM (cta_group::2) kernel, 1 = the 1-SM kernel; KREX_GEMM_SM picks
-// one (read on every call so a process can compare both).
-int gemm_variant() {
-    const char *e = getenv("KREX_GEMM_SM");
-    return (e && e[0] == '1') ? 1 : 2;
-}
-
-uint64_t wait_timeout_ns() {
-    static uint64_t t = [] {
-        const char *e = getenv("KREX_WAIT_TIMEOUT_MS");
-        long ms = e ? atol(e) : 0;
-        if (ms <= 0) ms = 2000;
-        return (uint64_t)ms * 1000000ull;
-    }();
-    return t;
+uint64_t wait_timeout_ns(const krex_tuning &t) {
+    return (uint64_t)(t.wait_timeout_ms > 0 ? t.wait_timeout_ms : 2000) * 1000000ull;
 }
 
 }  // namespace
@@ -1213,7 +934,7 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         KREX_CUDA_TRY(cudaMemset2DAsync(c, (size_t)ldc * 2, 0, (size_t)N * 2, (size_t)M, s));
         return KREX_OK;
     }
-    if (M > (1ll << 31) - BM || N > (1ll << 31) - BN || K > (1ll << 31) - BK)
+    if (M > (1ll << 31) - 2 * v2::BM || N > (1ll << 31) - v2::BN || K > (1ll << 31) - BK)
         return set_error(KREX_ERR_UNSUPPORTED, "GEMM dimension too large for the tcgen05 path");
     // Tensor-map encoding is a driver call and needs a current context on this
     // thread; a thread whose first CUDA work is this GEMM has none yet, so bind
@@ -1227,6 +948,7 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
             bound_dev = d;
         }
     }
+    const krex_tuning tun = tuning_snapshot();
     CUtensorMap ma, mb;
     krex_status st = make_map(a, (uint64_t)K, (uint64_t)M, (uint64_t)lda, BK, BM, f16, &ma);
     if (st != KREX_OK) return st;
@@ -1238,8 +960,6 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
     int dev = 0;
     KREX_CUDA_TRY(cudaGetDevice(&dev));
     if (attr_dev != dev) {
-        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_bf16_tcgen05, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)SMEM_BYTES));
         KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            (int)v2::Cfg<1>::SMEM_BYTES));
         KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -1262,7 +982,7 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         attr_dev = dev;
     }
     const int c_vec = ((reinterpret_cast<uintptr_t>(c) & 15u) == 0) && (ldc % 8 == 0);
-    if (gemm_variant() == 2 || f16) {  // the 1-SM form is bf16 only
+    {
         // TMA-store epilogue when C rows start on 16 bytes; else direct stores
         CUtensorMap mc;
         int c_tma = c_vec;
@@ -1273,19 +993,19 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
             mc = ma;  // unused
         }
         const int tiles_m = (int)((M + 2 * v2::BM - 1) / (2 * v2::BM));
-        const int bn = pick_pair_tile_n();
+        const int bn = pick_pair_tile_n(tun);
         const int tiles_n = (int)((N + bn - 1) / bn);
         const int64_t tiles = (int64_t)tiles_m * tiles_n;
         // Split the tiles of a final partial wave into column halves when that
         // at most fills the co-resident pairs (4096^2: 256 tiles on 76 pairs ->
         // 228 whole tiles + 56 halves instead of a last wave of 28 tiles).
         const int64_t rem = tiles % max_clusters;
-        const bool split = bn == 256 && rem > 0 && 2 * rem <= max_clusters && tail_split_enabled();
+        const bool split = bn == 256 && rem > 0 && 2 * rem <= max_clusters && tun.gemm_tail_split != 0;
         const int64_t full_items = split ? tiles - rem : tiles;
         const int64_t items = split ? tiles + rem : tiles;
         const int clusters = (int)(items < max_clusters ? items : max_clusters);
         // K halves (full-width MMAs) when a zero-initialised workspace is given,
-        // K has at least two ring stages and is long enough (split_k_mode), and
+        // K has at least two ring stages and is long enough (the tuning's split_k), and
         // the split tiles are the whole GEMM (one partial wave); else column
         // halves.  Measured on GB300: K
         // halves load a third less than column halves (1024 x 2048 x 8192:
@@ -1293,9 +1013,9 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         // written, then read) sits on the last wave's critical path: at 4096^3
         // the K halves end their MMAs 6.8 us earlier and spend about as long
         // exchanging partials, so the multi-wave case gains nothing.
-        const int ksub = stage_ksub();
+        const int ksub = stage_ksub(tun);
         const int64_t num_kb = (((K + 63) / 64) + ksub - 1) / ksub;
-        const int sk_mode = split_k_mode();
+        const int sk_mode = tun.gemm_split_k;
         const bool k_worth_it = sk_mode == 1 || (sk_mode < 0 && K >= kSplitKMinK);
         const int split_k = split && full_items == 0 && workspace && workspace_bytes >= WS_BYTES &&
                             rem <= WS_SLOTS && num_kb >= 2 && clusters >= 2 && k_worth_it;
@@ -1304,7 +1024,7 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         if (launch_id == 0) launch_id = launch_counter.fetch_add(1) + 1;  // 0 never tags a published partial
         // the tag the second K half waits for: this launch's, or (the failure-
         // detection test's switch) one that no launch publishes
-        const uint32_t wait_tag = debug_stall_handover() ? (launch_id ^ 0x80000000u) : launch_id;
+        const uint32_t wait_tag = g_debug_stall_handover.load() ? (launch_id ^ 0x80000000u) : launch_id;
         float *ws_partial = split_k ? static_cast<float *>(workspace) : nullptr;
         uint32_t *ws_count =
             split_k ? reinterpret_cast<uint32_t *>(static_cast<uint8_t *>(workspace) + WS_PARTIAL_BYTES) : nullptr;
@@ -1312,11 +1032,11 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         auto go = [&](auto kernel, size_t smem, int stages) {
             kernel<<<2 * clusters, THREADS, smem, s>>>(ma, mb, mc, c, ldc, (int)M, (int)N, (int)K, bn, tiles_m,
                                                        tiles_n, (int)full_items, (int)items,
-                                                       raster_group(tiles, max_clusters), c_vec,
-                                                       c_tma, stages, wait_timeout_ns(), split_k, ws_partial,
+                                                       raster_group(tun, tiles, max_clusters), c_vec,
+                                                       c_tma, stages, wait_timeout_ns(tun), split_k, ws_partial,
                                                        ws_count, ws_flag, launch_id, wait_tag);
         };
-        const int st2 = ring_stages(v2::Cfg<2>::STAGES), st1 = ring_stages(v2::Cfg<1>::STAGES);
+        const int st2 = ring_stages(tun, v2::Cfg<2>::STAGES), st1 = ring_stages(tun, v2::Cfg<1>::STAGES);
         if (ksub == 2 && f16)
             go(gemm_tcgen05_2sm<2, true>, v2::Cfg<2>::SMEM_BYTES, st2);
         else if (ksub == 2)
@@ -1325,16 +1045,12 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
             go(gemm_tcgen05_2sm<1, true>, v2::Cfg<1>::SMEM_BYTES, st1);
         else
             go(gemm_tcgen05_2sm<1, false>, v2::Cfg<1>::SMEM_BYTES, st1);
-    } else {
-        const int tiles_m = (int)((M + BM - 1) / BM), tiles_n = (int)((N + BN - 1) / BN);
-        const int64_t tiles = (int64_t)tiles_m * tiles_n;
-        const int grid = (int)(tiles < sm_count() ? tiles : sm_count());
-        gemm_bf16_tcgen05<<<grid, THREADS, SMEM_BYTES, s>>>(ma, mb, c, ldc, (int)M, (int)N, (int)K, tiles_m,
-                                                            tiles_n, c_vec, wait_timeout_ns());
     }
     KREX_CUDA_TRY(cudaGetLastError());
     return KREX_OK;
 }
+
+void set_debug_stall_handover(bool on) { g_debug_stall_handover.store(on ? 1 : 0); }
 
 cudaError_t read_device_status_detail(unsigned long long *words) {
     cudaError_t e = cudaDeviceSynchronize();

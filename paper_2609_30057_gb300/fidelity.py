@@ -32,7 +32,7 @@ import threading
 import time
 
 from . import (KREX_OP_GEMM_BF16, KREX_OP_SOFTMAX_F32, Gate, KrexError, build, krex_bench_candidate,
-               krex_device_status, krex_device_status_detail, krex_gen_inputs, krex_run_candidate)
+               krex_device_status, krex_device_status_detail, krex_gen_inputs, krex_run_candidate, tuning)
 
 
 def _device_status(details: dict | None = None, phase: str = "") -> int:
@@ -136,22 +136,22 @@ def candidates(device="cuda", quick: bool = False):
 
 
 # Variants of the tcgen05 kernel on one 4096^3 GEMM, as an agent tuning it
-# would produce: K depth per ring stage, pair-tile width, the 1-SM form, the
-# raster group and the ring depth (knob settings of gemm_tcgen05.cu).
+# would produce: K depth per ring stage, pair-tile width, the raster group and
+# the ring depth (fields of the library's tuning record, krex_set_tuning).
 TILE_VARIANTS = (
     ("sm2_k128_n256", {}),
-    ("sm2_k64_n256", {"KREX_GEMM_KSUB": "1"}),
-    ("sm2_k128_n192", {"KREX_GEMM_BN": "192"}),
-    ("sm2_k128_n128", {"KREX_GEMM_BN": "128"}),
-    ("sm2_k128_g8", {"KREX_GEMM_GROUP": "8"}),
-    ("sm2_k64_st5", {"KREX_GEMM_KSUB": "1", "KREX_GEMM_STAGES": "5"}),
-    ("sm1_n256", {"KREX_GEMM_SM": "1"}),
+    ("sm2_k64_n256", {"gemm_stage_k": 64}),
+    ("sm2_k128_n192", {"gemm_pair_tile_n": 192}),
+    ("sm2_k128_n128", {"gemm_pair_tile_n": 128}),
+    ("sm2_k128_g8", {"gemm_raster_group": 8}),
+    ("sm2_k64_st5", {"gemm_stage_k": 64, "gemm_ring_stages": 5}),
+    ("sm2_k128_g2", {"gemm_raster_group": 2}),
 )
 
 
 def tile_variant_candidates(device="cuda"):
-    """(name, op, inputs, out, env) for the kernel variants above on one
-    4096^3 GEMM; timing sets each variant's knobs in this process only, so
+    """(name, op, inputs, out, tuning) for the kernel variants above on one
+    4096^3 GEMM; timing sets each variant's tuning in this process only, so
     it is used where no thread of this process launches GEMMs concurrently."""
     import torch
     n = 4096
@@ -160,30 +160,21 @@ def tile_variant_candidates(device="cuda"):
     krex_gen_inputs(7, 0, 0, 0.0, a)
     krex_gen_inputs(7, 1, 0, 0.0, b)
     c = torch.empty(n, n, dtype=torch.bfloat16, device=device)
-    return [(f"gemm4096_{name}", KREX_OP_GEMM_BF16, [a, b], c, env) for name, env in TILE_VARIANTS]
+    return [(f"gemm4096_{name}", KREX_OP_GEMM_BF16, [a, b], c, knobs) for name, knobs in TILE_VARIANTS]
 
 
 def time_candidates(cands, flush, iters, stream, gate=None, tenant=0, per_iter=None):
     """Median of `iters` flushed, timed iterations of each candidate (the
     command's timed loop), optionally inside a gated region.  `per_iter`, if
     a list, receives every candidate's iteration durations.  A candidate's
-    optional fifth field is a dict of kernel knobs set while it is timed."""
-    import os
+    optional fifth field is a dict of tuning fields set while it is timed."""
     out = []
     for cand in cands:
         name, op, ins, o = cand[:4]
-        env = cand[4] if len(cand) > 4 else {}
-        saved = {k: os.environ.get(k) for k in env}
-        os.environ.update(env)
-        try:
+        knobs = cand[4] if len(cand) > 4 else {}
+        with tuning(**knobs):
             d, p50, _ = krex_bench_candidate(op, ins, o, warmup=3, iters=iters, flush_scratch=flush,
                                              flush_bytes=flush.numel(), stream=stream, gate=gate, tenant=tenant)
-        finally:
-            for k, v in saved.items():
-                if v is None:
-                    os.environ.pop(k, None)
-                else:
-                    os.environ[k] = v
         out.append(p50)
         if per_iter is not None:
             per_iter.append(list(d))

@@ -145,3 +145,42 @@ def test_command_argument_validation(lib):
         == krex.KREX_ERR_INVALID
     assert lib.krex_command_run(None, ctypes.byref(bufs), None, None, None, ctypes.byref(res), None) \
         == krex.KREX_ERR_INVALID
+
+
+def test_tuning_defaults_roundtrip_and_range_checks():
+    # the library's launch configuration is an explicit record, never its
+    # environment: defaults, a set/get round trip, rejection of out-of-range
+    # fields (which leaves the record unchanged), NULL restoring the defaults
+    import paper_2609_30057_gb300 as krex
+    lib = krex.lib()
+    d = krex.krex_tuning()
+    lib.krex_tuning_defaults(ctypes.byref(d))
+    assert (d.gemm_pair_tile_n, d.gemm_stage_k, d.gemm_ring_stages, d.gemm_raster_group, d.gemm_tail_split,
+            d.gemm_split_k, d.reference_tiling, d.wait_timeout_ms) == (0, 0, 0, 0, -1, -1, -1, 0)
+    try:
+        krex.krex_set_tuning(gemm_pair_tile_n=192, gemm_stage_k=64, gemm_ring_stages=5, gemm_raster_group=3,
+                             gemm_tail_split=0, gemm_split_k=1, reference_tiling=2, wait_timeout_ms=500)
+        got = krex.krex_get_tuning()
+        assert got == {"gemm_pair_tile_n": 192, "gemm_stage_k": 64, "gemm_ring_stages": 5, "gemm_raster_group": 3,
+                       "gemm_tail_split": 0, "gemm_split_k": 1, "reference_tiling": 2, "wait_timeout_ms": 500}
+        bad = [{"gemm_pair_tile_n": 100}, {"gemm_stage_k": 32}, {"gemm_ring_stages": 4},  # 4 > 3 stages of K 128
+               {"gemm_ring_stages": 1}, {"gemm_raster_group": 65}, {"gemm_tail_split": 2}, {"gemm_split_k": -2},
+               {"reference_tiling": 6}, {"wait_timeout_ms": -1}]
+        for b in bad:
+            with pytest.raises(krex.KrexError, match="INVALID"):
+                krex.krex_set_tuning(**b)
+            assert krex.krex_get_tuning() == got
+        with krex.tuning(gemm_raster_group=9):
+            assert krex.krex_get_tuning()["gemm_raster_group"] == 9
+        assert krex.krex_get_tuning() == got
+    finally:
+        assert lib.krex_set_tuning(None) == krex.KREX_OK
+    assert krex.krex_get_tuning()["reference_tiling"] == -1
+
+
+def test_library_reads_no_environment_variables():
+    # configuration is explicit (krex_tuning): no translation unit calls getenv
+    import glob
+    for f in glob.glob(os.path.join(ROOT, "paper_2609_30057_gb300", "csrc", "*")):
+        with open(f) as fh:
+            assert "getenv" not in fh.read(), f

@@ -1,10 +1,10 @@
 """GPU: failure detection without a fault.  A bounded wait inside the GEMM is
 made to run out (the second K half of a split tile waits for a tag that no
-launch publishes, switched on per launch by KREX_DEBUG_STALL_HANDOVER); the
-kernel must report it through the status word and its detail record, return,
-and leave the context usable: the same GEMM right after is correct.  Runs in
-a child process because the wait limit (KREX_WAIT_TIMEOUT_MS) is read once
-per process."""
+launch publishes, switched on by the krex_debug_stall_handover test hook);
+the kernel must report it through the status word and its detail record,
+return, and leave the context usable: the same GEMM right after is correct.
+Runs in a child process so that the shortened wait bound (the tuning's
+wait_timeout_ms) and the hook touch no other test."""
 import json
 import os
 import subprocess
@@ -25,7 +25,8 @@ import paper_2609_30057_gb300 as krex
 from oracle import gen, ref
 krex.build()
 M, N, K = 1024, 2048, 512            # one partial wave: K halves through the workspace
-os.environ["KREX_GEMM_SPLIT_K"] = "1"  # (at this K only when asked for)
+# K halves (at this K only when asked for) and a 300 ms bound on every wait
+krex.krex_set_tuning(gemm_split_k=1, wait_timeout_ms=300)
 a = torch.empty(M, K, dtype=torch.bfloat16, device="cuda")
 b = torch.empty(K, N, dtype=torch.bfloat16, device="cuda")
 krex.krex_gen_inputs(31, 0, 0, 0.0, a)
@@ -33,7 +34,7 @@ krex.krex_gen_inputs(31, 1, 0, 0.0, b)
 c = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
 ws = krex.gemm_workspace()
 out = {}
-os.environ["KREX_DEBUG_STALL_HANDOVER"] = "1"
+krex.krex_debug_stall_handover(True)
 t0 = time.monotonic()
 krex.krex_run_candidate_ws(krex.KREX_OP_GEMM_BF16, [a, b], c, ws)
 torch.cuda.synchronize()
@@ -43,7 +44,7 @@ try:
     out["status"] = krex.krex_device_status()
 except krex.KrexError as e:
     out["status"] = int(str(e).split("status 0x")[1].rstrip(")"), 16)
-del os.environ["KREX_DEBUG_STALL_HANDOVER"]
+krex.krex_debug_stall_handover(False)
 ws.zero_()
 krex.krex_run_candidate_ws(krex.KREX_OP_GEMM_BF16, [a, b], c, ws)
 torch.cuda.synchronize()
@@ -56,9 +57,7 @@ print("RESULT " + json.dumps(out))
 
 
 def test_bounded_wait_runs_out_and_the_context_stays_usable():
-    env = dict(os.environ, KREX_WAIT_TIMEOUT_MS="300", KREX_GEMM_SM="2")
-    env.pop("KREX_DEBUG_STALL_HANDOVER", None)
-    r = subprocess.run([sys.executable, "-c", "ROOT = %r\n" % ROOT + CHILD], env=env, capture_output=True,
+    r = subprocess.run([sys.executable, "-c", "ROOT = %r\n" % ROOT + CHILD], capture_output=True,
                        text=True, timeout=300)
     assert r.returncode == 0, r.stdout[-2000:] + r.stderr[-2000:]
     line = [l for l in r.stdout.splitlines() if l.startswith("RESULT ")][-1]

@@ -21,12 +21,19 @@ def built():
     krex.build()
 
 
-@pytest.fixture(params=["1", "2", "2k1"], ids=["1sm", "2sm", "2sm_ksub1"])
-def variant(request, monkeypatch):
-    """The tcgen05 kernels: 1-SM (cta_group::1), 2-SM (cta_group::2) with
-    128-deep stages (default) and with 64-deep stages."""
-    monkeypatch.setenv("KREX_GEMM_SM", request.param[0])
-    monkeypatch.setenv("KREX_GEMM_KSUB", "1" if request.param == "2k1" else "2")
+@pytest.fixture(autouse=True)
+def default_tuning():
+    """Every test starts and ends with the library's default tuning."""
+    krex.krex_set_tuning()
+    yield
+    krex.krex_set_tuning()
+
+
+@pytest.fixture(params=["2", "2k1"], ids=["2sm", "2sm_ksub1"])
+def variant(request):
+    """The tcgen05 kernel's two stage depths: 128-deep stages (default) and
+    64-deep stages."""
+    krex.krex_set_tuning(gemm_stage_k=64 if request.param == "2k1" else 128)
     return request.param
 
 
@@ -100,9 +107,8 @@ def test_seeded_gemm_within_tolerance(M, N, K, variant):
 
 @pytest.mark.parametrize("bn", [128, 192, 256])
 @pytest.mark.parametrize("M,N,K", [(300, 1000, 520), (512, 1792, 256), (256, 192, 64), (260, 328, 72)])
-def test_2sm_every_pair_tile_width(M, N, K, bn, monkeypatch):
-    monkeypatch.setenv("KREX_GEMM_SM", "2")
-    monkeypatch.setenv("KREX_GEMM_BN", str(bn))
+def test_2sm_every_pair_tile_width(M, N, K, bn):
+    krex.krex_set_tuning(gemm_pair_tile_n=bn)
     seed = 3000 + M + N + K
     a, b = _gen(seed, M, N, K)
     c = _candidate(a, b)
@@ -130,10 +136,9 @@ def test_output_row_stride(ldc_pad, variant):
 
 @pytest.mark.parametrize("split", ["0", "1"])
 @pytest.mark.parametrize("M,N,K", [(1024, 2048, 512), (4096, 1024, 256), (256, 256, 4096)])
-def test_2sm_tail_split_on_and_off(M, N, K, split, monkeypatch):
+def test_2sm_tail_split_on_and_off(M, N, K, split):
     # a final partial wave of pair tiles is split into column halves (or not)
-    monkeypatch.setenv("KREX_GEMM_SM", "2")
-    monkeypatch.setenv("KREX_GEMM_TAIL_SPLIT", split)
+    krex.krex_set_tuning(gemm_tail_split=int(split))
     seed = 5000 + M + N + K
     a, b = _gen(seed, M, N, K)
     c = _candidate(a, b)
@@ -242,14 +247,13 @@ def test_gemm_large_sampled(n, seed):
 @pytest.mark.parametrize("ksub", ["2", "1"])
 @pytest.mark.parametrize("M,N,K", [(1024, 2048, 512), (256, 256, 4096), (300, 1000, 520), (640, 384, 4104),
                                    (1536, 1536, 3072), (2064, 1000, 1032), (4096, 4096, 256)])
-def test_2sm_split_k_tail(M, N, K, ksub, monkeypatch):
+def test_2sm_split_k_tail(M, N, K, ksub):
     # with a workspace the tiles of a GEMM that fits in one partial wave are
     # split into K halves whose fp32 partials meet in the workspace (larger
     # GEMMs keep column halves); two calls in a row (the arrival counters
     # reset themselves, the flags are tagged per launch)
-    monkeypatch.setenv("KREX_GEMM_SM", "2")
-    monkeypatch.setenv("KREX_GEMM_KSUB", ksub)
-    monkeypatch.setenv("KREX_GEMM_SPLIT_K", "1")   # the hand-over at every K, not only where it pays
+    # the hand-over at every K, not only where it pays
+    krex.krex_set_tuning(gemm_stage_k=64 if ksub == "1" else 128, gemm_split_k=1)
     seed = 6000 + M + N + K
     a, b = _gen(seed, M, N, K)
     ws = krex.gemm_workspace()
@@ -267,10 +271,10 @@ def test_2sm_split_k_tail(M, N, K, ksub, monkeypatch):
         assert torch.count_nonzero(counters).item() == 0  # every arrival counter back at 0
 
 
-def test_split_k_matches_column_split_closely(monkeypatch):
+def test_split_k_matches_column_split_closely():
     # K halves and column halves sum the same products in different orders:
     # both within tolerance, and equal in most elements
-    monkeypatch.setenv("KREX_GEMM_SPLIT_K", "1")
+    krex.krex_set_tuning(gemm_split_k=1)
     M, N, K = 1536, 1536, 3072
     a, b = _gen(2, M, N, K)
     c0 = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
@@ -345,8 +349,8 @@ def _within_tol16(got_bits, want64, K):
 
 
 @pytest.mark.parametrize("ksub", ["2", "1"])
-def test_f16_identity_and_permutation_are_exact(ksub, monkeypatch):
-    monkeypatch.setenv("KREX_GEMM_KSUB", ksub)
+def test_f16_identity_and_permutation_are_exact(ksub):
+    krex.krex_set_tuning(gemm_stage_k=64 if ksub == "1" else 128)
     a, _ = _gen16(1, 256, 384, 384)
     eye = to_f16_tensor(gen.f32_to_f16(inputs.identity(384).ravel()).reshape(384, 384))
     assert np.array_equal(bits16(_candidate16(a, eye)), bits16(a))
@@ -369,8 +373,8 @@ def test_f16_small_integers_are_exact():
 
 @pytest.mark.parametrize("M,N,K", [(128, 256, 64), (100, 72, 40), (300, 1000, 520), (1024, 2048, 512),
                                    (640, 384, 4104), (2064, 1000, 1032), (4096, 4096, 4096)])
-def test_f16_seeded_gemm_within_tolerance(M, N, K, monkeypatch):
-    monkeypatch.setenv("KREX_GEMM_SPLIT_K", "1")
+def test_f16_seeded_gemm_within_tolerance(M, N, K):
+    krex.krex_set_tuning(gemm_split_k=1)
     seed = 7000 + M + N + K
     a, b = _gen16(seed, M, N, K)
     want = ref.gemm_f64(gen.uniform_f16(seed, 0, M, K), gen.uniform_f16(seed, 1, K, N), dtype="f16")
@@ -417,7 +421,7 @@ def test_f16_op_rejects_bf16_operands():
 
 @pytest.mark.parametrize("f16", [False, True], ids=["bf16", "f16"])
 @pytest.mark.parametrize("tile", ["0", "1", "2", "3", "4", "5"])
-def test_reference_tilings_are_bit_identical(tile, f16, monkeypatch):
+def test_reference_tilings_are_bit_identical(tile, f16):
     # every output of the reference is one fp32 FMA chain in k order, so the
     # tiling (5: one output per thread, the small-GEMM form) must not change a
     # bit (ragged shape: partial tiles in M, N, K)
@@ -425,11 +429,30 @@ def test_reference_tilings_are_bit_identical(tile, f16, monkeypatch):
     a, b = _gen16(99, M, N, K) if f16 else _gen(99, M, N, K)
     op = krex.KREX_OP_GEMM_F16 if f16 else krex.KREX_OP_GEMM_BF16
     r0 = torch.empty(M, N, dtype=torch.float32, device="cuda")
-    monkeypatch.setenv("KREX_REF_TILE", "0")
+    krex.krex_set_tuning(reference_tiling=0)
     krex.krex_run_reference(op, [a, b], r0)
     r = Guarded(M, N, torch.float32)
-    monkeypatch.setenv("KREX_REF_TILE", tile)
+    krex.krex_set_tuning(reference_tiling=int(tile))
     krex.krex_run_reference(op, [a, b], r.view)
     torch.cuda.synchronize()
     assert r.canaries_intact()
     assert torch.equal(r.view.contiguous().view(torch.int32), r0.view(torch.int32))
+
+
+@pytest.mark.parametrize("f16", [False, True], ids=["bf16", "f16"])
+def test_reference_unchecked_form_equals_checked_form(f16):
+    # a GEMM whose tiles and K slices all lie inside the matrices runs the
+    # reference without bounds checks; the same operands with an odd row
+    # stride of A (no 16-byte loads) take the checked form: identical bits
+    M, N, K = 512, 768, 1024
+    a, b = _gen16(77, M, N, K) if f16 else _gen(77, M, N, K)
+    op = krex.KREX_OP_GEMM_F16 if f16 else krex.KREX_OP_GEMM_BF16
+    r_in = torch.empty(M, N, dtype=torch.float32, device="cuda")
+    krex.krex_run_reference(op, [a, b], r_in)
+    wide = torch.zeros(M, K + 3, dtype=a.dtype, device="cuda")
+    wide[:, :K] = a
+    r_chk = Guarded(M, N, torch.float32)
+    krex.krex_run_reference(op, [wide[:, :K], b], r_chk.view)
+    torch.cuda.synchronize()
+    assert r_chk.canaries_intact()
+    assert torch.equal(r_chk.view.contiguous().view(torch.int32), r_in.view(torch.int32))
