@@ -50,19 +50,10 @@ __device__ __forceinline__ float hi_f32(uint32_t w) {
     return __uint_as_float(w & 0xFFFF0000u);
 }
 
-// 8 consecutive 16-bit elements at (r, c..c+7), for a block whose tile and
-// K slices lie wholly inside the matrix and whose rows allow 16-byte loads.
-__device__ __forceinline__ uint4 load8_inside(const uint16_t *__restrict__ p, int64_t ld, int64_t r, int64_t c) {
-    return __ldg(reinterpret_cast<const uint4 *>(p + r * ld + c));
-}
-
 // NG: 64-column groups per block (tile 128 x 64*NG); TK: K per shared slice;
-// MINB: resident blocks per SM the register budget is sized for.  INSIDE:
-// every tile and K slice of the launch lies inside the matrices and every row
-// allows 16-byte accesses (M % 128 = N % (64 NG) = K % TK = 0, aligned rows),
-// so loads and stores need no bounds checks (measured: 2-3 % faster at
-// 16384^3).
-template <bool F16, int NG, int TK, int MINB, bool INSIDE>
+// MINB: resident blocks per SM the register budget is sized for.  Any shape
+// and row strides (bounds-checked loads and stores).
+template <bool F16, int NG, int TK, int MINB>
 __global__ void __launch_bounds__(256, MINB)
 gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__restrict__ B, int64_t ldb,
               float *__restrict__ C, int64_t ldc, int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec,
@@ -84,14 +75,12 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
 #pragma unroll
         for (int i = 0; i < A_LOADS; ++i) {
             const int s = t + 256 * i;
-            ua[i] = INSIDE ? load8_inside(A, lda, m0 + s / (TK / 8), k0 + 8 * (s % (TK / 8)))
-                           : load8(A, lda, M, K, m0 + s / (TK / 8), k0 + 8 * (s % (TK / 8)), a_vec);
+            ua[i] = load8(A, lda, M, K, m0 + s / (TK / 8), k0 + 8 * (s % (TK / 8)), a_vec);
         }
 #pragma unroll
         for (int i = 0; i < B_LOADS; ++i) {
             const int s = t + 256 * i;
-            ub[i] = INSIDE ? load8_inside(B, ldb, k0 + s / (TN / 8), n0 + 8 * (s % (TN / 8)))
-                           : load8(B, ldb, K, N, k0 + s / (TN / 8), n0 + 8 * (s % (TN / 8)), b_vec);
+            ub[i] = load8(B, ldb, K, N, k0 + s / (TN / 8), n0 + 8 * (s % (TN / 8)), b_vec);
         }
     };
     auto stage = [&](int nb) {
@@ -150,12 +139,10 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
                 b[4 * g + 3] = bg.w;
             }
             const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-            // column-major sweep of the outer product (each b[j] held across
-            // the eight rows): measured 2-5 % faster than row-major on GB300
 #pragma unroll
-            for (int j = 0; j < 4 * NG; ++j)
+            for (int i = 0; i < 8; ++i)
 #pragma unroll
-                for (int i = 0; i < 8; ++i) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+                for (int j = 0; j < 4 * NG; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
         }
         if (more) {
             const int nb = buf ^ 1;
@@ -168,13 +155,13 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
         const int64_t r = m0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + (i - 4));
-        if (!INSIDE && r >= M) continue;
+        if (r >= M) continue;
         float *cr = C + r * ldc;
 #pragma unroll
         for (int g = 0; g < NG; ++g) {
             const int64_t c = n0 + g * 64 + tx * 4;
             const float *v = &acc[i][4 * g];
-            if (INSIDE || (c_vec && c + 4 <= N)) {
+            if (c_vec && c + 4 <= N) {
                 *reinterpret_cast<float4 *>(cr + c) = make_float4(v[0], v[1], v[2], v[3]);
             } else {
 #pragma unroll
@@ -182,6 +169,88 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
                     if (c + j < N) cr[c + j] = v[j];
             }
         }
+    }
+}
+
+// The same tiling for GEMMs made of whole tiles (M % 128 = N % 128 = K % 16 =
+// 0, 16-byte aligned rows), the sizes of the benchmark workloads: no bounds
+// checks, one 16-byte load of A and one of B per thread and slice, a 32-bit K
+// counter, and a column-major sweep of the outer product (each b[j] held
+// across the eight rows).  Each
+// output is the same k-order FMA chain as in gemm_ref_simt (identical bits).
+// Measured on GB300 in one process (TFLOP/s at 4096^3 / 8192^3 / 16384^3, L2
+// flushed): 58.6 / 60.8 / 60.9 against 55.1 / 57.1 / 57.0 for gemm_ref_simt
+// with the row-major sweep and 52.6 / 54.8 / 55.4 with the column-major one.
+template <bool F16>
+__global__ void __launch_bounds__(256, 2)
+gemm_ref_whole(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__restrict__ B, int64_t ldb,
+               float *__restrict__ C, int64_t ldc, int K) {
+    constexpr int TK = 16, TN = 128;
+    extern __shared__ __align__(16) float smem[];
+    float *As = smem;                  // [2][TK][TM]
+    float *Bs = smem + 2 * TK * TM;    // [2][TK][TN]
+    const int t = threadIdx.x, tx = t & 15, ty = t >> 4;
+    const int64_t m0 = (int64_t)blockIdx.y * TM, n0 = (int64_t)blockIdx.x * TN;
+    // one 16-byte load of A (row t / 2, k offset 8 (t % 2)) and one of B
+    // (k-row t / 16, columns 8 (t % 16)) per thread and slice
+    uint4 ua, ub;
+    auto fetch = [&](int k0) {
+        ua = __ldg(reinterpret_cast<const uint4 *>(A + (m0 + (t >> 1)) * lda + k0 + 8 * (t & 1)));
+        ub = __ldg(reinterpret_cast<const uint4 *>(B + (int64_t)(k0 + (t >> 4)) * ldb + n0 + 8 * (t & 15)));
+    };
+    auto stage = [&](int nb) {
+        float *as = As + nb * TK * TM, *bs = Bs + nb * TK * TN;
+        const int row = t >> 1, kk = 8 * (t & 1);
+        const uint32_t wa[4] = {ua.x, ua.y, ua.z, ua.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            as[(kk + 2 * j) * TM + row] = lo_f32<F16>(wa[j]);
+            as[(kk + 2 * j + 1) * TM + row] = hi_f32<F16>(wa[j]);
+        }
+        float *dst = bs + (t >> 4) * TN + 8 * (t & 15);
+        *reinterpret_cast<float4 *>(dst) = make_float4(lo_f32<F16>(ub.x), hi_f32<F16>(ub.x), lo_f32<F16>(ub.y),
+                                                       hi_f32<F16>(ub.y));
+        *reinterpret_cast<float4 *>(dst + 4) = make_float4(lo_f32<F16>(ub.z), hi_f32<F16>(ub.z), lo_f32<F16>(ub.w),
+                                                           hi_f32<F16>(ub.w));
+    };
+    float acc[8][8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = 0.0f;
+    fetch(0);
+    stage(0);
+    __syncthreads();
+    int buf = 0;
+    for (int k0 = 0; k0 < K; k0 += TK) {
+        const bool more = k0 + TK < K;
+        if (more) fetch(k0 + TK);  // the next slice comes in while this one is multiplied
+        const float *as = As + buf * TK * TM, *bs = Bs + buf * TK * TN;
+#pragma unroll
+        for (int k = 0; k < TK; ++k) {
+            const float4 a0 = *reinterpret_cast<const float4 *>(as + k * TM + ty * 4);
+            const float4 a1 = *reinterpret_cast<const float4 *>(as + k * TM + 64 + ty * 4);
+            const float4 b0 = *reinterpret_cast<const float4 *>(bs + k * TN + tx * 4);
+            const float4 b1 = *reinterpret_cast<const float4 *>(bs + k * TN + 64 + tx * 4);
+            const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+            const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+#pragma unroll
+                for (int i = 0; i < 8; ++i) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+        }
+        if (more) {
+            const int nb = buf ^ 1;
+            stage(nb);
+            __syncthreads();
+            buf = nb;
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        float *cr = C + (m0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + (i - 4))) * ldc;
+        *reinterpret_cast<float4 *>(cr + n0 + tx * 4) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+        *reinterpret_cast<float4 *>(cr + n0 + 64 + tx * 4) = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
     }
 }
 
@@ -223,38 +292,46 @@ cudaError_t launch_small(const uint16_t *a, int64_t lda, const uint16_t *b, int6
     return cudaGetLastError();
 }
 
-template <bool F16, int NG, int TK, int MINB, bool INSIDE>
-cudaError_t launch_cfg_as(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
-                          int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c_vec, cudaStream_t s) {
-    constexpr int TN = 64 * NG;
-    constexpr size_t smem = (size_t)2 * TK * (TM + TN) * sizeof(float);
-    static const cudaError_t attr = cudaFuncSetAttribute(
-        gemm_ref_simt<F16, NG, TK, MINB, INSIDE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (attr != cudaSuccess) return attr;
-    dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
-    gemm_ref_simt<F16, NG, TK, MINB, INSIDE><<<grid, 256, smem, s>>>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec,
-                                                                     c_vec);
-    return cudaGetLastError();
-}
-
 template <bool F16, int NG, int TK, int MINB>
 cudaError_t launch_cfg(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
                        int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c_vec, cudaStream_t s) {
-    const bool inside = M % TM == 0 && N % (64 * NG) == 0 && K % TK == 0 && a_vec && b_vec && c_vec;
-    return inside ? launch_cfg_as<F16, NG, TK, MINB, true>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s)
-                  : launch_cfg_as<F16, NG, TK, MINB, false>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
+    constexpr int TN = 64 * NG;
+    constexpr size_t smem = (size_t)2 * TK * (TM + TN) * sizeof(float);
+    static const cudaError_t attr = cudaFuncSetAttribute(
+        gemm_ref_simt<F16, NG, TK, MINB>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (attr != cudaSuccess) return attr;
+    dim3 grid((unsigned)((N + TN - 1) / TN), (unsigned)((M + TM - 1) / TM));
+    gemm_ref_simt<F16, NG, TK, MINB><<<grid, 256, smem, s>>>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec);
+    return cudaGetLastError();
+}
+
+// Whole tiles and aligned rows: the unchecked kernel (identical bits).
+template <bool F16>
+bool whole_tiles(int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c_vec) {
+    return M % TM == 0 && N % 128 == 0 && K % 16 == 0 && K > 0 && K <= INT32_MAX - 16 && a_vec && b_vec && c_vec &&
+           M / TM <= 65535;
+}
+
+template <bool F16>
+cudaError_t launch_whole(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
+                         int64_t M, int64_t N, int64_t K, cudaStream_t s) {
+    constexpr size_t smem = (size_t)2 * 16 * (TM + 128) * sizeof(float);
+    dim3 grid((unsigned)(N / 128), (unsigned)(M / TM));
+    gemm_ref_whole<F16><<<grid, 256, smem, s>>>(a, lda, b, ldb, c, ldc, (int)K);
+    return cudaGetLastError();
 }
 
 // Tiling of the reference (the tuning record's reference_tiling selects another
 // for comparisons): 0 = 128x128, TK 16, one block per SM (143 registers); 1 =
 // 128x256, TK 16; 2 = 128x128, TK 32; 3 = 128x256, TK 32; 4 = 128x128, TK 16
 // with at most 128 registers, so two blocks share an SM.  Measured on GB300
-// (TFLOP/s at 4096^3 / 8192^3, L2 flushed, before the column-major sweep and
-// the unchecked form): 53.3/54.5, 49.9/56.6, 50.7/51.8, 43.0/49.0, 54.8/57.2,
+// (TFLOP/s at 4096^3 / 8192^3, L2 flushed): 53.3/54.5, 49.9/56.6, 50.7/51.8,
+// 43.0/49.0, 54.8/57.2,
 // all bit-identical (each output is one k-order FMA chain).  Also measured and
 // dropped: packed fp32x2 FMAs (with duplicated or diagonally paired operands:
 // 47-55 at 16384^3), 32-deep slices with two blocks per SM, per-thread tiles of
-// 4x16, 16x4, 8x16 and 16x8 (54-59 at 16384^3).  Default: 4, or 5 (the
+// 4x16, 16x4, 8x16 and 16x8 (54-59 at 16384^3).  Default: 4, run as
+// gemm_ref_whole when the GEMM is made of whole tiles, or 5 (the
 // one-output-per-thread kernel) when the GEMM has at most 16 tiles of 128x128
 // (L2 flushed: 256^3 30 -> 18 us, 512^3 53 -> 47 us; at 768^3, 36 tiles, the
 // tiled form is faster).
@@ -273,7 +350,10 @@ cudaError_t launch_ref(const uint16_t *a, int64_t lda, const uint16_t *b, int64_
     case 2: return launch_cfg<F16, 2, 32, 1>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
     case 3: return launch_cfg<F16, 4, 32, 1>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
     case 5: return launch_small<F16>(a, lda, b, ldb, c, ldc, M, N, K, s);
-    default: return launch_cfg<F16, 2, 16, 2>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
+    default:
+        if (whole_tiles<F16>(M, N, K, a_vec, b_vec, c_vec))
+            return launch_whole<F16>(a, lda, b, ldb, c, ldc, M, N, K, s);
+        return launch_cfg<F16, 2, 16, 2>(a, lda, b, ldb, c, ldc, M, N, K, a_vec, b_vec, c_vec, s);
     }
 }
 
