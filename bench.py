@@ -49,14 +49,8 @@ CONFIG_WORKLOADS = {"gemm_bf16_256": 32, "gemm_bf16_4096": 20, "softmax_f32_6553
                     "gemm_bf16_8192": 8, "gemm_bf16_16384": 32}
 SOFTMAX_WORKLOAD = "softmax_f32_65536x8192"
 SMALL_GEMM_WORKLOAD = "gemm_bf16_4096"
-# 32-bit integer-ALU operations the uniform generator's definition takes per
-# 16-bit element: per SplitMix64 draw (two elements) a 64-bit add (2) and three
-# 64-bit xor-shifts (2 funnel shifts + 2 xors each: 12); per element the 24-bit
-# field to [-1, 1) (a shift, two masks, an integer subtract: 4).  The two 64-bit
-# multiplies per draw (3 multiply-adds each) run on the multiply-add pipe and
-# are counted separately (FILL_IMAD_OPS_PER_ELEMENT).
-FILL_ALU_OPS_PER_ELEMENT = (2 + 12) / 2 + 4
-FILL_IMAD_OPS_PER_ELEMENT = (2 * 3) / 2
+# Output bytes per SplitMix64 draw: two bf16 (uniform) or two fp32 (normal).
+DRAW_BYTES = {0: 4, 1: 8}
 # FP32 fused multiply-add lanes per SM (the CUDA-core reference GEMM's pipe)
 FMA_LANES_PER_SM = 128
 
@@ -177,11 +171,11 @@ def kernel_table(peaks, stream, gemm_names=(DEFAULT_WORKLOAD, SMALL_GEMM_WORKLOA
     out = {}
     dev = torch.cuda.current_device()
     n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
-    # integer-ALU roofline of the uniform fill: 64 ALU lanes per clock per SM
-    # at the 2070 MHz maximum SM clock (the clock the runs see under load)
-    alu_peak = n_sm * 64 * 2.070e9
+    ceiling = {d: generator_ceiling(d, n_sm, stream) for d in (0, 1)}
+    out["generator_probe_uniform"] = ceiling[0]
+    out["generator_probe_normal"] = ceiling[1]
 
-    def rec(name, fn, flush, nbytes=None, flops=None, alu_ops=None, n=20, fma_peak=None):
+    def rec(name, fn, flush, nbytes=None, flops=None, gen_dist=None, n=20, fma_peak=None):
         for _ in range(3):
             fn()
         ms = _time_launches(fn, n, stream, flush)
@@ -196,9 +190,11 @@ def kernel_table(peaks, stream, gemm_names=(DEFAULT_WORKLOAD, SMALL_GEMM_WORKLOA
                 e["frac_bf16"] = tf / peaks["bf16_tflops"]
             else:
                 e.update({"bound": "fp32 fma", "frac_fma": tf * 1e12 / fma_peak})
-        if alu_ops is not None:
-            e.update({"bound": "alu", "alu_ops": alu_ops, "Tops/s": alu_ops / ms / 1e9,
-                      "frac_alu": alu_ops / ms * 1e3 / alu_peak})
+        if gen_dist is not None:
+            # compute-bound generator: its roofline is the measured rate of
+            # its own per-draw arithmetic (generator_ceiling)
+            c = ceiling[gen_dist]["GB/s"]
+            e.update({"bound": "alu", "peak_GB/s": c, "frac_alu": (nbytes / ms / 1e6) / c})
         out[name] = e
 
     for gname in gemm_names:
@@ -208,7 +204,7 @@ def kernel_table(peaks, stream, gemm_names=(DEFAULT_WORKLOAD, SMALL_GEMM_WORKLOA
         flush = lambda ws=ws: krex.krex_flush_l2(ws.flush, stream=stream)  # noqa: E731
         A, B = ws.inputs
         rec("fill_uniform_bf16" + sfx, lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, A, stream), flush,
-            nbytes=A.numel() * 2, alu_ops=A.numel() * FILL_ALU_OPS_PER_ELEMENT, n=10)
+            nbytes=A.numel() * 2, gen_dist=0, n=10)
         krex.krex_gen_inputs(w.seed, 1, 0, 0.0, B, stream)
         if gname == gemm_names[0]:
             rec("flush_l2", flush, None, nbytes=ws.flush.numel())
@@ -227,7 +223,7 @@ def kernel_table(peaks, stream, gemm_names=(DEFAULT_WORKLOAD, SMALL_GEMM_WORKLOA
     flush = lambda: krex.krex_flush_l2(sws.flush, stream=stream)  # noqa: E731
     x, y = sws.inputs[0], sws.out
     rec("fill_normal_f32", lambda: krex.krex_gen_inputs(sw.seed, 0, 1, sw.sigma, x, stream), flush,
-        nbytes=x.numel() * 4, n=10)
+        nbytes=x.numel() * 4, gen_dist=1, n=10)
     rec("softmax_f32", lambda: krex.krex_run_candidate(1, [x], y, stream), flush, nbytes=x.numel() * 8, n=10)
     rec("check_f32_f32", lambda: krex.krex_check_launch(y, x, 1e-6, 0.0, sws.check_scratch, stream), flush,
         nbytes=x.numel() * 8, n=5)
@@ -238,13 +234,32 @@ def kernel_table(peaks, stream, gemm_names=(DEFAULT_WORKLOAD, SMALL_GEMM_WORKLOA
     flush = lambda: krex.krex_flush_l2(fws.flush, stream=stream)  # noqa: E731
     a16, b16 = fws.inputs
     rec("fill_uniform_f16@4096", lambda: krex.krex_gen_inputs(fw.seed, 0, 0, 0.0, a16, stream), flush,
-        nbytes=a16.numel() * 2, alu_ops=a16.numel() * FILL_ALU_OPS_PER_ELEMENT)
+        nbytes=a16.numel() * 2)
     krex.krex_gen_inputs(fw.seed, 1, 0, 0.0, b16, stream)
     rec("gemm_tcgen05_f16@4096", lambda: krex.krex_run_candidate_ws(fw.op, fws.inputs, fws.out, fws.gemm_ws, stream),
         flush, flops=fw.flops)
     del fws, a16, b16
     torch.cuda.empty_cache()
     return out
+
+
+def generator_ceiling(dist: int, n_sm: int, stream, draws_total: int = 1 << 27) -> dict:
+    """The rate at which this GPU computes SplitMix64 draws of one generator
+    (uniform: dist 0, normal: dist 1), measured with the library's probe (the
+    fills' per-draw arithmetic without stores) on the fills' residency (8
+    blocks of 256 threads per SM), as output GB/s: the fills' compute roofline."""
+    import torch
+    import paper_2609_30057_gb300 as krex
+    blocks = n_sm * 8
+    per_thread = max(4, (draws_total // (blocks * 256)) // 4 * 4)
+    sink = torch.empty(blocks * 256, dtype=torch.int32, device="cuda")
+    fn = lambda: krex.krex_probe_generator(dist, per_thread, blocks, sink, stream=stream)  # noqa: E731
+    for _ in range(3):
+        fn()
+    ms = _time_launches(fn, 10, stream)
+    draws = blocks * 256 * per_thread
+    return {"ms": ms, "draws": draws, "Gdraws/s": draws / ms / 1e6,
+            "GB/s": draws * DRAW_BYTES[dist] / ms / 1e6, "blocks": blocks, "draws_per_thread": per_thread}
 
 
 # ---------------------------------------------------------- CPU oracle ------

@@ -450,6 +450,21 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
                              const void *const *host_in, void *host_out, float *durations_ms,
                              krex_command_result *result, krex_stream_t stream);
 
+/* ------------------------------------------------------ measurement ----- */
+
+/* Measurement probe, not part of the paper's method: runs the per-draw
+ * arithmetic of a seeded generator (dist as in krex_gen_inputs; the uniform
+ * one in its bf16 form) on `blocks` blocks of 256 threads, `draws_per_thread`
+ * draws each (a positive multiple of 4), storing nothing but what keeps the
+ * arithmetic live, so that timing it gives the rate at which the GPU computes
+ * draws: the compute ceiling of the fill kernels, whose outputs are 2 bf16
+ * (uniform) or 2 fp32 (normal) per draw.  dev_sink: device memory of at least
+ * blocks * 256 * 4 bytes (its contents afterwards are unspecified).
+ * Asynchronous.  Errors: INVALID for a bad dist, a null sink, blocks < 1 or
+ * draws_per_thread not a positive multiple of 4. */
+krex_status krex_probe_generator(int32_t dist, uint64_t draws_per_thread, int32_t blocks, float sigma,
+                                 void *dev_sink, krex_stream_t stream);
+
 /* ------------------------------------------------------------ tuning ----- */
 
 /* The kernels' launch configuration, process-wide.  The library never reads

@@ -112,6 +112,7 @@ SIGNATURES = {
     "krex_set_tuning": (_i32, [_P(krex_tuning)]),
     "krex_get_tuning": (_i32, [_P(krex_tuning)]),
     "krex_debug_stall_handover": (_i32, [_i32]),
+    "krex_probe_generator": (_i32, [_i32, _u64, _i32, _f32, _vp, _vp]),
     "krex_gate_shared_bytes": (_sz, [_i32]),
     "krex_gate_shared_init": (_i32, [_vp, _sz, _i32]),
     "krex_gate_shared_attach": (_i32, [_vp, _sz, _P(_vp)]),
@@ -472,6 +473,13 @@ class tuning:
 
     def __exit__(self, *exc):
         krex_set_tuning(**self.saved)
+
+
+def krex_probe_generator(dist: int, draws_per_thread: int, blocks: int, sink, sigma: float = 2.0, stream=None):
+    """Launch the generator-arithmetic probe (asynchronous); sink: a device
+    tensor of at least blocks * 256 * 4 bytes."""
+    _ok(lib().krex_probe_generator(dist, draws_per_thread, blocks, sigma, sink.data_ptr(), _stream(stream)),
+        "krex_probe_generator")
 
 
 def krex_debug_stall_handover(on: bool) -> None:

@@ -783,6 +783,19 @@ static void CUDART_CB hold_fn(void *p) {
     delete a;
 }
 
+krex_status krex_probe_generator(int32_t dist, uint64_t draws_per_thread, int32_t blocks, float sigma,
+                                 void *dev_sink, krex_stream_t stream) {
+    if (dist != KREX_DIST_UNIFORM_PM1 && dist != KREX_DIST_NORMAL)
+        return set_error(KREX_ERR_INVALID, "probe: bad distribution %d", dist);
+    if (!dev_sink || blocks < 1 || draws_per_thread == 0 || draws_per_thread % 4 ||
+        draws_per_thread > ((uint64_t)1 << 40))
+        return set_error(KREX_ERR_INVALID, "probe: need a sink, blocks >= 1, draws a positive multiple of 4");
+    KREX_CUDA_TRY(launch_generator_probe(dist, 0x243F6A8885A308D3ull, (int64_t)draws_per_thread, sigma, blocks,
+                                         static_cast<uint32_t *>(dev_sink), reinterpret_cast<cudaStream_t>(stream)));
+    count_launches(1);
+    return ok();
+}
+
 void krex_tuning_defaults(krex_tuning *t) {
     if (t) *t = default_tuning();
 }

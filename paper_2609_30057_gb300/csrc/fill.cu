@@ -36,21 +36,34 @@ __device__ __forceinline__ uint64_t mix64(uint64_t z) {
 
 // ---------------------------------------------------------------- uniform --
 
-// 24-bit b -> (b - 2^23) 2^-23 exactly: 1.m with the low 23 bits of b, minus
-// 2 (bit 23 clear) or 1 (bit 23 set).  Both subtractions are exact.
-__device__ __forceinline__ float u24_to_pm1(uint32_t b) {
-    float f = __uint_as_float(0x3F800000u | (b & 0x7FFFFFu));
-    float sub = __uint_as_float(0x40000000u - (b & 0x800000u));
-    return __fsub_rn(f, sub);
+// Draw j's two 24-bit fields, each in bits 31..8 of a word with the low byte
+// clear: bits 63..40 of z_j (element 2j) and bits 31..8 (element 2j+1), from
+// the draw's state s = key + (j+1) G.  The last step of mix64 (z ^= z >> 31)
+// changes only bit 0 of the high word, and xors the high word shifted left by
+// one (plus one bit into bit 0) into the low word; so bits 31..8 of the final
+// words are those of hi and of lo ^ (hi << 1) before that step.
+__device__ __forceinline__ void draw_fields(uint64_t s, uint32_t &wh, uint32_t &wl) {
+    uint64_t z = (s ^ (s >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    const uint32_t hi = (uint32_t)(z >> 32), lo = (uint32_t)z;
+    wh = hi & 0xFFFFFF00u;
+    wl = (lo ^ (hi << 1)) & 0xFFFFFF00u;
 }
 
-// Elements 2j (low half) and 2j+1 (high half) from draw z_j, rounded to
-// bf16 or (F16) to IEEE binary16, both round-to-nearest-even.
+// A field w = b 2^8 (b its 24-bit value) -> (b - 2^23) 2^-23, exactly: w
+// converts to fp32 without rounding (24 significant bits), and w 2^-31 - 1 =
+// (b - 2^23) 2^-23 is representable, so the fused multiply-add is exact.
+__device__ __forceinline__ float field_to_pm1(uint32_t w) {
+    return __fmaf_rn(__uint2float_rn(w), 0x1p-31f, -1.0f);
+}
+
+// Elements 2j (low half) and 2j+1 (high half) from the state of draw j,
+// rounded to bf16 or (F16) to IEEE binary16, both round-to-nearest-even.
 template <bool F16>
-__device__ __forceinline__ uint32_t uniform_16x2(uint64_t z) {
-    uint32_t hi = (uint32_t)(z >> 32), lo = (uint32_t)z;
-    float x0 = u24_to_pm1(hi >> 8);
-    float x1 = u24_to_pm1(lo >> 8);
+__device__ __forceinline__ uint32_t uniform_16x2(uint64_t s) {
+    uint32_t wh, wl;
+    draw_fields(s, wh, wl);
+    const float x0 = field_to_pm1(wh), x1 = field_to_pm1(wl);
     if constexpr (F16) {
         __half2 h = __floats2half2_rn(x0, x1);
         return *reinterpret_cast<uint32_t *>(&h);
@@ -62,7 +75,7 @@ __device__ __forceinline__ uint32_t uniform_16x2(uint64_t z) {
 
 template <bool F16>
 __device__ __forceinline__ uint16_t uniform_16_at(uint64_t key, uint64_t e) {
-    uint32_t p = uniform_16x2<F16>(mix64(key + ((e >> 1) + 1ull) * kGamma));
+    uint32_t p = uniform_16x2<F16>(key + ((e >> 1) + 1ull) * kGamma);
     return (uint16_t)((e & 1ull) ? (p >> 16) : (p & 0xFFFFu));
 }
 
@@ -81,13 +94,13 @@ fill_uniform_16_vec(uint64_t key, uint16_t *__restrict__ out, int64_t rows, int6
         for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < groups; g += stride) {
             uint64_t s = key + (((e_row + (uint64_t)(g << 3)) >> 1) + 1ull) * kGamma;
             uint4 v;
-            v.x = uniform_16x2<F16>(mix64(s));
+            v.x = uniform_16x2<F16>(s);
             s += kGamma;
-            v.y = uniform_16x2<F16>(mix64(s));
+            v.y = uniform_16x2<F16>(s);
             s += kGamma;
-            v.z = uniform_16x2<F16>(mix64(s));
+            v.z = uniform_16x2<F16>(s);
             s += kGamma;
-            v.w = uniform_16x2<F16>(mix64(s));
+            v.w = uniform_16x2<F16>(s);
             *reinterpret_cast<uint4 *>(row + (g << 3)) = v;
         }
         if (blockIdx.x == 0 && threadIdx.x == 0) {
@@ -203,6 +216,33 @@ fill_normal_f32_vec(uint64_t key, float sigma, float *__restrict__ out, int64_t 
     }
 }
 
+// Measurement probe: the generators' per-draw arithmetic (the same device
+// functions as the fill kernels) with no stores, to measure the rate at which
+// this GPU can compute draws.  Each thread runs `draws` consecutive draws of
+// its own stretch of the stream and folds every result into one word, which
+// it stores only if it equals a value no fold produces in practice (the store
+// keeps the arithmetic live; `sink` must hold one word per thread anyway).
+template <int DIST>
+__global__ void __launch_bounds__(256)
+generator_probe(uint64_t key, int64_t draws, float sigma, uint32_t *sink) {
+    const uint64_t t = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    uint64_t s = key + (t * (uint64_t)draws + 1ull) * kGamma;
+    uint32_t acc = 0;
+    for (int64_t i = 0; i < draws; i += 4) {
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if constexpr (DIST == KREX_DIST_UNIFORM_PM1) {
+                acc ^= uniform_16x2<false>(s);
+            } else {
+                const float2 p = normal_pair(mix64(s), sigma);
+                acc ^= __float_as_uint(p.x) ^ (__float_as_uint(p.y) << 1);
+            }
+            s += kGamma;
+        }
+    }
+    if (acc == 0x5EED5EEDu) sink[t] = acc;
+}
+
 // Any layout: one element per thread step (each element recomputes its draw).
 template <bool F16>
 __global__ void __launch_bounds__(256)
@@ -262,6 +302,15 @@ void launch_uniform(uint64_t key, uint16_t *p, bool aligned, int64_t rows, int64
 }
 
 }  // namespace
+
+cudaError_t launch_generator_probe(int32_t dist, uint64_t key, int64_t draws, float sigma, int blocks,
+                                   uint32_t *sink, cudaStream_t s) {
+    if (dist == KREX_DIST_UNIFORM_PM1)
+        generator_probe<KREX_DIST_UNIFORM_PM1><<<blocks, 256, 0, s>>>(key, draws, sigma, sink);
+    else
+        generator_probe<KREX_DIST_NORMAL><<<blocks, 256, 0, s>>>(key, draws, sigma, sink);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_fill_uniform_16(uint64_t key, bool f16, void *out, int64_t rows, int64_t cols,
                                    int64_t ld, cudaStream_t s) {

@@ -145,13 +145,17 @@ __device__ __forceinline__ void block_reduce_publish(Acc acc, CheckScratch *sc) 
     __syncthreads();
     if (!s_last) return;
     __threadfence();
-    // last block: combine all partials (exact max and sum)
+    // last block: combine all partials (exact max and sum).  The partials were
+    // published before their blocks' tickets (fence, then atomic), and this
+    // block has fenced after taking the last ticket, so L2 loads (which bypass
+    // L1) see them; being plain loads they can all be in flight at once.
     uint32_t bm = 0;
     unsigned long long bc = 0;
+#pragma unroll 4
     for (int b = threadIdx.x; b < (int)gridDim.x; b += blockDim.x) {
-        volatile Partial *p = &sc->partial[b];
-        bm = max(bm, p->max_bits);
-        bc += p->count;
+        const uint4 p = __ldcg(reinterpret_cast<const uint4 *>(&sc->partial[b]));
+        bm = max(bm, p.x);
+        bc += (unsigned long long)p.z | ((unsigned long long)p.w << 32);
     }
     bm = __reduce_max_sync(0xffffffffu, bm);
     for (int o = 16; o > 0; o >>= 1) bc += __shfl_xor_sync(0xffffffffu, bc, o);
@@ -197,10 +201,7 @@ check_16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref, 
     Acc acc;
     clear_done(sc);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < n8; g += stride) {
-        uint4 o = __ldcs(out + g);
-        float4 r0 = __ldcs(ref + 2 * g);
-        float4 r1 = __ldcs(ref + 2 * g + 1);
+    auto add8 = [&](const uint4 &o, const float4 &r0, const float4 &r1) {
         float f[8];
         x8_to_f32<T>(o, f);
         acc.add(f[0], r0.x, atol, rtol);
@@ -211,7 +212,17 @@ check_16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref, 
         acc.add(f[5], r1.y, atol, rtol);
         acc.add(f[6], r1.z, atol, rtol);
         acc.add(f[7], r1.w, atol, rtol);
+    };
+    int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    // two steps per pass, all six loads issued before either is used
+    for (; g + stride < n8; g += 2 * stride) {
+        const uint4 o0 = __ldcs(out + g), o1 = __ldcs(out + g + stride);
+        const float4 r00 = __ldcs(ref + 2 * g), r01 = __ldcs(ref + 2 * g + 1);
+        const float4 r10 = __ldcs(ref + 2 * (g + stride)), r11 = __ldcs(ref + 2 * (g + stride) + 1);
+        add8(o0, r00, r01);
+        add8(o1, r10, r11);
     }
+    for (; g < n8; g += stride) add8(__ldcs(out + g), __ldcs(ref + 2 * g), __ldcs(ref + 2 * g + 1));
     if (blockIdx.x == 0)
         for (int64_t i = n8 * 8 + threadIdx.x; i < n; i += blockDim.x)
             acc.add(widen(out_s, i), ref_s[i], atol, rtol);

@@ -184,3 +184,13 @@ def test_library_reads_no_environment_variables():
     for f in glob.glob(os.path.join(ROOT, "paper_2609_30057_gb300", "csrc", "*")):
         with open(f) as fh:
             assert "getenv" not in fh.read(), f
+
+
+def test_generator_probe_rejects_bad_arguments_before_any_launch():
+    import paper_2609_30057_gb300 as krex
+    lib = krex.lib()
+    assert lib.krex_probe_generator(7, 64, 1, 2.0, 16, None) == krex.KREX_ERR_INVALID      # bad distribution
+    assert lib.krex_probe_generator(0, 64, 1, 2.0, None, None) == krex.KREX_ERR_INVALID    # no sink
+    assert lib.krex_probe_generator(0, 62, 1, 2.0, 16, None) == krex.KREX_ERR_INVALID      # not a multiple of 4
+    assert lib.krex_probe_generator(1, 0, 1, 2.0, 16, None) == krex.KREX_ERR_INVALID       # no draws
+    assert lib.krex_probe_generator(1, 64, 0, 2.0, 16, None) == krex.KREX_ERR_INVALID      # no blocks

@@ -134,3 +134,15 @@ def test_empty_buffers_are_noops(rows, cols, dtype, dist):
     krex.krex_gen_inputs(1, 0, dist, 2.0, g.view)
     torch.cuda.synchronize()
     assert g.canaries_intact()
+
+
+@pytest.mark.parametrize("dist", [0, 1], ids=["uniform", "normal"])
+def test_generator_probe_runs_and_leaves_the_context_clean(dist):
+    # the measurement probe (the fills' per-draw arithmetic without stores)
+    # completes and reports no device error; its sink is only written on a
+    # fold value no run produces in practice
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    sink = torch.zeros(n_sm * 256, dtype=torch.int32, device="cuda")
+    krex.krex_probe_generator(dist, 64, n_sm, sink)
+    torch.cuda.synchronize()
+    assert krex.krex_device_status() == 0
