@@ -171,9 +171,11 @@ def kernel_table(peaks, stream, gemm_names=(DEFAULT_WORKLOAD, SMALL_GEMM_WORKLOA
     out = {}
     dev = torch.cuda.current_device()
     n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
-    ceiling = {d: generator_ceiling(d, n_sm, stream) for d in (0, 1)}
-    out["generator_probe_uniform"] = ceiling[0]
-    out["generator_probe_normal"] = ceiling[1]
+    # the fills' compute ceilings at the sizes they are timed at
+    ceiling = {0: generator_ceiling(0, n_sm, stream, 16384 * 16384),
+               1: generator_ceiling(1, n_sm, stream, WORKLOADS[SOFTMAX_WORKLOAD].M * WORKLOADS[SOFTMAX_WORKLOAD].N)}
+    out["generator_probe_uniform@16384"] = ceiling[0]
+    out["generator_probe_normal@65536x8192"] = ceiling[1]
 
     def rec(name, fn, flush, nbytes=None, flops=None, gen_dist=None, n=20, fma_peak=None):
         for _ in range(3):
@@ -243,23 +245,22 @@ def kernel_table(peaks, stream, gemm_names=(DEFAULT_WORKLOAD, SMALL_GEMM_WORKLOA
     return out
 
 
-def generator_ceiling(dist: int, n_sm: int, stream, draws_total: int = 1 << 27) -> dict:
-    """The rate at which this GPU computes SplitMix64 draws of one generator
-    (uniform: dist 0, normal: dist 1), measured with the library's probe (the
-    fills' per-draw arithmetic without stores) on the fills' residency (8
-    blocks of 256 threads per SM), as output GB/s: the fills' compute roofline."""
+def generator_ceiling(dist: int, n_sm: int, stream, n_elements: int) -> dict:
+    """The rate at which this GPU computes a generator (uniform: dist 0,
+    normal: dist 1), measured with the library's probe: the fill kernel's loop
+    over n_elements on the fills' residency (8 blocks of 256 threads per SM)
+    with folds instead of stores, as output GB/s: the fills' compute roofline."""
     import torch
     import paper_2609_30057_gb300 as krex
     blocks = n_sm * 8
-    per_thread = max(4, (draws_total // (blocks * 256)) // 4 * 4)
     sink = torch.empty(blocks * 256, dtype=torch.int32, device="cuda")
-    fn = lambda: krex.krex_probe_generator(dist, per_thread, blocks, sink, stream=stream)  # noqa: E731
+    fn = lambda: krex.krex_probe_generator(dist, n_elements, blocks, sink, stream=stream)  # noqa: E731
     for _ in range(3):
         fn()
     ms = _time_launches(fn, 10, stream)
-    draws = blocks * 256 * per_thread
-    return {"ms": ms, "draws": draws, "Gdraws/s": draws / ms / 1e6,
-            "GB/s": draws * DRAW_BYTES[dist] / ms / 1e6, "blocks": blocks, "draws_per_thread": per_thread}
+    draws = n_elements // 2
+    return {"ms": ms, "elements": n_elements, "Gdraws/s": draws / ms / 1e6,
+            "GB/s": draws * DRAW_BYTES[dist] / ms / 1e6, "blocks": blocks}
 
 
 # ---------------------------------------------------------- CPU oracle ------

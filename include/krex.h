@@ -452,18 +452,18 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
 
 /* ------------------------------------------------------ measurement ----- */
 
-/* Measurement probe, not part of the paper's method: runs the per-draw
- * arithmetic of a seeded generator (dist as in krex_gen_inputs; the uniform
- * one in its bf16 form) on `blocks` blocks of 256 threads, `draws_per_thread`
- * draws each (a positive multiple of 4), storing nothing but what keeps the
- * arithmetic live, so that timing it gives the rate at which the GPU computes
- * draws: the compute ceiling of the fill kernels, whose outputs are 2 bf16
- * (uniform) or 2 fp32 (normal) per draw.  dev_sink: device memory of at least
- * blocks * 256 * 4 bytes (its contents afterwards are unspecified).
- * Asynchronous.  Errors: INVALID for a bad dist, a null sink, blocks < 1 or
- * draws_per_thread not a positive multiple of 4. */
-krex_status krex_probe_generator(int32_t dist, uint64_t draws_per_thread, int32_t blocks, float sigma,
-                                 void *dev_sink, krex_stream_t stream);
+/* Measurement probe, not part of the paper's method: the fill kernel of a
+ * seeded generator (dist as in krex_gen_inputs; the uniform one in its bf16
+ * form) walking a contiguous buffer of n_elements elements on `blocks` blocks
+ * of 256 threads (the fills use 8 per SM), with each 16-byte group folded into
+ * a per-thread word instead of stored.  Timing it gives the rate at which the
+ * GPU computes the generator: the compute ceiling the fills are measured
+ * against (their outputs are 2 bf16 (uniform) or 2 fp32 (normal) per draw).
+ * dev_sink: device memory of at least blocks * 256 * 4 bytes (its contents
+ * afterwards are unspecified).  Asynchronous.  Errors: INVALID for a bad dist,
+ * a null sink, blocks < 1 or n_elements not a positive multiple of 8. */
+krex_status krex_probe_generator(int32_t dist, uint64_t n_elements, int32_t blocks, float sigma, void *dev_sink,
+                                 krex_stream_t stream);
 
 /* ------------------------------------------------------------ tuning ----- */
 
@@ -483,6 +483,9 @@ typedef struct {
     int32_t gemm_split_k;      /* split a single partial wave into K halves (needs the workspace of
                                   krex_run_candidate_ws): -1 = when K >= 4096 (default), 0 = never,
                                   1 = whenever the shape allows */
+    int32_t gemm_k_alternate;  /* walk K backwards on every other wave of pair tiles, so a wave starts on
+                                  the K blocks the previous one left in L2: -1 = yes (default), 0 = no,
+                                  1 = yes */
     int32_t reference_tiling;  /* the CUDA-core reference GEMM's tiling: -1 = by size (default); 0..5 as
                                   documented in gemm_ref.cu (all give identical bits) */
     int32_t wait_timeout_ms;   /* bound on every wait inside a kernel: 0 = 2000 ms; else 1..600000 */

@@ -47,7 +47,8 @@ class krex_tuning(ctypes.Structure):
     _fields_ = [("gemm_pair_tile_n", ctypes.c_int32), ("gemm_stage_k", ctypes.c_int32),
                 ("gemm_ring_stages", ctypes.c_int32), ("gemm_raster_group", ctypes.c_int32),
                 ("gemm_tail_split", ctypes.c_int32), ("gemm_split_k", ctypes.c_int32),
-                ("reference_tiling", ctypes.c_int32), ("wait_timeout_ms", ctypes.c_int32)]
+                ("gemm_k_alternate", ctypes.c_int32), ("reference_tiling", ctypes.c_int32),
+                ("wait_timeout_ms", ctypes.c_int32)]
 
 
 class krex_command(ctypes.Structure):
@@ -475,10 +476,11 @@ class tuning:
         krex_set_tuning(**self.saved)
 
 
-def krex_probe_generator(dist: int, draws_per_thread: int, blocks: int, sink, sigma: float = 2.0, stream=None):
-    """Launch the generator-arithmetic probe (asynchronous); sink: a device
-    tensor of at least blocks * 256 * 4 bytes."""
-    _ok(lib().krex_probe_generator(dist, draws_per_thread, blocks, sigma, sink.data_ptr(), _stream(stream)),
+def krex_probe_generator(dist: int, n_elements: int, blocks: int, sink, sigma: float = 2.0, stream=None):
+    """Launch the generator probe (asynchronous): the fill of `dist` over
+    n_elements with folds instead of stores; sink: a device tensor of at
+    least blocks * 256 * 4 bytes."""
+    _ok(lib().krex_probe_generator(dist, n_elements, blocks, sigma, sink.data_ptr(), _stream(stream)),
         "krex_probe_generator")
 
 

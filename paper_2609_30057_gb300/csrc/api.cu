@@ -89,6 +89,7 @@ krex_tuning default_tuning() {
     memset(&t, 0, sizeof(t));
     t.gemm_tail_split = -1;
     t.gemm_split_k = -1;
+    t.gemm_k_alternate = -1;
     t.reference_tiling = -1;
     return t;
 }
@@ -102,6 +103,7 @@ bool tuning_valid(const krex_tuning &t) {
             (t.gemm_ring_stages >= 2 && t.gemm_ring_stages <= (t.gemm_stage_k == 64 ? 6 : 3))) &&
            (t.gemm_raster_group >= 0 && t.gemm_raster_group <= 64) &&
            (t.gemm_tail_split >= -1 && t.gemm_tail_split <= 1) && (t.gemm_split_k >= -1 && t.gemm_split_k <= 1) &&
+           (t.gemm_k_alternate >= -1 && t.gemm_k_alternate <= 1) &&
            (t.reference_tiling >= -1 && t.reference_tiling <= 5) &&
            (t.wait_timeout_ms >= 0 && t.wait_timeout_ms <= 600000);
 }
@@ -783,14 +785,13 @@ static void CUDART_CB hold_fn(void *p) {
     delete a;
 }
 
-krex_status krex_probe_generator(int32_t dist, uint64_t draws_per_thread, int32_t blocks, float sigma,
-                                 void *dev_sink, krex_stream_t stream) {
+krex_status krex_probe_generator(int32_t dist, uint64_t n_elements, int32_t blocks, float sigma, void *dev_sink,
+                                 krex_stream_t stream) {
     if (dist != KREX_DIST_UNIFORM_PM1 && dist != KREX_DIST_NORMAL)
         return set_error(KREX_ERR_INVALID, "probe: bad distribution %d", dist);
-    if (!dev_sink || blocks < 1 || draws_per_thread == 0 || draws_per_thread % 4 ||
-        draws_per_thread > ((uint64_t)1 << 40))
-        return set_error(KREX_ERR_INVALID, "probe: need a sink, blocks >= 1, draws a positive multiple of 4");
-    KREX_CUDA_TRY(launch_generator_probe(dist, 0x243F6A8885A308D3ull, (int64_t)draws_per_thread, sigma, blocks,
+    if (!dev_sink || blocks < 1 || n_elements == 0 || n_elements % 8 || n_elements > ((uint64_t)1 << 50))
+        return set_error(KREX_ERR_INVALID, "probe: need a sink, blocks >= 1, n_elements a positive multiple of 8");
+    KREX_CUDA_TRY(launch_generator_probe(dist, 0x243F6A8885A308D3ull, (int64_t)n_elements, sigma, blocks,
                                          static_cast<uint32_t *>(dev_sink), reinterpret_cast<cudaStream_t>(stream)));
     count_launches(1);
     return ok();

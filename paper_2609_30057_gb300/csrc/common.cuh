@@ -23,10 +23,10 @@ cudaError_t launch_fill_uniform_16(uint64_t key, bool f16, void *out, int64_t ro
 // K2: SplitMix64 -> Box-Muller -> N(0, sigma^2) fp32, 16-byte stores.
 cudaError_t launch_fill_normal_f32(uint64_t key, float sigma, float *out, int64_t rows,
                                    int64_t cols, int64_t ld, cudaStream_t s);
-// Probe: `blocks` x 256 threads each compute `draws` (a multiple of 4) draws
-// of a generator without storing them (sink: one word per thread).
-cudaError_t launch_generator_probe(int32_t dist, uint64_t key, int64_t draws, float sigma, int blocks,
-                                   uint32_t *sink, cudaStream_t s);
+// Probe: the fill kernel of `dist` over n contiguous elements on `blocks` x
+// 256 threads, folding instead of storing (sink: one word per thread).
+cudaError_t launch_generator_probe(int32_t dist, uint64_t key, int64_t n, float sigma, int blocks, uint32_t *sink,
+                                   cudaStream_t s);
 // K3: grid-stride writer of `bytes` bytes of `value`.
 cudaError_t launch_flush(void *p, size_t bytes, uint32_t value, cudaStream_t s);
 // K6: compare-and-reduce; result (16 bytes) lands in scratch, whose 32-byte

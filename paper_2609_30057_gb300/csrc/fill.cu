@@ -216,28 +216,37 @@ fill_normal_f32_vec(uint64_t key, float sigma, float *__restrict__ out, int64_t 
     }
 }
 
-// Measurement probe: the generators' per-draw arithmetic (the same device
-// functions as the fill kernels) with no stores, to measure the rate at which
-// this GPU can compute draws.  Each thread runs `draws` consecutive draws of
-// its own stretch of the stream and folds every result into one word, which
-// it stores only if it equals a value no fold produces in practice (the store
-// keeps the arithmetic live; `sink` must hold one word per thread anyway).
+// Measurement probe: each fill kernel's loop (the same grid-stride walk over
+// 16-byte groups of a contiguous buffer of n elements, the same per-draw device
+// functions) with every group folded into one word instead of stored, to
+// measure the rate at which this GPU computes the generator: the fills'
+// compute ceiling.  The fold is stored only if it equals a value no run
+// produces in practice (it keeps the arithmetic live; `sink` must hold one
+// word per thread anyway).
 template <int DIST>
 __global__ void __launch_bounds__(256)
-generator_probe(uint64_t key, int64_t draws, float sigma, uint32_t *sink) {
-    const uint64_t t = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    uint64_t s = key + (t * (uint64_t)draws + 1ull) * kGamma;
+generator_probe(uint64_t key, int64_t n, float sigma, uint32_t *sink) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t t = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     uint32_t acc = 0;
-    for (int64_t i = 0; i < draws; i += 4) {
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            if constexpr (DIST == KREX_DIST_UNIFORM_PM1) {
-                acc ^= uniform_16x2<false>(s);
-            } else {
-                const float2 p = normal_pair(mix64(s), sigma);
-                acc ^= __float_as_uint(p.x) ^ (__float_as_uint(p.y) << 1);
-            }
+    if constexpr (DIST == KREX_DIST_UNIFORM_PM1) {
+        for (int64_t g = t; g < (n >> 3); g += stride) {
+            uint64_t s = key + (((uint64_t)(g << 3) >> 1) + 1ull) * kGamma;
+            uint32_t v = uniform_16x2<false>(s);
             s += kGamma;
+            v ^= uniform_16x2<false>(s);
+            s += kGamma;
+            v ^= uniform_16x2<false>(s);
+            s += kGamma;
+            v ^= uniform_16x2<false>(s);
+            acc ^= v;
+        }
+    } else {
+        for (int64_t g = t; g < (n >> 2); g += stride) {
+            uint64_t s = key + (((uint64_t)(g << 2) >> 1) + 1ull) * kGamma;
+            float2 p0 = normal_pair(mix64(s), sigma);
+            float2 p1 = normal_pair(mix64(s + kGamma), sigma);
+            acc ^= __float_as_uint(p0.x) ^ __float_as_uint(p0.y) ^ __float_as_uint(p1.x) ^ __float_as_uint(p1.y);
         }
     }
     if (acc == 0x5EED5EEDu) sink[t] = acc;
@@ -303,12 +312,12 @@ void launch_uniform(uint64_t key, uint16_t *p, bool aligned, int64_t rows, int64
 
 }  // namespace
 
-cudaError_t launch_generator_probe(int32_t dist, uint64_t key, int64_t draws, float sigma, int blocks,
-                                   uint32_t *sink, cudaStream_t s) {
+cudaError_t launch_generator_probe(int32_t dist, uint64_t key, int64_t n, float sigma, int blocks, uint32_t *sink,
+                                   cudaStream_t s) {
     if (dist == KREX_DIST_UNIFORM_PM1)
-        generator_probe<KREX_DIST_UNIFORM_PM1><<<blocks, 256, 0, s>>>(key, draws, sigma, sink);
+        generator_probe<KREX_DIST_UNIFORM_PM1><<<blocks, 256, 0, s>>>(key, n, sigma, sink);
     else
-        generator_probe<KREX_DIST_NORMAL><<<blocks, 256, 0, s>>>(key, draws, sigma, sink);
+        generator_probe<KREX_DIST_NORMAL><<<blocks, 256, 0, s>>>(key, n, sigma, sink);
     return cudaGetLastError();
 }
 

@@ -201,7 +201,10 @@ check_16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref, 
     Acc acc;
     clear_done(sc);
     const int64_t stride = (int64_t)gridDim.x * blockDim.x;
-    auto add8 = [&](const uint4 &o, const float4 &r0, const float4 &r1) {
+    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < n8; g += stride) {
+        uint4 o = __ldcs(out + g);
+        float4 r0 = __ldcs(ref + 2 * g);
+        float4 r1 = __ldcs(ref + 2 * g + 1);
         float f[8];
         x8_to_f32<T>(o, f);
         acc.add(f[0], r0.x, atol, rtol);
@@ -212,17 +215,7 @@ check_16_f32_vec(const uint4 *__restrict__ out, const float4 *__restrict__ ref, 
         acc.add(f[5], r1.y, atol, rtol);
         acc.add(f[6], r1.z, atol, rtol);
         acc.add(f[7], r1.w, atol, rtol);
-    };
-    int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    // two steps per pass, all six loads issued before either is used
-    for (; g + stride < n8; g += 2 * stride) {
-        const uint4 o0 = __ldcs(out + g), o1 = __ldcs(out + g + stride);
-        const float4 r00 = __ldcs(ref + 2 * g), r01 = __ldcs(ref + 2 * g + 1);
-        const float4 r10 = __ldcs(ref + 2 * (g + stride)), r11 = __ldcs(ref + 2 * (g + stride) + 1);
-        add8(o0, r00, r01);
-        add8(o1, r10, r11);
     }
-    for (; g < n8; g += stride) add8(__ldcs(out + g), __ldcs(ref + 2 * g), __ldcs(ref + 2 * g + 1));
     if (blockIdx.x == 0)
         for (int64_t i = n8 * 8 + threadIdx.x; i < n; i += blockDim.x)
             acc.add(widen(out_s, i), ref_s[i], atol, rtol);

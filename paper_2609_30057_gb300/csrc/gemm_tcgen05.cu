@@ -402,6 +402,18 @@ __device__ __forceinline__ WorkItem work_item(int w, int full_items, int tiles_m
     return it;
 }
 
+// Whether whole pair tile w walks K from its end: every other wave of the
+// persistent grid (w / nclusters odd) when k_alternate is set.  All pairs of a
+// wave run at about the same time and step through K together, and the
+// previous wave's last K blocks are the ones still in L2, A's rows of them
+// shared with this wave; so a wave that starts where the previous one ended
+// reads them from L2 instead of HBM.  The accumulation order of a tile changes
+// with it (each output stays within the tolerance of the exact product).
+// Split tiles (the final partial wave's halves) keep the forward order.
+__device__ __forceinline__ bool k_reversed(int w, int nclusters, int full_items, int k_alternate) {
+    return k_alternate && w < full_items && ((w / nclusters) & 1);
+}
+
 // Two fp32 values rounded (RNE) to bf16 or binary16, packed low | high << 16.
 template <bool F16>
 __device__ __forceinline__ uint32_t pack2(float lo, float hi) {
@@ -454,7 +466,7 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                       int N, int K, int bn, int tiles_m, int tiles_n, int full_items, int num_items,
                       int group_m, int c_vec, int c_tma, int stages, uint64_t timeout_ns, int split_k,
                       float *ws_partial, uint32_t *ws_count, uint32_t *ws_flag, uint32_t launch_id,
-                      uint32_t wait_tag) {
+                      uint32_t wait_tag, int k_alternate) {
     // the pair kernel's tile constants (the file-level BM, BK serve the host's tensor maps)
     using CF = v2::Cfg<KSUB>;
     constexpr int BM = v2::BM, BN = v2::BN, BK = v2::BK, STAGES = CF::STAGES;
@@ -541,7 +553,9 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             const int m0 = mb * 2 * BM + (int)rank * BM;
             const int n0 = col0 + (int)rank * b_half;
             abort_flag[1] = (uint32_t)w;
-            for (int kb = it.kb0; kb < it.kb1; ++kb) {
+            const bool rev = k_reversed(w, nclusters, full_items, k_alternate);
+            for (int i = it.kb0; i < it.kb1; ++i) {
+                const int kb = rev ? it.kb0 + it.kb1 - 1 - i : i;
                 abort_flag[2] = (uint32_t)kb;
                 if (!mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, timeout_ns, 0x31)) {
                     ok = false;
@@ -591,7 +605,9 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             }
             tc_fence_after();
             const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
-            for (int kb = it.kb0; kb < it.kb1; ++kb) {
+            const bool rev = k_reversed(w, nclusters, full_items, k_alternate);
+            for (int i = it.kb0; i < it.kb1; ++i) {
+                const int kb = rev ? it.kb0 + it.kb1 - 1 - i : i;  // the stage the producer loaded
                 abort_flag[4] = (uint32_t)kb;
                 if (!mbar_wait(full_bar(stage), phase, abort_flag, timeout_ns, 0x42)) {
                     ok = false;
@@ -609,7 +625,7 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
 #pragma unroll
                         for (int k = 0; k < BK / 16; ++k)
                             mma_bf16_pair(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(128 * k), idesc,
-                                          ((kb - it.kb0) | h | k) != 0 ? 1u : 0u);
+                                          ((i - it.kb0) | h | k) != 0 ? 1u : 0u);
                     }
                 }
                 mma_commit_pair(empty_bar(stage));
@@ -1034,7 +1050,8 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
                                                        tiles_n, (int)full_items, (int)items,
                                                        raster_group(tun, tiles, max_clusters), c_vec,
                                                        c_tma, stages, wait_timeout_ns(tun), split_k, ws_partial,
-                                                       ws_count, ws_flag, launch_id, wait_tag);
+                                                       ws_count, ws_flag, launch_id, wait_tag,
+                                                       tun.gemm_k_alternate == 0 ? 0 : 1);
         };
         const int st2 = ring_stages(tun, v2::Cfg<2>::STAGES), st1 = ring_stages(tun, v2::Cfg<1>::STAGES);
         if (ksub == 2 && f16)

@@ -156,15 +156,18 @@ def test_tuning_defaults_roundtrip_and_range_checks():
     d = krex.krex_tuning()
     lib.krex_tuning_defaults(ctypes.byref(d))
     assert (d.gemm_pair_tile_n, d.gemm_stage_k, d.gemm_ring_stages, d.gemm_raster_group, d.gemm_tail_split,
-            d.gemm_split_k, d.reference_tiling, d.wait_timeout_ms) == (0, 0, 0, 0, -1, -1, -1, 0)
+            d.gemm_split_k, d.gemm_k_alternate, d.reference_tiling, d.wait_timeout_ms) == (0, 0, 0, 0, -1, -1, -1, -1, 0)
     try:
         krex.krex_set_tuning(gemm_pair_tile_n=192, gemm_stage_k=64, gemm_ring_stages=5, gemm_raster_group=3,
-                             gemm_tail_split=0, gemm_split_k=1, reference_tiling=2, wait_timeout_ms=500)
+                             gemm_tail_split=0, gemm_split_k=1, gemm_k_alternate=0, reference_tiling=2,
+                             wait_timeout_ms=500)
         got = krex.krex_get_tuning()
         assert got == {"gemm_pair_tile_n": 192, "gemm_stage_k": 64, "gemm_ring_stages": 5, "gemm_raster_group": 3,
-                       "gemm_tail_split": 0, "gemm_split_k": 1, "reference_tiling": 2, "wait_timeout_ms": 500}
+                       "gemm_tail_split": 0, "gemm_split_k": 1, "gemm_k_alternate": 0, "reference_tiling": 2,
+                       "wait_timeout_ms": 500}
         bad = [{"gemm_pair_tile_n": 100}, {"gemm_stage_k": 32}, {"gemm_ring_stages": 4},  # 4 > 3 stages of K 128
                {"gemm_ring_stages": 1}, {"gemm_raster_group": 65}, {"gemm_tail_split": 2}, {"gemm_split_k": -2},
+               {"gemm_k_alternate": 2},
                {"reference_tiling": 6}, {"wait_timeout_ms": -1}]
         for b in bad:
             with pytest.raises(krex.KrexError, match="INVALID"):
@@ -191,6 +194,6 @@ def test_generator_probe_rejects_bad_arguments_before_any_launch():
     lib = krex.lib()
     assert lib.krex_probe_generator(7, 64, 1, 2.0, 16, None) == krex.KREX_ERR_INVALID      # bad distribution
     assert lib.krex_probe_generator(0, 64, 1, 2.0, None, None) == krex.KREX_ERR_INVALID    # no sink
-    assert lib.krex_probe_generator(0, 62, 1, 2.0, 16, None) == krex.KREX_ERR_INVALID      # not a multiple of 4
+    assert lib.krex_probe_generator(0, 60, 1, 2.0, 16, None) == krex.KREX_ERR_INVALID      # not a multiple of 8
     assert lib.krex_probe_generator(1, 0, 1, 2.0, 16, None) == krex.KREX_ERR_INVALID       # no draws
     assert lib.krex_probe_generator(1, 64, 0, 2.0, 16, None) == krex.KREX_ERR_INVALID      # no blocks

@@ -143,6 +143,6 @@ def test_generator_probe_runs_and_leaves_the_context_clean(dist):
     # fold value no run produces in practice
     n_sm = torch.cuda.get_device_properties(0).multi_processor_count
     sink = torch.zeros(n_sm * 256, dtype=torch.int32, device="cuda")
-    krex.krex_probe_generator(dist, 64, n_sm, sink)
+    krex.krex_probe_generator(dist, 1 << 20, n_sm, sink)
     torch.cuda.synchronize()
     assert krex.krex_device_status() == 0
