@@ -575,28 +575,38 @@ def main():
     # ------------------------------------------------ e2e (host buffers)
     e2e = None
     if not args.no_e2e:
-        host_in = [torch.empty(t.shape, dtype=t.dtype).pin_memory() for t in ws.inputs]
+        # page-locked, huge-page-backed host buffers (krex_host_alloc)
+        host_in = [krex.host_buffer(t.shape, t.dtype) for t in ws.inputs]
         for h, t in zip(host_in, ws.inputs):
             h.copy_(t)
-        host_out = torch.empty(ws.out.shape, dtype=ws.out.dtype).pin_memory()
+        host_out = krex.host_buffer(ws.out.shape, ws.out.dtype)
         ptrs = [h.data_ptr() for h in host_in]
         for _ in range(max(1, min(args.warmup, 2))):
             ws.run(host_in=ptrs, host_out=host_out.data_ptr())
         barrier()
         torch.cuda.synchronize()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(args.steps):
-            r = ws.run(host_in=ptrs, host_out=host_out.data_ptr())
-            if not r.passed:
-                raise SystemExit("check failed (e2e)")
-        e1.record(stream)
-        torch.cuda.synchronize()
+        e_phases = []
+        e_clocks = ClockSampler(torch.cuda.current_device())
+        with e_clocks:
+            e0.record(stream)
+            for _ in range(args.steps):
+                r = ws.run(host_in=ptrs, host_out=host_out.data_ptr())
+                if not r.passed:
+                    raise SystemExit("check failed (e2e)")
+                e_phases.append(list(r.phase_ms))
+            e1.record(stream)
+            torch.cuda.synchronize()
         barrier()
         te_ms = replicas.max_over_ranks(dist, e0.elapsed_time(e1), device="cuda")
         e2e = {"value": replicas.aggregate_throughput(args.steps, world, te_ms / 1e3), "unit": "cmds/s",
                "h2d_bytes_per_step": sum(h.numel() * h.element_size() for h in host_in),
-               "d2h_bytes_per_step": host_out.numel() * host_out.element_size() + 16}
+               "d2h_bytes_per_step": host_out.numel() * host_out.element_size() + 16,
+               "ms_per_step": te_ms / args.steps,
+               # the phases of these commands (inputs = the host-to-device copies)
+               "phase_ms": dict(zip(["inputs", "reference", "candidate", "check", "timed_loop"],
+                                    [statistics.fmean(p[i] for p in e_phases) for i in range(5)])),
+               "clocks": e_clocks.summary()}
         del host_in, host_out
 
     cs = clocks.summary()

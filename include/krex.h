@@ -450,6 +450,25 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
                              const void *const *host_in, void *host_out, float *durations_ms,
                              krex_command_result *result, krex_stream_t stream);
 
+/* ------------------------------------------------------- host memory ----- */
+
+/* Page-locked host memory for a command's host-side inputs and outputs
+ * (krex_command_run's host_in / host_out).  Not part of the paper's method.
+ * The buffer is an anonymous mapping advised to use transparent huge pages,
+ * aligned to the huge-page size, then registered with CUDA (page-locked, so
+ * copies run asynchronously at the host link's rate).  On hosts whose kernel
+ * gives huge pages only on request (transparent hugepage mode "madvise"), a
+ * buffer without them keeps its copies at full rate only while they run back
+ * to back: measured on GB300 (64 KiB base pages), a 512 MiB host-to-device
+ * copy took 2.6 ms back to back but 15-90 ms after a pause of a quarter
+ * second, every other time, with memory pinned by cudaHostAlloc or by
+ * registering an unadvised mapping; with huge pages it took 2.6 ms every
+ * time.  bytes > 0; *ptr receives the buffer (zero-filled).  Free it with
+ * krex_host_free(ptr, bytes).  Errors: INVALID for a null ptr or zero bytes,
+ * CUDA if registration fails (nothing stays allocated then). */
+krex_status krex_host_alloc(size_t bytes, void **ptr);
+krex_status krex_host_free(void *ptr, size_t bytes);
+
 /* ------------------------------------------------------ measurement ----- */
 
 /* Measurement probe, not part of the paper's method: the fill kernel of a

@@ -114,6 +114,8 @@ SIGNATURES = {
     "krex_get_tuning": (_i32, [_P(krex_tuning)]),
     "krex_debug_stall_handover": (_i32, [_i32]),
     "krex_probe_generator": (_i32, [_i32, _u64, _i32, _f32, _vp, _vp]),
+    "krex_host_alloc": (_i32, [_sz, _P(_vp)]),
+    "krex_host_free": (_i32, [_vp, _sz]),
     "krex_gate_shared_bytes": (_sz, [_i32]),
     "krex_gate_shared_init": (_i32, [_vp, _sz, _i32]),
     "krex_gate_shared_attach": (_i32, [_vp, _sz, _P(_vp)]),
@@ -482,6 +484,26 @@ def krex_probe_generator(dist: int, n_elements: int, blocks: int, sink, sigma: f
     least blocks * 256 * 4 bytes."""
     _ok(lib().krex_probe_generator(dist, n_elements, blocks, sigma, sink.data_ptr(), _stream(stream)),
         "krex_probe_generator")
+
+
+def host_buffer(shape, dtype):
+    """A CPU tensor over page-locked, huge-page-backed host memory from
+    krex_host_alloc (for a command's host_in / host_out); the memory is freed
+    with the tensor."""
+    import weakref
+
+    import torch
+    shape = tuple(int(x) for x in shape)
+    nbytes = max(1, math.prod(shape) * torch.empty((), dtype=dtype).element_size())
+    p = ctypes.c_void_p()
+    _ok(lib().krex_host_alloc(nbytes, ctypes.byref(p)), "krex_host_alloc")
+    raw = (ctypes.c_uint8 * nbytes).from_address(p.value)
+    t = torch.frombuffer(raw, dtype=torch.uint8, count=nbytes)
+    out = t[:math.prod(shape) * torch.empty((), dtype=dtype).element_size()].view(dtype).view(shape)
+    addr = p.value
+    weakref.finalize(raw, lambda: lib().krex_host_free(addr, nbytes))
+    out._krex_host_owner = raw   # keeps the mapping alive as long as the tensor
+    return out
 
 
 def krex_debug_stall_handover(on: bool) -> None:

@@ -4,6 +4,7 @@
 // kernels live in the other translation units.
 #include <pthread.h>
 #include <sched.h>
+#include <sys/mman.h>
 #include <stdarg.h>
 #include <stdio.h>
 #include <string.h>
@@ -783,6 +784,63 @@ static void CUDART_CB hold_fn(void *p) {
         nanosleep(&ts, nullptr);
     }
     delete a;
+}
+
+// Host buffers: anonymous mappings aligned to the transparent huge-page size
+// (read from the kernel, 2 MiB if it does not say), advised to use huge pages,
+// zero-filled (which allocates the pages), then registered with CUDA.  The
+// mapping is over-allocated by one alignment and trimmed, so krex_host_free
+// unmaps exactly [ptr, ptr + rounded bytes).
+static size_t host_huge_page_bytes() {
+    static const size_t v = [] {
+        size_t b = 0;
+        if (FILE *f = fopen("/sys/kernel/mm/transparent_hugepage/hpage_pmd_size", "r")) {
+            unsigned long long x = 0;
+            if (fscanf(f, "%llu", &x) == 1) b = (size_t)x;
+            fclose(f);
+        }
+        if (b < ((size_t)2 << 20) || b > ((size_t)1 << 30) || (b & (b - 1))) b = (size_t)2 << 20;
+        return b;
+    }();
+    return v;
+}
+
+static size_t host_rounded(size_t bytes) {
+    const size_t a = host_huge_page_bytes();
+    return (bytes + a - 1) / a * a;
+}
+
+krex_status krex_host_alloc(size_t bytes, void **ptr) {
+    if (!ptr || bytes == 0 || bytes > ((size_t)1 << 46)) return set_error(KREX_ERR_INVALID, "host_alloc: bad arguments");
+    *ptr = nullptr;
+    const size_t align = host_huge_page_bytes(), len = host_rounded(bytes);
+    void *raw = mmap(nullptr, len + align, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
+    if (raw == MAP_FAILED) return set_error(KREX_ERR_INVALID, "host_alloc: mmap of %zu bytes failed", len + align);
+    const uintptr_t r = reinterpret_cast<uintptr_t>(raw);
+    const uintptr_t a = (r + align - 1) / align * align;
+    if (a > r) munmap(raw, a - r);
+    if (r + len + align > a + len) munmap(reinterpret_cast<void *>(a + len), r + len + align - (a + len));
+    void *p = reinterpret_cast<void *>(a);
+#ifdef MADV_HUGEPAGE
+    madvise(p, len, MADV_HUGEPAGE);  // advice only: without it the buffer still works
+#endif
+    memset(p, 0, len);
+    cudaError_t e = cudaHostRegister(p, len, cudaHostRegisterDefault);
+    if (e != cudaSuccess) {
+        munmap(p, len);
+        return cuda_error(e, "cudaHostRegister (host_alloc)");
+    }
+    *ptr = p;
+    return ok();
+}
+
+krex_status krex_host_free(void *ptr, size_t bytes) {
+    if (!ptr || bytes == 0) return set_error(KREX_ERR_INVALID, "host_free: bad arguments");
+    const size_t len = host_rounded(bytes);
+    cudaError_t e = cudaHostUnregister(ptr);
+    munmap(ptr, len);
+    if (e != cudaSuccess) return cuda_error(e, "cudaHostUnregister (host_free)");
+    return ok();
 }
 
 krex_status krex_probe_generator(int32_t dist, uint64_t n_elements, int32_t blocks, float sigma, void *dev_sink,

@@ -197,3 +197,12 @@ def test_generator_probe_rejects_bad_arguments_before_any_launch():
     assert lib.krex_probe_generator(0, 60, 1, 2.0, 16, None) == krex.KREX_ERR_INVALID      # not a multiple of 8
     assert lib.krex_probe_generator(1, 0, 1, 2.0, 16, None) == krex.KREX_ERR_INVALID       # no draws
     assert lib.krex_probe_generator(1, 64, 0, 2.0, 16, None) == krex.KREX_ERR_INVALID      # no blocks
+
+
+def test_host_alloc_rejects_bad_arguments():
+    import paper_2609_30057_gb300 as krex
+    lib = krex.lib()
+    p = ctypes.c_void_p()
+    assert lib.krex_host_alloc(0, ctypes.byref(p)) == krex.KREX_ERR_INVALID
+    assert lib.krex_host_alloc(4096, None) == krex.KREX_ERR_INVALID
+    assert lib.krex_host_free(None, 4096) == krex.KREX_ERR_INVALID

@@ -155,3 +155,23 @@ def test_gemm_16384_command_against_the_oracle():
     mx, nv = ref.check_f32(gen.bf16_to_f32(bits16(ws.out)), ws.ref.cpu().numpy(), w.atol, w.rtol)
     assert nv == 0 == int(res.check.n_violations)
     assert ref.check_bits(res.check.max_abs_err) == ref.check_bits(mx)
+
+
+def test_command_with_library_host_buffers():
+    # inputs and output in krex_host_alloc buffers (page-locked, huge-page
+    # backed): the same output as device-generated inputs, twice in a row
+    w = scaled(WORKLOADS["gemm_bf16_256"], M=512, N=384, K=640, iters=3)
+    ws = Workspace(w)
+    res = ws.run()
+    assert res.passed == 1
+    want = bits16(ws.out)
+    hin = [krex.host_buffer(t.shape, t.dtype) for t in ws.inputs]
+    for h, t in zip(hin, ws.inputs):
+        h.copy_(t)
+    hout = krex.host_buffer(ws.out.shape, ws.out.dtype)
+    assert all(h.is_pinned() for h in hin) and hout.is_pinned()
+    for _ in range(2):
+        hout.zero_()
+        r = ws.run(host_in=[h.data_ptr() for h in hin], host_out=hout.data_ptr())
+        assert r.passed == 1
+        assert np.array_equal(hout.view(torch.int16).numpy().view(np.uint16), want)
