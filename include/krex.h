@@ -184,10 +184,11 @@ krex_status krex_l2_bytes(size_t *bytes);
 /* Bytes of device scratch krex_check needs (at least 16-byte aligned). */
 size_t krex_check_scratch_bytes(void);
 
-/* Make a check scratch ready for its first use: zeroes its 32-byte header on
- * `stream` (asynchronous).  Equivalent to allocating the scratch zero-filled.
- * Needed once per scratch buffer; every check leaves the header ready for the
- * next one (its ticket re-armed), so no per-call reset runs in front of the
+/* Make a check scratch ready for its first use: zeroes its
+ * krex_check_scratch_bytes() bytes on `stream` (asynchronous).  Equivalent to
+ * allocating the scratch zero-filled.  Needed once per scratch buffer; every
+ * check leaves the scratch ready for the next one (the next call's result slot
+ * cleared, its ticket re-armed), so no per-call reset runs in front of the
  * check kernel.  Errors: INVALID for a null or small scratch, UNSUPPORTED if
  * it is not 16-byte aligned. */
 krex_status krex_check_scratch_init(void *dev_scratch, size_t scratch_bytes, krex_stream_t stream);
@@ -197,12 +198,12 @@ krex_status krex_check_scratch_init(void *dev_scratch, size_t scratch_bytes, kre
  *   d = |out - ref|, violation iff !(d <= atol + rtol*|ref|)  (NaN counts).
  * out may be bf16 or fp32 (widened exactly); ref is fp32 or bf16.  Shapes must
  * match.  dev_scratch: caller-owned device memory of >= krex_check_scratch_bytes()
- * bytes whose 32-byte header was zeroed once before its first check (zero-
- * filled allocation or krex_check_scratch_init) and has since been used only
- * by checks; one check at a time per scratch.  SYNCHRONISES `stream` and writes
+ * bytes that were zeroed once before its first check (zero-filled allocation
+ * or krex_check_scratch_init) and have since been used only by checks; one
+ * check at a time per scratch.  SYNCHRONISES `stream` and writes
  * *host_result.  The result is bit-identical for any launch shape (max and
  * count are exact).  Errors: INVALID for null pointers, shape/dtype mismatch,
- * small scratch; STATE if the header shows the scratch was not ready (never
+ * small scratch; STATE if the scratch shows it was not ready (never
  * zeroed, or written by something else since): no result is returned then. */
 krex_status krex_check(krex_buf out, krex_buf ref, float atol, float rtol, void *dev_scratch,
                        size_t scratch_bytes, krex_check_result *host_result,
@@ -210,9 +211,9 @@ krex_status krex_check(krex_buf out, krex_buf ref, float atol, float rtol, void 
 
 /* The check in two halves, for callers that overlap it with other work:
  * krex_check_launch enqueues the compare-and-reduce on `stream` and leaves the
- * 16-byte krex_check_result at the start of dev_scratch (asynchronous; same
- * arguments and errors as krex_check); krex_check_fetch copies that result to
- * *host_result and SYNCHRONISES `stream`.  krex_check = launch + fetch. */
+ * result in dev_scratch (asynchronous; same arguments and errors as
+ * krex_check); krex_check_fetch copies that result to *host_result and
+ * SYNCHRONISES `stream`.  krex_check = launch + fetch. */
 krex_status krex_check_launch(krex_buf out, krex_buf ref, float atol, float rtol, void *dev_scratch,
                               size_t scratch_bytes, krex_stream_t stream);
 krex_status krex_check_fetch(const void *dev_scratch, krex_check_result *host_result,
@@ -228,9 +229,9 @@ krex_status krex_check_fetch(const void *dev_scratch, krex_check_result *host_re
  * every GPU that loads the library until the process exits.  The first call on
  * a device (and the first after that device's context was destroyed and
  * created again) does the set-up there: it resolves the array's address
- * (cudaGetSymbolAddress) and zeroes its header on `stream`; make that first
- * call before any stream capture.  It allocates nothing and calls no
- * allocating routine.  Every call shares the one array per device and
+ * (cudaGetSymbolAddress) and zeroes the check's scratch in it on `stream`;
+ * make that first call before any stream capture.  It allocates nothing and
+ * calls no allocating routine.  Every call shares the one array per device and
  * leaves the last result in it; the call clears what must start at zero, but
  * calls that overlap on the GPU (other streams, other threads) race on it, so
  * serialise them.  Same arguments, result and bit-exact semantics as

@@ -10,17 +10,20 @@
 // max |d| is reduced over the IEEE bit pattern as unsigned (valid ordering for
 // non-negative floats; a NaN dominates and is reported as the canonical quiet
 // NaN 0x7FC00000).  Warp reduction with __reduce_max_sync/__reduce_add_sync,
-// one partial per block in scratch, one atomic ticket per block; the last
-// block to take a ticket combines the partials, writes the result, re-arms
-// the ticket and marks the call done.  Max and count are exact, so the result
-// does not depend on the launch shape.
+// then each block adds its count and maxes its bits into the call's result
+// slot with two atomics and takes a ticket; the last block to take one
+// prepares the other slot for the next call, re-arms the ticket and marks the
+// call done.  Max and count are exact, so the result does not depend on the
+// launch shape or the order of the atomics.
 //
-// The scratch header is zeroed once (by the caller or krex_check_scratch_init)
-// and every call leaves it ready for the next, so a check is one launch with
-// no reset in front of it.  Block 0 clears the done word at its start; a
-// scratch whose ticket was not zero on entry ends with done = 0 (no block saw
-// itself last) or a non-zero ticket (a block saw itself last too early), and
-// the host's fetch reports that instead of a result.
+// The scratch is zeroed once (by the caller or krex_check_scratch_init) and
+// every call leaves it ready for the next, so a check is one launch with no
+// reset in front of it: calls alternate between two result slots (the slot of
+// call g is g mod 2, g counted in the scratch), and a call's last block
+// clears the slot the next call uses.  Block 0 clears the done word at its
+// start; a scratch whose ticket was not zero on entry ends with done = 0 (no
+// block saw itself last) or a non-zero ticket (a block saw itself last too
+// early), and the host's fetch reports that instead of a result.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -63,22 +66,23 @@ constexpr int kVecBlocksPerSM = 8;
 constexpr int kGenericBlocksPerSM = 4;
 constexpr uint32_t kCanonicalNaN = 0x7FC00000u;
 
-struct Partial {
-    uint32_t max_bits;
-    uint32_t pad;
+// Scratch layout (device, caller-owned): two result slots and the call state,
+// each on its own 128-byte line (the atomics of a call hit the slot's line and
+// the ticket's line).
+struct Slot {
     unsigned long long count;
+    uint32_t max_bits;
+    uint32_t pad[29];
 };
-
-// Scratch layout (device, caller-owned).  Header: 32 bytes.
 struct CheckScratch {
-    Partial result;          // final {max_bits, count}
-    unsigned int ticket;     // blocks that have published a partial; 0 between calls
-    unsigned int done;       // 1 once the last block has written result
-    unsigned int pad[2];
-    Partial partial[kCheckMaxBlocks];
+    Slot slot[2];            // results of alternating calls
+    unsigned int ticket;     // blocks that have added their results; 0 between calls
+    unsigned int done;       // 1 once the last block has finished
+    unsigned int gen;        // calls completed on this scratch (call g uses slot g % 2)
+    unsigned int pad[29];
 };
-constexpr size_t kCheckHeaderBytes = offsetof(CheckScratch, partial);
-static_assert(kCheckHeaderBytes == 32, "check scratch header is 32 bytes");
+static_assert(sizeof(Slot) == 128 && sizeof(CheckScratch) == 384, "check scratch layout");
+constexpr size_t kCheckHeaderBytes = sizeof(CheckScratch);
 
 __device__ __forceinline__ float widen(const __nv_bfloat16 *p, int64_t i) {
     return __uint_as_float((uint32_t)(*reinterpret_cast<const uint16_t *>(p + i)) << 16);
@@ -116,11 +120,11 @@ __device__ __forceinline__ void x8_to_f32(const uint4 &u, float *f) {
     }
 }
 
-// Publish the block's partial and, in the last block, the final result.
+// Add the block's count and max into the call's slot; in the last block,
+// prepare the next call's slot and mark this call done.
 __device__ __forceinline__ void block_reduce_publish(Acc acc, CheckScratch *sc) {
     __shared__ uint32_t s_max[kCheckThreads / 32];
     __shared__ uint32_t s_cnt[kCheckThreads / 32];
-    __shared__ bool s_last;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     uint32_t m = __reduce_max_sync(0xffffffffu, acc.max_bits);
     uint32_t c = __reduce_add_sync(0xffffffffu, acc.count);
@@ -136,49 +140,25 @@ __device__ __forceinline__ void block_reduce_publish(Acc acc, CheckScratch *sc) 
             bm = max(bm, s_max[w]);
             bc += s_cnt[w];
         }
-        sc->partial[blockIdx.x].max_bits = bm;
-        sc->partial[blockIdx.x].count = bc;
+        // gen changes only in the previous call's last block (stream order)
+        const unsigned int g = __ldcg(&sc->gen);
+        Slot &slot = sc->slot[g & 1u];
+        if (bc) atomicAdd(&slot.count, bc);
+        if (bm) atomicMax(&slot.max_bits, bm);
         __threadfence();
-        unsigned int t = atomicAdd(&sc->ticket, 1u);
-        s_last = (t == gridDim.x - 1);
-    }
-    __syncthreads();
-    if (!s_last) return;
-    __threadfence();
-    // last block: combine all partials (exact max and sum).  The partials were
-    // published before their blocks' tickets (fence, then atomic), and this
-    // block has fenced after taking the last ticket, so L2 loads (which bypass
-    // L1) see them; being plain loads they can all be in flight at once.
-    uint32_t bm = 0;
-    unsigned long long bc = 0;
-#pragma unroll 4
-    for (int b = threadIdx.x; b < (int)gridDim.x; b += blockDim.x) {
-        const uint4 p = __ldcg(reinterpret_cast<const uint4 *>(&sc->partial[b]));
-        bm = max(bm, p.x);
-        bc += (unsigned long long)p.z | ((unsigned long long)p.w << 32);
-    }
-    bm = __reduce_max_sync(0xffffffffu, bm);
-    for (int o = 16; o > 0; o >>= 1) bc += __shfl_xor_sync(0xffffffffu, bc, o);
-    __syncthreads();
-    __shared__ unsigned long long s_cnt64[kCheckThreads / 32];
-    if (lane == 0) {
-        s_max[warp] = bm;
-        s_cnt64[warp] = bc;
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        uint32_t fm = 0;
-        unsigned long long fc = 0;
-        for (int w = 0; w < kCheckThreads / 32; ++w) {
-            fm = max(fm, s_max[w]);
-            fc += s_cnt64[w];
+        const unsigned int t = atomicAdd(&sc->ticket, 1u);
+        if (t == gridDim.x - 1) {
+            // every block's atomics precede its ticket: this call's slot is
+            // final; clear the next call's, re-arm, count the call, mark done
+            __threadfence();
+            Slot &next = sc->slot[(g + 1u) & 1u];
+            next.count = 0ull;
+            next.max_bits = 0u;
+            sc->ticket = 0u;
+            sc->gen = g + 1u;
+            __threadfence();
+            sc->done = 1u;
         }
-        sc->result.max_bits = fm;
-        sc->result.pad = 0;
-        sc->result.count = fc;
-        sc->ticket = 0;  // re-arm for the next call
-        __threadfence();
-        sc->done = 1u;
     }
 }
 
@@ -330,12 +310,13 @@ krex_status read_check_header(const void *scratch, krex_check_result *r, cudaStr
     if (e != cudaSuccess) return cuda_error(e, "cudaStreamSynchronize (check result)");
     if (h.done != 1u || h.ticket != 0u)
         return set_error(KREX_ERR_STATE,
-                         "check scratch was not ready (done %u, ticket %u): zero its first %zu bytes once before "
-                         "its first check (krex_check_scratch_init)",
+                         "check scratch was not ready (done %u, ticket %u): zero its %zu bytes once before its "
+                         "first check (krex_check_scratch_init)",
                          h.done, h.ticket, kCheckHeaderBytes);
-    memcpy(&r->max_abs_err, &h.result.max_bits, sizeof(float));
+    const Slot &res = h.slot[(h.gen - 1u) & 1u];  // the call just completed
+    memcpy(&r->max_abs_err, &res.max_bits, sizeof(float));
     r->reserved = 0;
-    r->n_violations = h.result.count;
+    r->n_violations = res.count;
     return KREX_OK;
 }
 
@@ -393,9 +374,9 @@ cudaError_t launch_check(const void *out, int out_dtype, int64_t ldo, const void
 // measurement around them.  The scratch is a fixed static device array that
 // each GPU loading this library keeps until the process exits.
 
-// Capacity: the check's 32-byte header (result, ticket, done word, padding)
-// plus one 16-byte partial for each of its at most 2048 blocks (32,800 bytes),
-// rounded up to a multiple of 256.
+// Capacity: room for the check's scratch (two result slots and the call
+// state, 384 bytes) with a wide margin, fixed so the array's size does not
+// change with the check's layout.
 #define KREX_CHECK_NOALLOC_SCRATCH_BYTES 33024
 static __device__ __align__(256) unsigned char g_check_noalloc_scratch[KREX_CHECK_NOALLOC_SCRATCH_BYTES];
 static_assert(sizeof(krex::CheckScratch) <= KREX_CHECK_NOALLOC_SCRATCH_BYTES,
