@@ -525,6 +525,8 @@ def main():
                     choices=["gemm", "gemm_ref", "fill_uniform", "fill_normal", "flush", "check", "softmax"],
                     help="launch one kernel of the workload --launches times and exit (for ncu captures)")
     ap.add_argument("--launches", type=int, default=3)
+    ap.add_argument("--tuning", action="append", default=[], metavar="FIELD=VALUE",
+                    help="with --kernel-only: set a field of the library's tuning record first (repeatable)")
     args = ap.parse_args()
 
     from paper_2609_30057_gb300 import replicas
@@ -698,6 +700,8 @@ def kernel_only(args):
     from paper_2609_30057_gb300.command import WORKLOADS, Workspace
     krex.build()
     torch.cuda.set_device(0)
+    if args.tuning:
+        krex.krex_set_tuning(**{k: int(v) for k, v in (t.split("=", 1) for t in args.tuning)})
     stream = torch.cuda.current_stream()
     name = args.workload
     if args.kernel_only in ("softmax", "fill_normal") and WORKLOADS[name].is_gemm:
