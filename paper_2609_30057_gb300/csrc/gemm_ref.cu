@@ -173,22 +173,35 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
 }
 
 // The same tiling for GEMMs made of whole tiles (M % 128 = N % 128 = K % 16 =
-// 0, 16-byte aligned rows), the sizes of the benchmark workloads: no bounds
-// checks, one 16-byte load of A and one of B per thread and slice, a 32-bit K
-// counter, and a column-major sweep of the outer product (each b[j] held
-// across the eight rows).  Each
-// output is the same k-order FMA chain as in gemm_ref_simt (identical bits).
-// Measured on GB300 in one process (TFLOP/s at 4096^3 / 8192^3 / 16384^3, L2
-// flushed): 58.6 / 60.8 / 60.9 against 55.1 / 57.1 / 57.0 for gemm_ref_simt
-// with the row-major sweep and 52.6 / 54.8 / 55.4 with the column-major one.
+// 0, 16-byte aligned rows), the sizes of the benchmark workloads.  Operands
+// stay 16-bit in shared memory (the A slice transposed to k-major, the B
+// slice as loaded), and the outer product uses the mixed-precision FMA
+// (fma.rn.f32.bf16 / .f16: 16-bit a and b, fp32 c and d), which widens both
+// factors exactly and rounds once like fmaf on the widened values: each
+// output is the same k-order FMA chain as in gemm_ref_simt (identical bits),
+// with half the shared-memory traffic and fragment registers and no
+// conversion in the slice staging.  No bounds checks, one 16-byte load of A
+// and one of B per thread and slice, a 32-bit K loop, 8 x 8 outputs per
+// thread swept column by column.  Measured on GB300 in one process (TFLOP/s
+// at 4096^3 / 16384^3, L2 flushed): 64.4 / 67.6, against 58.8 / 60.4 for the
+// same tiling with operands widened to fp32 in shared memory and 55.0 / 57.0
+// for gemm_ref_simt.
+template <bool F16>
+__device__ __forceinline__ void fma_mixed(float &acc, unsigned short a, unsigned short b) {
+    if constexpr (F16) asm("fma.rn.f32.f16 %0, %1, %2, %0;" : "+f"(acc) : "h"(a), "h"(b));
+    else asm("fma.rn.f32.bf16 %0, %1, %2, %0;" : "+f"(acc) : "h"(a), "h"(b));
+}
+__device__ __forceinline__ void halves(uint32_t w, unsigned short &lo, unsigned short &hi) {
+    asm("mov.b32 {%0, %1}, %2;" : "=h"(lo), "=h"(hi) : "r"(w));
+}
+
 template <bool F16>
 __global__ void __launch_bounds__(256, 2)
 gemm_ref_whole(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__restrict__ B, int64_t ldb,
                float *__restrict__ C, int64_t ldc, int K) {
     constexpr int TK = 16, TN = 128;
-    extern __shared__ __align__(16) float smem[];
-    float *As = smem;                  // [2][TK][TM]
-    float *Bs = smem + 2 * TK * TM;    // [2][TK][TN]
+    __shared__ __align__(16) uint16_t As[2][TK][TM];   // k-major
+    __shared__ __align__(16) uint16_t Bs[2][TK][TN];
     const int t = threadIdx.x, tx = t & 15, ty = t >> 4;
     const int64_t m0 = (int64_t)blockIdx.y * TM, n0 = (int64_t)blockIdx.x * TN;
     // one 16-byte load of A (row t / 2, k offset 8 (t % 2)) and one of B
@@ -199,19 +212,14 @@ gemm_ref_whole(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__re
         ub = __ldg(reinterpret_cast<const uint4 *>(B + (int64_t)(k0 + (t >> 4)) * ldb + n0 + 8 * (t & 15)));
     };
     auto stage = [&](int nb) {
-        float *as = As + nb * TK * TM, *bs = Bs + nb * TK * TN;
         const int row = t >> 1, kk = 8 * (t & 1);
         const uint32_t wa[4] = {ua.x, ua.y, ua.z, ua.w};
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-            as[(kk + 2 * j) * TM + row] = lo_f32<F16>(wa[j]);
-            as[(kk + 2 * j + 1) * TM + row] = hi_f32<F16>(wa[j]);
+            As[nb][kk + 2 * j][row] = (uint16_t)(wa[j] & 0xFFFFu);
+            As[nb][kk + 2 * j + 1][row] = (uint16_t)(wa[j] >> 16);
         }
-        float *dst = bs + (t >> 4) * TN + 8 * (t & 15);
-        *reinterpret_cast<float4 *>(dst) = make_float4(lo_f32<F16>(ub.x), hi_f32<F16>(ub.x), lo_f32<F16>(ub.y),
-                                                       hi_f32<F16>(ub.y));
-        *reinterpret_cast<float4 *>(dst + 4) = make_float4(lo_f32<F16>(ub.z), hi_f32<F16>(ub.z), lo_f32<F16>(ub.w),
-                                                           hi_f32<F16>(ub.w));
+        *reinterpret_cast<uint4 *>(&Bs[nb][t >> 4][8 * (t & 15)]) = ub;
     };
     float acc[8][8];
 #pragma unroll
@@ -225,19 +233,25 @@ gemm_ref_whole(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__re
     for (int k0 = 0; k0 < K; k0 += TK) {
         const bool more = k0 + TK < K;
         if (more) fetch(k0 + TK);  // the next slice comes in while this one is multiplied
-        const float *as = As + buf * TK * TM, *bs = Bs + buf * TK * TN;
 #pragma unroll
         for (int k = 0; k < TK; ++k) {
-            const float4 a0 = *reinterpret_cast<const float4 *>(as + k * TM + ty * 4);
-            const float4 a1 = *reinterpret_cast<const float4 *>(as + k * TM + 64 + ty * 4);
-            const float4 b0 = *reinterpret_cast<const float4 *>(bs + k * TN + tx * 4);
-            const float4 b1 = *reinterpret_cast<const float4 *>(bs + k * TN + 64 + tx * 4);
-            const float a[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
-            const float b[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
+            const uint2 a0 = *reinterpret_cast<const uint2 *>(&As[buf][k][ty * 4]);
+            const uint2 a1 = *reinterpret_cast<const uint2 *>(&As[buf][k][64 + ty * 4]);
+            const uint2 b0 = *reinterpret_cast<const uint2 *>(&Bs[buf][k][tx * 4]);
+            const uint2 b1 = *reinterpret_cast<const uint2 *>(&Bs[buf][k][64 + tx * 4]);
+            unsigned short a[8], b[8];
+            halves(a0.x, a[0], a[1]);
+            halves(a0.y, a[2], a[3]);
+            halves(a1.x, a[4], a[5]);
+            halves(a1.y, a[6], a[7]);
+            halves(b0.x, b[0], b[1]);
+            halves(b0.y, b[2], b[3]);
+            halves(b1.x, b[4], b[5]);
+            halves(b1.y, b[6], b[7]);
 #pragma unroll
             for (int j = 0; j < 8; ++j)
 #pragma unroll
-                for (int i = 0; i < 8; ++i) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+                for (int i = 0; i < 8; ++i) fma_mixed<F16>(acc[i][j], a[i], b[j]);
         }
         if (more) {
             const int nb = buf ^ 1;
@@ -315,9 +329,8 @@ bool whole_tiles(int64_t M, int64_t N, int64_t K, bool a_vec, bool b_vec, bool c
 template <bool F16>
 cudaError_t launch_whole(const uint16_t *a, int64_t lda, const uint16_t *b, int64_t ldb, float *c, int64_t ldc,
                          int64_t M, int64_t N, int64_t K, cudaStream_t s) {
-    constexpr size_t smem = (size_t)2 * 16 * (TM + 128) * sizeof(float);
     dim3 grid((unsigned)(N / 128), (unsigned)(M / TM));
-    gemm_ref_whole<F16><<<grid, 256, smem, s>>>(a, lda, b, ldb, c, ldc, (int)K);
+    gemm_ref_whole<F16><<<grid, 256, 0, s>>>(a, lda, b, ldb, c, ldc, (int)K);
     return cudaGetLastError();
 }
 
