@@ -422,6 +422,22 @@ def candidate_roofline(w, mean_ms: float, peaks) -> dict:
             "kernel": "softmax_rows_reg", "algorithmic_bytes_per_launch": w.candidate_bytes}
 
 
+def fma_rate(n_sm: int, stream) -> dict:
+    """The FP32 FMA pipe's rate measured with the library's probe (16
+    independent FMA chains per thread, 8 blocks of 256 threads per SM), as
+    TFLOP/s: the measured counterpart of the derived FMA peak."""
+    import torch
+    import paper_2609_30057_gb300 as krex
+    blocks, iters = n_sm * 8, 4096
+    sink = torch.empty(blocks * 256, dtype=torch.float32, device="cuda")
+    fn = lambda: krex.krex_probe_fma(iters, blocks, sink, stream=stream)  # noqa: E731
+    for _ in range(3):
+        fn()
+    ms = _time_launches(fn, 10, stream)
+    flops = 2 * 16 * iters * blocks * 256
+    return {"ms": ms, "TFLOP/s": flops / ms / 1e9, "blocks": blocks, "iters": iters}
+
+
 def reference_kernel(w) -> str:
     """The reference GEMM kernel the library runs for this shape: one output
     per thread for at most 16 tiles of 128x128, the unchecked kernel for
@@ -433,10 +449,10 @@ def reference_kernel(w) -> str:
     return "gemm_ref_simt"
 
 
-def reference_roofline(w, mean_ms: float, n_sm: int, sm_mhz) -> dict | None:
+def reference_roofline(w, mean_ms: float, n_sm: int, sm_mhz, fma_measured=None) -> dict | None:
     """The CUDA-core reference GEMM on the FP32 fused multiply-add pipe: peak =
     SMs x 128 FMA lanes x 2 flops x clock (the 2070 MHz maximum; also at the
-    median SM clock sampled during the run)."""
+    median SM clock sampled during the run), beside the probe's measured rate."""
     if not w.is_gemm:
         return None
     achieved = w.flops / (mean_ms / 1e3) / 1e12
@@ -447,6 +463,9 @@ def reference_roofline(w, mean_ms: float, n_sm: int, sm_mhz) -> dict | None:
          "kernel": reference_kernel(w), "algorithmic_flops_per_launch": w.flops, "ms_per_launch": mean_ms}
     if sm_mhz:
         r["frac_at_sampled_clock"] = achieved / (peak * sm_mhz / 2070.0)
+    if fma_measured:
+        r["peak_measured"] = fma_measured["TFLOP/s"]
+        r["frac_of_measured"] = achieved / fma_measured["TFLOP/s"]
     return r
 
 
@@ -629,7 +648,8 @@ def main():
                 "ms_per_command": elapsed / args.steps}
     rl_c = candidate_roofline(w, statistics.fmean(cand_ms), peaks)
     rl_c["launches_timed"] = len(cand_ms)
-    rl_r = reference_roofline(w, ph[1], n_sm, cs.get("sm_mhz") if cs else None)
+    rl_r = reference_roofline(w, ph[1], n_sm, cs.get("sm_mhz") if cs else None,
+                              fma_rate(n_sm, stream) if w.is_gemm else None)
     if rl_r:
         rl_r["launches_timed"] = len(phases)
     # device time per command of each GEMM: the candidate runs once for the

@@ -485,6 +485,15 @@ krex_status krex_host_free(void *ptr, size_t bytes);
 krex_status krex_probe_generator(int32_t dist, uint64_t n_elements, int32_t blocks, float sigma, void *dev_sink,
                                  krex_stream_t stream);
 
+/* Measurement probe, not part of the paper's method: the FP32 fused
+ * multiply-add pipe's rate, for the CUDA-core reference GEMM's roofline.
+ * `blocks` blocks of 256 threads each run `iters` rounds of 16 independent
+ * fp32 FMAs (2 * 16 * iters flops per thread) and store nothing but what keeps
+ * the chains live.  dev_sink: device memory of at least blocks * 256 * 4 bytes
+ * (contents afterwards unspecified).  Asynchronous.  Errors: INVALID for a
+ * null sink, blocks < 1 or iters < 1. */
+krex_status krex_probe_fma(int32_t iters, int32_t blocks, void *dev_sink, krex_stream_t stream);
+
 /* ------------------------------------------------------------ tuning ----- */
 
 /* The kernels' launch configuration, process-wide.  The library never reads

@@ -114,6 +114,7 @@ SIGNATURES = {
     "krex_get_tuning": (_i32, [_P(krex_tuning)]),
     "krex_debug_stall_handover": (_i32, [_i32]),
     "krex_probe_generator": (_i32, [_i32, _u64, _i32, _f32, _vp, _vp]),
+    "krex_probe_fma": (_i32, [_i32, _i32, _vp, _vp]),
     "krex_host_alloc": (_i32, [_sz, _P(_vp)]),
     "krex_host_free": (_i32, [_vp, _sz]),
     "krex_gate_shared_bytes": (_sz, [_i32]),
@@ -484,6 +485,12 @@ def krex_probe_generator(dist: int, n_elements: int, blocks: int, sink, sigma: f
     least blocks * 256 * 4 bytes."""
     _ok(lib().krex_probe_generator(dist, n_elements, blocks, sigma, sink.data_ptr(), _stream(stream)),
         "krex_probe_generator")
+
+
+def krex_probe_fma(iters: int, blocks: int, sink, stream=None):
+    """Launch the FP32 FMA-rate probe (asynchronous); sink: a device tensor of
+    at least blocks * 256 * 4 bytes."""
+    _ok(lib().krex_probe_fma(iters, blocks, sink.data_ptr(), _stream(stream)), "krex_probe_fma")
 
 
 def host_buffer(shape, dtype):

@@ -855,6 +855,15 @@ krex_status krex_probe_generator(int32_t dist, uint64_t n_elements, int32_t bloc
     return ok();
 }
 
+krex_status krex_probe_fma(int32_t iters, int32_t blocks, void *dev_sink, krex_stream_t stream) {
+    if (!dev_sink || blocks < 1 || iters < 1)
+        return set_error(KREX_ERR_INVALID, "probe_fma: need a sink, blocks >= 1, iters >= 1");
+    KREX_CUDA_TRY(launch_fma_probe(iters, blocks, static_cast<float *>(dev_sink),
+                                   reinterpret_cast<cudaStream_t>(stream)));
+    count_launches(1);
+    return ok();
+}
+
 void krex_tuning_defaults(krex_tuning *t) {
     if (t) *t = default_tuning();
 }

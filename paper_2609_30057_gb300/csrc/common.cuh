@@ -27,6 +27,9 @@ cudaError_t launch_fill_normal_f32(uint64_t key, float sigma, float *out, int64_
 // 256 threads, folding instead of storing (sink: one word per thread).
 cudaError_t launch_generator_probe(int32_t dist, uint64_t key, int64_t n, float sigma, int blocks, uint32_t *sink,
                                    cudaStream_t s);
+// Probe: `blocks` x 256 threads, each `iters` rounds of 16 independent fp32
+// FMAs (2 x 16 x iters flops per thread).
+cudaError_t launch_fma_probe(int iters, int blocks, float *sink, cudaStream_t s);
 // K3: grid-stride writer of `bytes` bytes of `value`.
 cudaError_t launch_flush(void *p, size_t bytes, uint32_t value, cudaStream_t s);
 // K6: compare-and-reduce; result (16 bytes) lands in scratch, whose 32-byte

@@ -206,3 +206,11 @@ def test_host_alloc_rejects_bad_arguments():
     assert lib.krex_host_alloc(0, ctypes.byref(p)) == krex.KREX_ERR_INVALID
     assert lib.krex_host_alloc(4096, None) == krex.KREX_ERR_INVALID
     assert lib.krex_host_free(None, 4096) == krex.KREX_ERR_INVALID
+
+
+def test_fma_probe_rejects_bad_arguments():
+    import paper_2609_30057_gb300 as krex
+    lib = krex.lib()
+    assert lib.krex_probe_fma(16, 1, None, None) == krex.KREX_ERR_INVALID
+    assert lib.krex_probe_fma(0, 1, 16, None) == krex.KREX_ERR_INVALID
+    assert lib.krex_probe_fma(16, 0, 16, None) == krex.KREX_ERR_INVALID

@@ -476,3 +476,12 @@ def test_k_direction_alternating_by_wave(M, N, K, alternate):
         c0 = _candidate(a, b)
         same = (c0.view(torch.int16) == c.view(torch.int16)).float().mean().item()
         assert same > 0.5
+
+
+def test_fma_probe_runs_and_leaves_the_context_clean():
+    n_sm = torch.cuda.get_device_properties(0).multi_processor_count
+    sink = torch.zeros(n_sm * 256, dtype=torch.float32, device="cuda")
+    krex.krex_probe_fma(256, n_sm, sink)
+    torch.cuda.synchronize()
+    assert krex.krex_device_status() == 0
+    assert torch.count_nonzero(sink).item() == 0     # the sum is never the stored value
