@@ -2,7 +2,7 @@
 """Benchmark: whole benchmarking commands per second on GB300.
 
 A step is one benchmarking command (the paper's Section 2.1): generate the
-seeded inputs, run the reference, run the candidate once, check it, then time
+seeded inputs, run the candidate once and the reference, check it, then time
 the candidate in a critical region (drain, L2 flush, warm-up, timed
 iterations each preceded by an L2-flush write).  Every step is one
 ``krex_command_run`` call into libkrex.so.

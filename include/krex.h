@@ -436,15 +436,20 @@ typedef struct {
     int32_t launches;          /* kernels this command launched */
     int32_t reserved;
     double phase_ms[5];        /* inputs, reference, candidate, check: device time between CUDA
-                                  events (the four run back to back; the check's ends when its
-                                  verdict is on the host); timed loop: host wall time */
+                                  events (they run back to back in the order inputs, candidate,
+                                  reference, check; the check's ends when its verdict is on the
+                                  host); timed loop: host wall time */
 } krex_command_result;
 
-/* Run one command.  host_in (may be NULL): if given, host_in[i] (pinned host
- * memory, rows*cols contiguous elements of in[i]) is copied to the device
- * instead of generating the inputs.  host_out (may be NULL): if given, the
- * candidate output is copied back to it (rows*cols contiguous elements) after
- * the timed loop.  durations_ms (may be NULL) receives the `iters` timed
+/* Run one command (Section 2.1): inputs, the candidate once, the reference,
+ * the check, then (if it passed) the timed loop in a critical region.
+ * host_in (may be NULL): if given, host_in[i] (page-locked host memory, e.g.
+ * from krex_host_alloc; rows*cols contiguous elements of in[i]) is copied to
+ * the device instead of generating the inputs.  host_out (may be NULL): if
+ * given, the output of the candidate's checked run (rows*cols contiguous
+ * elements; the timed runs write the same values) is copied back to it on a
+ * side stream while the reference runs, and the copy is complete before the
+ * timed region starts.  durations_ms (may be NULL) receives the `iters` timed
  * durations.  A failing check skips the timed loop (passed = 0, n_iters = 0)
  * and still returns KREX_OK: the verdict is the result.  SYNCHRONISES. */
 krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *bufs,

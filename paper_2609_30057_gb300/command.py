@@ -1,7 +1,7 @@
 """Benchmarking-command workloads and a device workspace for them.
 
 A workload is one benchmarking command of the paper's Section 2.1 (generate
-seeded inputs, run the reference, run the candidate once, check it, then time
+seeded inputs, run the candidate once and the reference, check it, then time
 it in a flushed warm-up + timed loop).  The workloads below are named by
 what they are; sizes, seeds and iteration counts are part of the workload
 (the last one is a smaller softmax for full ncu captures).

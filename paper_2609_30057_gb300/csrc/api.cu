@@ -672,16 +672,26 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
     // between them (a host synchronisation per phase would add an idle gap to
     // each); the check ends by reading its verdict back to the host, and its
     // phase ends with an event recorded after that.  The timed loop is host
-    // wall time.
+    // wall time.  The candidate's checked run comes before the reference, so
+    // that with host_out its output (the command's result) is copied back on a
+    // side stream while the reference runs; the copy is complete before the
+    // timed region starts, so nothing overlaps the measurement.
     int dev = 0;
     KREX_CUDA_TRY(cudaGetDevice(&dev));
     std::vector<cudaEvent_t> pev;
-    KREX_CUDA_TRY(event_pool().take(dev, 5, pev));
-    struct GiveBack {
+    KREX_CUDA_TRY(event_pool().take(dev, 6, pev));
+    struct Cleanup {
         int dev;
         std::vector<cudaEvent_t> &ev;
-        ~GiveBack() { event_pool().give(dev, ev); }
-    } give_back{dev, pev};
+        cudaStream_t side = nullptr;
+        ~Cleanup() {
+            if (side) {
+                cudaStreamSynchronize(side);  // a copy in flight finishes before anything is released
+                cudaStreamDestroy(side);
+            }
+            event_pool().give(dev, ev);
+        }
+    } cleanup{dev, pev};
     KREX_CUDA_TRY(cudaEventRecord(pev[0], s));
     // 1) inputs: generated on the device, or copied from the caller's host buffers
     for (int i = 0; i < n_in; ++i) {
@@ -698,23 +708,40 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
         }
     }
     KREX_CUDA_TRY(cudaEventRecord(pev[1], s));
-    // 2) reference
-    if ((st = do_reference(op, bufs->in, bufs->ref, s))) return st;
-    KREX_CUDA_TRY(cudaEventRecord(pev[2], s));
-    // 3) candidate once, for the check
+    // 2) candidate once, for the check
     if ((st = do_candidate(op, bufs->in, bufs->out, s, bufs->gemm_workspace, bufs->gemm_workspace_bytes))) return st;
+    KREX_CUDA_TRY(cudaEventRecord(pev[2], s));
+    if (host_out) {
+        // the result back to the host while the reference runs
+        KREX_CUDA_TRY(cudaStreamCreateWithFlags(&cleanup.side, cudaStreamNonBlocking));
+        KREX_CUDA_TRY(cudaStreamWaitEvent(cleanup.side, pev[2], 0));
+        const krex_buf &b = bufs->out;
+        const size_t es = elem_size(b.dtype);
+        KREX_CUDA_TRY(copy_rows(host_out, (size_t)b.cols * es, b.ptr, (size_t)b.ld * es, (size_t)b.cols * es,
+                                (size_t)b.rows, cudaMemcpyDeviceToHost, cleanup.side));
+        KREX_CUDA_TRY(cudaEventRecord(pev[5], cleanup.side));
+    }
+    // 3) reference
+    if ((st = do_reference(op, bufs->in, bufs->ref, s))) return st;
     KREX_CUDA_TRY(cudaEventRecord(pev[3], s));
-    // 4) check (synchronous: every earlier phase has completed when it returns)
+    // 4) check (synchronous: every earlier phase on the stream has completed when it returns)
     if ((st = krex_check(bufs->out, bufs->ref, cmd->atol, cmd->rtol, bufs->check_scratch, bufs->check_scratch_bytes,
                          &result->check, stream)))
         return st;
     KREX_CUDA_TRY(cudaEventRecord(pev[4], s));
     KREX_CUDA_TRY(cudaEventSynchronize(pev[4]));
-    for (int i = 0; i < 4; ++i) {
+    {
         float ms = 0.0f;
-        KREX_CUDA_TRY(cudaEventElapsedTime(&ms, pev[i], pev[i + 1]));
-        result->phase_ms[i] = ms;
+        KREX_CUDA_TRY(cudaEventElapsedTime(&ms, pev[0], pev[1]));
+        result->phase_ms[0] = ms;  // inputs
+        KREX_CUDA_TRY(cudaEventElapsedTime(&ms, pev[2], pev[3]));
+        result->phase_ms[1] = ms;  // reference
+        KREX_CUDA_TRY(cudaEventElapsedTime(&ms, pev[1], pev[2]));
+        result->phase_ms[2] = ms;  // candidate
+        KREX_CUDA_TRY(cudaEventElapsedTime(&ms, pev[3], pev[4]));
+        result->phase_ms[3] = ms;  // check
     }
+    if (host_out) KREX_CUDA_TRY(cudaEventSynchronize(pev[5]));  // the copy back is done
     result->passed = result->check.n_violations == 0;
     // 5) timed loop inside a critical region (skipped when the check failed)
     const auto t = clk::now();
@@ -735,13 +762,6 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
         result->n_iters = cmd->iters;
     }
     result->phase_ms[4] = ms_since(t);
-    if (host_out) {
-        const krex_buf &b = bufs->out;
-        const size_t es = elem_size(b.dtype);
-        KREX_CUDA_TRY(copy_rows(host_out, (size_t)b.cols * es, b.ptr, (size_t)b.ld * es, (size_t)b.cols * es,
-                                (size_t)b.rows, cudaMemcpyDeviceToHost, s));
-        KREX_CUDA_TRY(cudaStreamSynchronize(s));
-    }
     result->launches = (int32_t)(g_launches.load() - launches0);
     return ok();
 }
