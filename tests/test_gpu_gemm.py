@@ -485,3 +485,41 @@ def test_fma_probe_runs_and_leaves_the_context_clean():
     torch.cuda.synchronize()
     assert krex.krex_device_status() == 0
     assert torch.count_nonzero(sink).item() == 0     # the sum is never the stored value
+
+
+@pytest.mark.parametrize("f16", [False, True], ids=["bf16", "f16"])
+def test_reference_whole_tile_form_keeps_special_values(f16):
+    # the whole-tile reference multiplies 16-bit operands with the mixed-precision
+    # FMA; with subnormal operands, signed zeros, infinite operands (inf x 0
+    # gives NaN) and (bf16) products that overflow to +-inf it still equals the
+    # checked form (operands widened to fp32 first) bit for bit, NaN for NaN
+    M, N, K = 640, 640, 64          # 25 tiles of 128 x 128: the tiled (whole-tile) form, not the small one
+    g = inputs.rng(11)
+    if f16:
+        vals = np.array([0.0, -0.0, 2.0 ** -24, -(2.0 ** -20), 2.0 ** -14, 1.0, -2.0, 60000.0, -60000.0],
+                        dtype=np.float32)
+        enc, dec, tt = gen.f32_to_f16, gen.f16_to_f32, to_f16_tensor
+        op = krex.KREX_OP_GEMM_F16
+    else:
+        vals = np.array([0.0, -0.0, 2.0 ** -130, -(2.0 ** -126), 2.0 ** -133, 1.0, -3.0, 2.0 ** 120, -(2.0 ** 121)],
+                        dtype=np.float32)
+        enc, dec, tt = gen.f32_to_bf16, gen.bf16_to_f32, to_bf16_tensor
+        op = krex.KREX_OP_GEMM_BF16
+    a_bits = enc(g.choice(vals, size=M * K)).reshape(M, K)
+    b_bits = enc(g.choice(vals, size=K * N)).reshape(K, N)
+    assert np.array_equal(dec(enc(vals)), vals)                 # every value is exact in the 16-bit format
+    # infinite operands in one row of A and one column of B: inf x 0 = NaN there
+    a_bits[3, 5] = enc(np.array([np.inf], dtype=np.float32))[0]
+    b_bits[10, 20] = enc(np.array([-np.inf], dtype=np.float32))[0]
+    a, b = tt(a_bits), tt(b_bits)
+    r_whole = torch.empty(M, N, dtype=torch.float32, device="cuda")
+    krex.krex_run_reference(op, [a, b], r_whole)
+    wide = torch.zeros(M, K + 3, dtype=a.dtype, device="cuda")
+    wide[:, :K] = a
+    r_chk = torch.empty(M, N, dtype=torch.float32, device="cuda")
+    krex.krex_run_reference(op, [wide[:, :K], b], r_chk)       # odd row stride: the checked form
+    torch.cuda.synchronize()
+    x, y = r_whole.cpu().numpy(), r_chk.cpu().numpy()
+    nan = np.isnan(x)
+    assert np.array_equal(nan, np.isnan(y)) and nan.any() and np.isinf(x).any() and np.isfinite(x).any()
+    assert np.array_equal(x[~nan].view(np.uint32), y[~nan].view(np.uint32))
