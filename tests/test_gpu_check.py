@@ -158,3 +158,16 @@ def test_scratch_init_rejects_small_or_unaligned_buffers():
     assert lib.krex_check_scratch_init(buf.data_ptr() + 8, krex.krex_check_scratch_bytes(),
                                        None) == krex.KREX_ERR_UNSUPPORTED
     assert lib.krex_check_scratch_init(None, krex.krex_check_scratch_bytes(), None) == krex.KREX_ERR_INVALID
+
+
+def test_consecutive_checks_alternate_slots_and_stay_exact():
+    # each call uses the result slot of its parity and readies the other: seven
+    # calls in a row on one scratch, interleaved with calls on a second scratch,
+    # with inputs whose results all differ, each equal to the oracle's check
+    s1 = torch.zeros(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
+    s2 = torch.zeros(krex.krex_check_scratch_bytes(), dtype=torch.uint8, device="cuda")
+    for i in range(7):
+        o = inputs.normal_f32(100 + i, (257, 1000 + 37 * i))
+        r = inputs.perturbed(o, 200 + i, 0.05 * (i + 1), 10.0 ** -(i % 4 + 2))
+        for sc in (s1, s2) if i % 2 else (s1,):
+            _run(o, r, 1e-4, 1e-3, sc)

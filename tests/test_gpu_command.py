@@ -175,3 +175,18 @@ def test_command_with_library_host_buffers():
         r = ws.run(host_in=[h.data_ptr() for h in hin], host_out=hout.data_ptr())
         assert r.passed == 1
         assert np.array_equal(hout.view(torch.int16).numpy().view(np.uint16), want)
+
+
+@pytest.mark.parametrize("nbytes", [1, 4096, (2 << 20) + 3, (96 << 20) + 12345])
+def test_host_buffer_sizes_round_trip(nbytes):
+    # krex_host_alloc buffers of any size (the mapping is rounded up to whole
+    # huge pages): page-locked, and a copy to the device and back is exact
+    h = krex.host_buffer((nbytes,), torch.uint8)
+    assert h.is_pinned() and h.numel() == nbytes
+    g = np.random.default_rng(nbytes).integers(0, 256, nbytes, dtype=np.uint8)
+    h.copy_(torch.from_numpy(g))
+    d = h.to("cuda", non_blocking=True)
+    back = krex.host_buffer((nbytes,), torch.uint8)
+    back.copy_(d, non_blocking=True)
+    torch.cuda.synchronize()
+    assert np.array_equal(back.numpy(), g)

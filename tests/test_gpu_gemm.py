@@ -523,3 +523,14 @@ def test_reference_whole_tile_form_keeps_special_values(f16):
     nan = np.isnan(x)
     assert np.array_equal(nan, np.isnan(y)) and nan.any() and np.isinf(x).any() and np.isfinite(x).any()
     assert np.array_equal(x[~nan].view(np.uint32), y[~nan].view(np.uint32))
+
+
+@pytest.mark.parametrize("alternate", [0, 1], ids=["forward", "alternating"])
+def test_f16_k_direction_alternating_by_wave(alternate):
+    krex.krex_set_tuning(gemm_k_alternate=alternate)
+    M, N, K = 3072, 3072, 1032
+    seed = 8100 + alternate
+    a, b = _gen16(seed, M, N, K)
+    want = ref.gemm_f64(gen.uniform_f16(seed, 0, M, K), gen.uniform_f16(seed, 1, K, N), dtype="f16")
+    ok, worst = _within_tol16(bits16(_candidate16(a, b)), want, K)
+    assert ok, worst
