@@ -181,11 +181,19 @@ gemm_ref_simt(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__res
 // output is the same k-order FMA chain as in gemm_ref_simt (identical bits),
 // with half the shared-memory traffic and fragment registers and no
 // conversion in the slice staging.  No bounds checks, one 16-byte load of A
-// and one of B per thread and slice, a 32-bit K loop, 8 x 8 outputs per
-// thread swept column by column.  Measured on GB300 in one process (TFLOP/s
-// at 4096^3 / 16384^3, L2 flushed): 64.4 / 67.6, against 58.8 / 60.4 for the
-// same tiling with operands widened to fp32 in shared memory and 55.0 / 57.0
-// for gemm_ref_simt.
+// and one of B per thread and slice, a 32-bit K loop.  Each thread owns 8
+// consecutive rows x 8 consecutive columns, so its per-k operands are one
+// 16-byte shared load of A (two distinct addresses per warp) and one of B
+// (256 contiguous bytes per warp), swept column by column.  Measured on GB300
+// in one process (TFLOP/s at 4096^3 / 16384^3, L2 flushed): 65.5 / 68.7,
+// against 64.3 / 67.4 with the 4x4-block ownership of gemm_ref_simt (two
+// 8-byte loads of each operand per k), 58.8 / 60.4 with operands widened to
+// fp32 in shared memory and 55.0 / 57.0 for gemm_ref_simt.  Also measured and
+// dropped here: 128x256 and 256x128 tiles with 8x16 / 16x8 outputs per thread
+// (one block per SM: 52-55 / 61-65), 32-deep slices (58-60 / 61-64), raster
+// groups of 8 or 32 rows (no change), and the slices brought in by TMA
+// through an mbarrier ring with operand rows kept m-major (no block barrier,
+// no staging: 53 / 56).
 template <bool F16>
 __device__ __forceinline__ void fma_mixed(float &acc, unsigned short a, unsigned short b) {
     if constexpr (F16) asm("fma.rn.f32.f16 %0, %1, %2, %0;" : "+f"(acc) : "h"(a), "h"(b));
@@ -251,19 +259,17 @@ gemm_ref_whole(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__re
         if (more) fetch(k0 + TK);  // the next slice comes in while this one is multiplied
 #pragma unroll
         for (int k = 0; k < TK; ++k) {
-            const uint2 a0 = *reinterpret_cast<const uint2 *>(&As[buf][k][ty * 4]);
-            const uint2 a1 = *reinterpret_cast<const uint2 *>(&As[buf][k][64 + ty * 4]);
-            const uint2 b0 = *reinterpret_cast<const uint2 *>(&Bs[buf][k][tx * 4]);
-            const uint2 b1 = *reinterpret_cast<const uint2 *>(&Bs[buf][k][64 + tx * 4]);
+            const uint4 av = *reinterpret_cast<const uint4 *>(&As[buf][k][ty * 8]);
+            const uint4 bv = *reinterpret_cast<const uint4 *>(&Bs[buf][k][tx * 8]);
             unsigned short a[8], b[8];
-            halves(a0.x, a[0], a[1]);
-            halves(a0.y, a[2], a[3]);
-            halves(a1.x, a[4], a[5]);
-            halves(a1.y, a[6], a[7]);
-            halves(b0.x, b[0], b[1]);
-            halves(b0.y, b[2], b[3]);
-            halves(b1.x, b[4], b[5]);
-            halves(b1.y, b[6], b[7]);
+            halves(av.x, a[0], a[1]);
+            halves(av.y, a[2], a[3]);
+            halves(av.z, a[4], a[5]);
+            halves(av.w, a[6], a[7]);
+            halves(bv.x, b[0], b[1]);
+            halves(bv.y, b[2], b[3]);
+            halves(bv.z, b[4], b[5]);
+            halves(bv.w, b[6], b[7]);
 #pragma unroll
             for (int j = 0; j < 8; ++j)
 #pragma unroll
@@ -278,9 +284,9 @@ gemm_ref_whole(const uint16_t *__restrict__ A, int64_t lda, const uint16_t *__re
     }
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
-        float *cr = C + (m0 + (i < 4 ? ty * 4 + i : 64 + ty * 4 + (i - 4))) * ldc;
-        *reinterpret_cast<float4 *>(cr + n0 + tx * 4) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
-        *reinterpret_cast<float4 *>(cr + n0 + 64 + tx * 4) = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
+        float *cr = C + (m0 + ty * 8 + i) * ldc + n0 + tx * 8;
+        *reinterpret_cast<float4 *>(cr) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+        *reinterpret_cast<float4 *>(cr + 4) = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
     }
 }
 
