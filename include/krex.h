@@ -443,9 +443,16 @@ typedef struct {
 
 /* Run one command (Section 2.1): inputs, the candidate once, the reference,
  * the check, then (if it passed) the timed loop in a critical region.
- * host_in (may be NULL): if given, host_in[i] (page-locked host memory, e.g.
- * from krex_host_alloc; rows*cols contiguous elements of in[i]) is copied to
- * the device instead of generating the inputs.  host_out (may be NULL): if
+ * host_in (may be NULL): if given, host_in[i] (host memory, e.g. from
+ * krex_host_alloc; rows*cols contiguous elements of in[i]) is copied to the
+ * device instead of generating the inputs: by a copy kernel (SM loads over
+ * the host link, one launch per operand) when the device reads the buffer
+ * directly at the same address (page-locked, mapped, registered over the
+ * whole copy) and the buffer, in[i] and their row pitches are multiples of 16
+ * bytes; otherwise by the copy engine (pageable memory included, no launch).
+ * On GB300 the kernel reads as fast as the copy engine from huge pages and
+ * stays at that rate from 64 KiB pages, where a copy-engine read after a
+ * pause slowed to 12-14 GB/s (see krex_host_alloc).  host_out (may be NULL): if
  * given, the output of the candidate's checked run (rows*cols contiguous
  * elements; the timed runs write the same values) is copied back to it on a
  * side stream while the reference runs, and the copy is complete before the
@@ -469,8 +476,12 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
  * copy took 2.6 ms back to back but 15-90 ms after a pause of a quarter
  * second, every other time, with memory pinned by cudaHostAlloc or by
  * registering an unadvised mapping; with huge pages it took 2.6 ms every
- * time.  bytes > 0; *ptr receives the buffer (zero-filled).  Free it with
- * krex_host_free(ptr, bytes).  Errors: INVALID for a null ptr or zero bytes,
+ * time.  (krex_command_run now reads page-locked inputs with SM loads, which
+ * showed no such slowdown; huge pages still help the copy engine's reads.)
+ * The host grants a huge page only where it finds that much contiguous free
+ * memory (512 MiB on a 64 KiB-page kernel); a buffer without them works the
+ * same, at those rates.  bytes > 0; *ptr receives the buffer (zero-filled).
+ * Free it with krex_host_free(ptr, bytes).  Errors: INVALID for a null ptr or zero bytes,
  * CUDA if registration fails (nothing stays allocated then). */
 krex_status krex_host_alloc(size_t bytes, void **ptr);
 krex_status krex_host_free(void *ptr, size_t bytes);

@@ -22,7 +22,7 @@ BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libkrex.so")
 
 SOURCES = ["api.cu", "gate.cu", "xproc.cu", "fill.cu", "flush_check.cu", "softmax.cu", "gemm_ref.cu", "probe.cu",
-           "gemm_tcgen05.cu"]
+           "host_copy.cu", "gemm_tcgen05.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", *ARCH, "-Xcompiler", "-fPIC,-ffp-contract=off",
               "-I", INCLUDE, "-I", CSRC]

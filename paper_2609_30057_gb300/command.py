@@ -96,7 +96,9 @@ def scaled(w: Workload, **kw) -> Workload:
 class Workspace:
     """Caller-owned device buffers of one workload (allocated with torch)."""
 
-    def __init__(self, w: Workload, device="cuda"):
+    def __init__(self, w: Workload, device="cuda", inputs=None):
+        """``inputs``: the caller's own device tensors for the operands (any
+        row stride), instead of contiguous new ones."""
         import torch
         self.w = w
         f32 = torch.float32
@@ -108,6 +110,11 @@ class Workspace:
         else:
             self.inputs = [torch.empty(w.M, w.N, dtype=f32, device=device)]
             self.out = torch.empty(w.M, w.N, dtype=f32, device=device)
+        if inputs is not None:
+            if len(inputs) != len(self.inputs) or any(
+                    a.shape != b.shape or a.dtype != b.dtype for a, b in zip(inputs, self.inputs)):
+                raise ValueError("inputs must match the workload's operand shapes and dtypes")
+            self.inputs = list(inputs)
         self.ref = torch.empty(w.M, w.N, dtype=f32, device=device)
         self.flush = torch.empty(max(w.flush_bytes, 16), dtype=torch.uint8, device=device)
         self.check_scratch = torch.zeros(krex_check_scratch_bytes(), dtype=torch.uint8, device=device)

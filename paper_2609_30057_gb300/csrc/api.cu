@@ -641,6 +641,62 @@ static cudaError_t copy_rows(void *dst, size_t dpitch, const void *src, size_t s
     return cudaMemcpy2DAsync(dst, dpitch, src, spitch, width, rows, kind, s);
 }
 
+// The driver's cuPointerGetAttribute, through the runtime's entry-point query
+// (the library links no driver library); nullptr if the driver lacks it.
+typedef CUresult (*PointerAttrFn)(void *, CUpointer_attribute, CUdeviceptr);
+static PointerAttrFn pointer_attr_fn() {
+    static PointerAttrFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuPointerGetAttribute", &p, 4000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PointerAttrFn>(p);
+    });
+    return fn;
+}
+
+// True if the device can read all `bytes` at host address p directly, at the
+// same address: page-locked memory mapped into the device's address space
+// (cudaHostRegister / cudaHostAlloc) whose registered range covers the bytes.
+// Anything else (pageable memory, a range that ends early, a device-side
+// address that differs) is copied by the copy engine.
+static bool device_reads_host(const void *p, size_t bytes) {
+    cudaPointerAttributes a;
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    if (a.type != cudaMemoryTypeHost || a.devicePointer != p) return false;
+    PointerAttrFn get = pointer_attr_fn();
+    if (!get) return false;
+    CUdeviceptr start = 0;
+    size_t size = 0;
+    const CUdeviceptr at = reinterpret_cast<CUdeviceptr>(p);
+    if (get(&start, CU_POINTER_ATTRIBUTE_RANGE_START_ADDR, at) != CUDA_SUCCESS ||
+        get(&size, CU_POINTER_ATTRIBUTE_RANGE_SIZE, at) != CUDA_SUCCESS)
+        return false;
+    return at >= start && bytes <= size && at - start <= size - bytes;
+}
+
+// Rows from a caller's host buffer into device memory: SM loads when the
+// device reads the buffer directly (see host_copy.cu for why), else the copy
+// engine.  *kernel counts the launches.
+static cudaError_t copy_rows_in(void *dst, size_t dpitch, const void *src, size_t spitch, size_t width, size_t rows,
+                                cudaStream_t s, int *kernel) {
+    if (rows > 0 && width > 0 && device_reads_host(src, spitch * (rows - 1) + width)) {
+        bool launched = false;
+        cudaError_t e = launch_copy_rows_from_host(src, spitch, dst, dpitch, width, rows, s, &launched);
+        if (e != cudaSuccess || launched) {
+            *kernel += e == cudaSuccess;
+            return e;
+        }
+    }
+    return copy_rows(dst, dpitch, src, spitch, width, rows, cudaMemcpyHostToDevice, s);
+}
+
 krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *bufs, const void *const *host_in,
                              void *host_out, float *durations_ms, krex_command_result *result,
                              krex_stream_t stream) {
@@ -698,8 +754,10 @@ krex_status krex_command_run(const krex_command *cmd, const krex_command_bufs *b
         const krex_buf &b = bufs->in[i];
         if (host_in && host_in[i]) {
             const size_t es = elem_size(b.dtype);
-            KREX_CUDA_TRY(copy_rows(b.ptr, (size_t)b.ld * es, host_in[i], (size_t)b.cols * es, (size_t)b.cols * es,
-                                    (size_t)b.rows, cudaMemcpyHostToDevice, s));
+            int kernels = 0;
+            KREX_CUDA_TRY(copy_rows_in(b.ptr, (size_t)b.ld * es, host_in[i], (size_t)b.cols * es,
+                                       (size_t)b.cols * es, (size_t)b.rows, s, &kernels));
+            count_launches(kernels);
         } else {
             st = is_gemm(op)
                      ? krex_gen_inputs(cmd->seed, (uint32_t)i, KREX_DIST_UNIFORM_PM1, 0.0f, b, stream)

@@ -30,6 +30,12 @@ cudaError_t launch_generator_probe(int32_t dist, uint64_t key, int64_t n, float 
 // Probe: `blocks` x 256 threads, each `iters` rounds of 16 independent fp32
 // FMAs (2 x 16 x iters flops per thread).
 cudaError_t launch_fma_probe(int iters, int blocks, float *sink, cudaStream_t s);
+// Rows of `width` bytes from a host buffer the device reads directly (src is
+// its device-side address) into device memory, by SM loads.  Launches only
+// when src, dst, both pitches and width are multiples of 16 bytes; *launched
+// tells the caller whether to copy another way.
+cudaError_t launch_copy_rows_from_host(const void *src, size_t spitch, void *dst, size_t dpitch, size_t width,
+                                       size_t rows, cudaStream_t s, bool *launched);
 // K3: grid-stride writer of `bytes` bytes of `value`.
 cudaError_t launch_flush(void *p, size_t bytes, uint32_t value, cudaStream_t s);
 // K6: compare-and-reduce; result (16 bytes) lands in scratch, whose 32-byte

@@ -60,6 +60,51 @@ def test_command_with_host_buffers_equals_device_generated():
     assert np.array_equal(bits16(ws.out), dev_out)      # same inputs either way: same output
 
 
+@pytest.mark.parametrize("route", ["pinned", "pinned_strided_device_rows", "pageable", "pinned_misaligned"])
+def test_command_host_inputs_by_each_copy_route(route):
+    # host inputs reach the device by SM loads when the device reads the
+    # buffer directly (page-locked, registered over the whole copy, 16-byte
+    # words): one copy kernel per operand in place of its fill; else by the
+    # copy engine (no launch).  Every route gives the device-generated output.
+    w = scaled(WORKLOADS["gemm_bf16_256"], M=384, N=512, K=320, iters=3)
+    ws0 = Workspace(w)
+    r0 = ws0.run()
+    assert r0.passed == 1
+    want = bits16(ws0.out)
+    a = gen.uniform_bf16(w.seed, 0, w.M, w.K).view(np.int16)
+    b = gen.uniform_bf16(w.seed, 1, w.K, w.N).view(np.int16)
+    inputs = pads = None
+    if route == "pinned_strided_device_rows":
+        pads = (torch.zeros(w.M, w.K + 8, dtype=torch.bfloat16, device="cuda"),
+                torch.zeros(w.K, w.N + 8, dtype=torch.bfloat16, device="cuda"))
+        inputs = [pads[0][:, :w.K], pads[1][:, :w.N]]
+    ws = Workspace(w, inputs=inputs)
+    if route == "pageable":
+        hosts = [torch.from_numpy(a.copy()), torch.from_numpy(b.copy())]
+        assert not any(h.is_pinned() for h in hosts)
+    elif route == "pinned_misaligned":
+        # 2 bytes past a 16-byte boundary: no 16-byte words, so the copy engine
+        hosts = []
+        for x in (a, b):
+            big = torch.empty(x.size + 8, dtype=torch.int16).pin_memory()
+            v = big[1:1 + x.size].view(x.shape)
+            v.copy_(torch.from_numpy(x))
+            assert v.data_ptr() % 16 == 2
+            hosts.append(v)
+    else:
+        hosts = [torch.from_numpy(a).pin_memory(), torch.from_numpy(b).pin_memory()]
+    hc = torch.empty(w.M, w.N, dtype=torch.int16).pin_memory()
+    res = ws.run(host_in=[h.data_ptr() for h in hosts], host_out=hc.data_ptr())
+    assert res.passed == 1
+    assert np.array_equal(bits16(ws.out), want)
+    assert np.array_equal(hc.numpy().view(np.uint16), want)
+    by_kernel = route in ("pinned", "pinned_strided_device_rows")
+    assert res.launches == r0.launches - (0 if by_kernel else 2)
+    if pads is not None:   # the padding columns of the strided rows are untouched
+        assert not pads[0].view(torch.int16)[:, w.K:].any()
+        assert not pads[1].view(torch.int16)[:, w.N:].any()
+
+
 def test_softmax_command_small():
     w = scaled(WORKLOADS["softmax_f32_65536x8192"], M=512, iters=5)
     ws = Workspace(w)
