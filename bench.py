@@ -544,8 +544,10 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--kernel-only", default=None,
-                    choices=["gemm", "gemm_ref", "fill_uniform", "fill_normal", "flush", "check", "softmax"],
-                    help="launch one kernel of the workload --launches times and exit (for ncu captures)")
+                    choices=["gemm", "gemm_ref", "fill_uniform", "fill_normal", "flush", "check", "softmax",
+                             "cublas"],
+                    help="launch one kernel of the workload --launches times and exit (for ncu captures); "
+                         "cublas: torch.matmul on the same operands, a library comparison outside the command")
     ap.add_argument("--launches", type=int, default=3)
     ap.add_argument("--tuning", action="append", default=[], metavar="FIELD=VALUE",
                     help="with --kernel-only: set a field of the library's tuning record first (repeatable)")
@@ -730,8 +732,10 @@ def kernel_only(args):
     if args.kernel_only in ("softmax", "fill_normal") and WORKLOADS[name].is_gemm:
         name = SOFTMAX_WORKLOAD
     w = WORKLOADS[name]
-    ws = Workspace(w)
     k = args.kernel_only
+    if k == "cublas" and not w.is_gemm:
+        raise SystemExit("--kernel-only cublas needs a GEMM workload")
+    ws = Workspace(w)
     # minimal set-up: inputs, and for the check the two outputs it compares
     if w.is_gemm:
         krex.krex_gen_inputs(w.seed, 0, 0, 0.0, ws.inputs[0], stream)
@@ -749,6 +753,7 @@ def kernel_only(args):
         "flush": lambda: krex.krex_flush_l2(ws.flush, stream=stream),
         "check": lambda: krex.krex_check(ws.out, ws.ref, w.atol, w.rtol, ws.check_scratch, stream),
         "softmax": lambda: krex.krex_run_candidate(1, ws.inputs, ws.out, stream),
+        "cublas": lambda: torch.matmul(ws.inputs[0], ws.inputs[1], out=ws.out),
     }[k]
     for _ in range(args.launches):
         if k != "flush":
