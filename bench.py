@@ -167,18 +167,39 @@ def kernel_table(peaks, stream, gemm_names=(SMALL_GEMM_WORKLOAD, DEFAULT_WORKLOA
     """Each kernel of the path timed alone (after warm-up, L2 flushed before
     every launch), with its algorithmic bytes or flops per launch: the GEMM
     path's kernels at the sizes of `gemm_names`, the softmax path's at its
-    workload's size."""
+    workload's size.  The fills come first and the largest GEMMs last: after
+    seconds of those the power controller holds the SM clock down for a while
+    (GB300, sw_power_cap), which would charge the next kernels for it."""
     import torch
     import paper_2609_30057_gb300 as krex
     from paper_2609_30057_gb300.command import WORKLOADS, Workspace
     out = {}
     dev = torch.cuda.current_device()
     n_sm = torch.cuda.get_device_properties(dev).multi_processor_count
-    # the fills' compute ceilings at the sizes they are timed at
-    ceiling = {0: generator_ceiling(0, n_sm, stream, 16384 * 16384),
-               1: generator_ceiling(1, n_sm, stream, WORKLOADS[SOFTMAX_WORKLOAD].M * WORKLOADS[SOFTMAX_WORKLOAD].N)}
+    # the fills at the headline sizes beside their compute ceilings, first
+    # (before seconds of GEMMs leave the clock under the power cap), each
+    # launched alternately with its generator probe
+    sw = WORKLOADS[SOFTMAX_WORKLOAD]
+    flush_buf = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    flush0 = lambda: krex.krex_flush_l2(flush_buf, stream=stream)  # noqa: E731
+    ceiling, fill_ms = {}, {}
+    big = torch.empty(16384, 16384, dtype=torch.bfloat16, device="cuda")
+    ceiling[0], fill_ms[0] = fill_beside_ceiling(
+        0, n_sm, stream, lambda: krex.krex_gen_inputs(1, 0, 0, 0.0, big, stream), big.numel(), flush0)
+    del big
+    big = torch.empty(sw.M, sw.N, dtype=torch.float32, device="cuda")
+    ceiling[1], fill_ms[1] = fill_beside_ceiling(
+        1, n_sm, stream, lambda: krex.krex_gen_inputs(sw.seed, 0, 1, sw.sigma, big, stream), big.numel(), flush0)
+    del big, flush_buf
+    torch.cuda.empty_cache()
     out["generator_probe_uniform@16384"] = ceiling[0]
     out["generator_probe_normal@65536x8192"] = ceiling[1]
+    for dist, name, nbytes in ((0, "fill_uniform_bf16@16384", 16384 * 16384 * 2),
+                               (1, "fill_normal_f32", sw.M * sw.N * 4)):
+        gbs = nbytes / fill_ms[dist] / 1e6
+        out[name] = {"ms": fill_ms[dist], "launches": 10, "GB/s": gbs, "frac_hbm": gbs / peaks["hbm_gbs"],
+                     "bytes": nbytes, "bound": "alu", "peak_GB/s": ceiling[dist]["GB/s"],
+                     "frac_alu": gbs / ceiling[dist]["GB/s"]}
 
     def rec(name, fn, flush, nbytes=None, flops=None, gen_dist=None, n=20, fma_peak=None):
         for _ in range(3):
@@ -197,38 +218,16 @@ def kernel_table(peaks, stream, gemm_names=(SMALL_GEMM_WORKLOAD, DEFAULT_WORKLOA
                 e.update({"bound": "fp32 fma", "frac_fma": tf * 1e12 / fma_peak})
         if gen_dist is not None:
             # compute-bound generator: its roofline is the measured rate of
-            # its own per-draw arithmetic (generator_ceiling)
+            # its own per-draw arithmetic (fill_beside_ceiling)
             c = ceiling[gen_dist]["GB/s"]
             e.update({"bound": "alu", "peak_GB/s": c, "frac_alu": (nbytes / ms / 1e6) / c})
         out[name] = e
 
-    for gname in gemm_names:
-        w = WORKLOADS[gname]
-        ws = Workspace(w)
-        sfx = f"@{w.M}"
-        flush = lambda ws=ws: krex.krex_flush_l2(ws.flush, stream=stream)  # noqa: E731
-        A, B = ws.inputs
-        rec("fill_uniform_bf16" + sfx, lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, A, stream), flush,
-            nbytes=A.numel() * 2, gen_dist=0, n=10)
-        krex.krex_gen_inputs(w.seed, 1, 0, 0.0, B, stream)
-        if gname == gemm_names[0]:
-            rec("flush_l2", flush, None, nbytes=ws.flush.numel())
-        rec(reference_kernel(w) + sfx, lambda: krex.krex_run_reference(w.op, ws.inputs, ws.ref, stream), flush,
-            flops=w.flops, n=2 if w.M >= 16384 else 10, fma_peak=n_sm * FMA_LANES_PER_SM * 2 * 2.070e9)
-        rec("gemm_tcgen05" + sfx, lambda: krex.krex_run_candidate_ws(w.op, ws.inputs, ws.out, ws.gemm_ws, stream),
-            flush, flops=w.flops, n=10 if w.M >= 16384 else 20)
-        rec("check_bf16_f32" + sfx,
-            lambda: krex.krex_check_launch(ws.out, ws.ref, w.atol, w.rtol, ws.check_scratch, stream), flush,
-            nbytes=ws.out.numel() * 6, n=10)
-        del ws, A, B
-        torch.cuda.empty_cache()
     # the bandwidth-bound candidate at its own workload size
-    sw = WORKLOADS[SOFTMAX_WORKLOAD]
     sws = Workspace(sw)
     flush = lambda: krex.krex_flush_l2(sws.flush, stream=stream)  # noqa: E731
     x, y = sws.inputs[0], sws.out
-    rec("fill_normal_f32", lambda: krex.krex_gen_inputs(sw.seed, 0, 1, sw.sigma, x, stream), flush,
-        nbytes=x.numel() * 4, gen_dist=1, n=10)
+    krex.krex_gen_inputs(sw.seed, 0, 1, sw.sigma, x, stream)
     rec("softmax_f32", lambda: krex.krex_run_candidate(1, [x], y, stream), flush, nbytes=x.numel() * 8, n=10)
     rec("check_f32_f32", lambda: krex.krex_check_launch(y, x, 1e-6, 0.0, sws.check_scratch, stream), flush,
         nbytes=x.numel() * 8, n=5)
@@ -245,26 +244,64 @@ def kernel_table(peaks, stream, gemm_names=(SMALL_GEMM_WORKLOAD, DEFAULT_WORKLOA
         flush, flops=fw.flops)
     del fws, a16, b16
     torch.cuda.empty_cache()
+    for gname in gemm_names:
+        w = WORKLOADS[gname]
+        ws = Workspace(w)
+        sfx = f"@{w.M}"
+        flush = lambda ws=ws: krex.krex_flush_l2(ws.flush, stream=stream)  # noqa: E731
+        A, B = ws.inputs
+        if w.M != 16384:   # (the 16384^2 fill is timed above, beside its ceiling)
+            rec("fill_uniform_bf16" + sfx, lambda: krex.krex_gen_inputs(w.seed, 0, 0, 0.0, A, stream), flush,
+                nbytes=A.numel() * 2, gen_dist=0, n=10)
+        krex.krex_gen_inputs(w.seed, 0, 0, 0.0, A, stream)
+        krex.krex_gen_inputs(w.seed, 1, 0, 0.0, B, stream)
+        if gname == gemm_names[0]:
+            rec("flush_l2", flush, None, nbytes=ws.flush.numel())
+        rec(reference_kernel(w) + sfx, lambda: krex.krex_run_reference(w.op, ws.inputs, ws.ref, stream), flush,
+            flops=w.flops, n=2 if w.M >= 16384 else 10, fma_peak=n_sm * FMA_LANES_PER_SM * 2 * 2.070e9)
+        rec("gemm_tcgen05" + sfx, lambda: krex.krex_run_candidate_ws(w.op, ws.inputs, ws.out, ws.gemm_ws, stream),
+            flush, flops=w.flops, n=10 if w.M >= 16384 else 20)
+        rec("check_bf16_f32" + sfx,
+            lambda: krex.krex_check_launch(ws.out, ws.ref, w.atol, w.rtol, ws.check_scratch, stream), flush,
+            nbytes=ws.out.numel() * 6, n=10)
+        del ws, A, B
+        torch.cuda.empty_cache()
     return out
 
 
-def generator_ceiling(dist: int, n_sm: int, stream, n_elements: int) -> dict:
-    """The rate at which this GPU computes a generator (uniform: dist 0,
-    normal: dist 1), measured with the library's probe: the fill kernel's loop
-    over n_elements on the fills' residency (8 blocks of 256 threads per SM)
-    with folds instead of stores, best of 10 launches, as output GB/s: the
-    fills' compute roofline."""
+def fill_beside_ceiling(dist: int, n_sm: int, stream, fill, n_elements: int, flush, n: int = 10):
+    """A fill and its generator probe launched alternately, so both see the
+    same clock and power state.  The probe (krex_probe_generator) runs the
+    fill kernel's loop over as many elements on the fills' residency (8 blocks
+    of 256 threads per SM) with folds instead of stores: the rate at which
+    this GPU computes the generator, the fill's compute roofline.  Returns the
+    probe's best of n launches (a peak, like the driver's) as output GB/s and
+    the fill's mean of n launches, each fill after an L2 flush."""
     import torch
     import paper_2609_30057_gb300 as krex
     blocks = n_sm * 8
     sink = torch.empty(blocks * 256, dtype=torch.int32, device="cuda")
-    fn = lambda: krex.krex_probe_generator(dist, n_elements, blocks, sink, stream=stream)  # noqa: E731
+    probe = lambda: krex.krex_probe_generator(dist, n_elements, blocks, sink, stream=stream)  # noqa: E731
     for _ in range(3):
-        fn()
-    ms = _time_launches(fn, 10, stream, best=True)   # a peak: best of 10, like the driver's peaks
+        probe()
+        fill()
+    pe = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    fe = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    for i in range(n):
+        pe[i][0].record(stream)
+        probe()
+        pe[i][1].record(stream)
+        flush()
+        fe[i][0].record(stream)
+        fill()
+        fe[i][1].record(stream)
+    stream.synchronize()
+    p_ms = min(a.elapsed_time(b) for a, b in pe)
+    f_ms = statistics.fmean(a.elapsed_time(b) for a, b in fe)
     draws = n_elements // 2
-    return {"ms": ms, "elements": n_elements, "Gdraws/s": draws / ms / 1e6,
-            "GB/s": draws * DRAW_BYTES[dist] / ms / 1e6, "blocks": blocks}
+    ceiling = {"ms": p_ms, "elements": n_elements, "Gdraws/s": draws / p_ms / 1e6,
+               "GB/s": draws * DRAW_BYTES[dist] / p_ms / 1e6, "blocks": blocks}
+    return ceiling, f_ms
 
 
 # ---------------------------------------------------------- CPU oracle ------
