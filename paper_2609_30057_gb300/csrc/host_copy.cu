@@ -47,8 +47,8 @@ cudaError_t launch_copy_rows_from_host(const void *src, size_t spitch, void *dst
         return cudaSuccess;
     }
     const int64_t w16 = (int64_t)(width / 16), n = w16 * (int64_t)rows;
-    // 8 blocks of 256 threads per SM on 152 SMs, fewer for small copies
-    const int64_t blocks = std::min<int64_t>(152 * 8, (n + 1023) / 1024);
+    // 8 blocks of 256 threads per SM, fewer for small copies
+    const int64_t blocks = std::min<int64_t>((int64_t)sm_count() * 8, (n + 1023) / 1024);
     const auto *s16 = static_cast<const uint4 *>(src);
     auto *d16 = static_cast<uint4 *>(dst);
     if (spitch == width && dpitch == width)
