@@ -394,7 +394,8 @@ def oracle_full_command(w):
 
 def cpu_baseline_record(w, budget_s: float = 12.0):
     """The oracle as it stands on the host cores (a bounded sample of the
-    workload), plus one whole small command timed in full."""
+    workload), plus one whole small command timed in full and each oracle
+    routine timed on its own."""
     from paper_2609_30057_gb300.command import WORKLOADS
     rate, steps, secs, info = oracle_rate(w, budget_s)
     small = WORKLOADS["gemm_bf16_256"]
@@ -405,7 +406,63 @@ def cpu_baseline_record(w, budget_s: float = 12.0):
             "measured_wall_s": secs, "steps": steps,
             "threads": "fp64 GEMM through numpy's BLAS on all host cores; generation and check single-threaded",
             "cpu_model": cpu_model(),
-            "full_command_unextrapolated": {"workload": small.name, "seconds": full_s, "cmds_per_s": 1.0 / full_s}}
+            "full_command_unextrapolated": {"workload": small.name, "seconds": full_s, "cmds_per_s": 1.0 / full_s},
+            "components": oracle_components()}
+
+
+_ONE_THREAD_GEMM = r"""
+import json, sys, time
+sys.path.insert(0, sys.argv[1])
+from oracle import gen, ref
+n = int(sys.argv[2])
+a, b = gen.uniform_bf16(2, 0, n, n), gen.uniform_bf16(2, 1, n, n)
+ref.gemm_f64(a, b)
+t = time.perf_counter()
+ref.gemm_f64(a, b)
+print(json.dumps({"seconds": time.perf_counter() - t}))
+"""
+
+
+def oracle_components() -> dict:
+    """Baseline only: each oracle routine timed once on the host, with the
+    threads it runs on.  Generation (GB/s of output: the 4096^2 bf16 operand,
+    2^21 Box-Muller values), the fp64 GEMM (GFLOP/s: the 4096^3 workload in
+    full on all cores through numpy's BLAS, and 1024^3 on one thread in a
+    child process with the BLAS limited to one thread), the fp64 softmax (rows
+    of 8192 per second) and the fp32 check (GB/s of a 16-bit output and an
+    fp32 reference, 6 B per element, 4096^2 elements)."""
+    import subprocess
+    import sys
+    import numpy as np
+    from oracle import gen, ref
+
+    def timed(fn):
+        t = time.perf_counter()
+        r = fn()
+        return r, time.perf_counter() - t
+
+    out = {"label": "baseline only"}
+    a, s = timed(lambda: gen.uniform_bf16(2, 0, 4096, 4096))
+    out["gen_uniform_bf16"] = {"GB/s": a.nbytes / s / 1e9, "elements": int(a.size), "threads": 1}
+    x, s = timed(lambda: gen.normal_f32(3, 0, 256, 8192, 2.0))
+    out["gen_normal_f32"] = {"GB/s": x.nbytes / s / 1e9, "elements": int(x.size), "threads": 1}
+    b = gen.uniform_bf16(2, 1, 4096, 4096)
+    c, s = timed(lambda: ref.gemm_f64(a, b))
+    out["gemm_f64_4096"] = {"GFLOP/s": 2 * 4096 ** 3 / s / 1e9, "seconds": s, "threads": cpu_cores()}
+    env = dict(os.environ, OPENBLAS_NUM_THREADS="1", OMP_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    try:
+        r = subprocess.run([sys.executable, "-c", _ONE_THREAD_GEMM, os.path.dirname(os.path.abspath(__file__)),
+                            "1024"], env=env, capture_output=True, text=True, timeout=300)
+        one = json.loads(r.stdout.strip().splitlines()[-1])["seconds"]
+        out["gemm_f64_1024_one_thread"] = {"GFLOP/s": 2 * 1024 ** 3 / one / 1e9, "seconds": one, "threads": 1}
+    except (subprocess.SubprocessError, ValueError, IndexError, KeyError) as e:
+        out["gemm_f64_1024_one_thread"] = {"error": str(e)[:200]}
+    y, s = timed(lambda: ref.softmax_rows_f64(x.astype(np.float64)))
+    out["softmax_f64_8192"] = {"rows/s": x.shape[0] / s, "rows": int(x.shape[0]), "threads": 1}
+    c32 = c.astype(np.float32)
+    _, s = timed(lambda: ref.check_f32(c32, c32, 2.0 ** -6, 2.0 ** -7))
+    out["check_f32_4096"] = {"GB/s": c32.size * 6 / s / 1e9, "elements": int(c32.size), "threads": 1}
+    return out
 
 
 def _p95(xs) -> float:
