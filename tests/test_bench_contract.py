@@ -47,6 +47,20 @@ def test_reference_arm_config_keys_match_our_arm():
     assert abs(d["value"] - 2 * f / (d["ms_per_step"] * 2 / 1e3)) < 1e-9 * d["value"]
 
 
+def test_oracle_components_are_labelled_timings():
+    # cpu_baseline.components: each oracle routine timed once on the host,
+    # labelled baseline only, every rate positive, with its thread count
+    sys.path.insert(0, ROOT)
+    import bench
+    c = bench.oracle_components()
+    assert c["label"] == "baseline only"
+    keys = {"gen_uniform_bf16": "GB/s", "gen_normal_f32": "GB/s", "gemm_f64_4096": "GFLOP/s",
+            "gemm_f64_1024_one_thread": "GFLOP/s", "softmax_f64_8192": "rows/s", "check_f32_4096": "GB/s"}
+    for k, unit in keys.items():
+        assert c[k][unit] > 0 and c[k]["threads"] >= 1, (k, c[k])
+    assert c["gemm_f64_1024_one_thread"]["threads"] == 1
+
+
 @pytest.mark.gpu
 def test_our_arm_line():
     d = _bench("--steps", "3", "--warmup", "3", "--no-kernels", "--no-configs", "--workload", "gemm_bf16_4096")
