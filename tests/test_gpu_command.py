@@ -105,6 +105,26 @@ def test_command_host_inputs_by_each_copy_route(route):
         assert not pads[1].view(torch.int16)[:, w.N:].any()
 
 
+def test_command_8192_host_inputs_by_copy_kernel_equal_generated():
+    # 2 x 128 MiB of page-locked inputs read by the copy kernel (2^23 16-byte
+    # words per operand): the candidate's output and the verdict equal those of
+    # the same command with device-generated inputs, bit for bit
+    w = scaled(WORKLOADS["gemm_bf16_8192"], iters=3)
+    ws = Workspace(w)
+    r0 = ws.run()
+    assert r0.passed == 1
+    want = bits16(ws.out)
+    hosts = [t.cpu().pin_memory() for t in ws.inputs]
+    ws.out.zero_()
+    hc = torch.empty(w.M, w.N, dtype=torch.bfloat16).pin_memory()
+    r = ws.run(host_in=[h.data_ptr() for h in hosts], host_out=hc.data_ptr())
+    assert r.passed == 1 and r.launches == r0.launches   # two copy kernels in place of the two fills
+    assert np.array_equal(bits16(ws.out), want)
+    assert np.array_equal(hc.view(torch.int16).numpy().view(np.uint16), want)
+    assert r.check.n_violations == r0.check.n_violations == 0
+    assert ref.check_bits(r.check.max_abs_err) == ref.check_bits(r0.check.max_abs_err)
+
+
 def test_softmax_command_small():
     w = scaled(WORKLOADS["softmax_f32_65536x8192"], M=512, iters=5)
     ws = Workspace(w)
