@@ -518,7 +518,8 @@ krex_status krex_probe_fma(int32_t iters, int32_t blocks, void *dev_sink, krex_s
  * paper: the knobs of this implementation's kernels.  Changing it affects
  * launches issued after the call (it is read once per launch). */
 typedef struct {
-    int32_t gemm_pair_tile_n;  /* columns of a 2-SM pair tile: 0 = 256; else 128, 192 or 256 */
+    int32_t gemm_pair_tile_n;  /* columns of a 2-SM pair tile: 0 = 256; else 128, 192, 256 or 512 (two MMAs
+                                  of N = 256 per K step into one 512-column accumulator) */
     int32_t gemm_stage_k;      /* K depth of a shared-memory ring stage: 0 = 128; else 64 or 128 */
     int32_t gemm_ring_stages;  /* stages of the ring in use: 0 = all that fit (3 of K 128, 6 of K 64); else
                                   2 .. that number */

@@ -98,7 +98,7 @@ krex_tuning g_tuning = default_tuning();
 
 bool tuning_valid(const krex_tuning &t) {
     return (t.gemm_pair_tile_n == 0 || t.gemm_pair_tile_n == 128 || t.gemm_pair_tile_n == 192 ||
-            t.gemm_pair_tile_n == 256) &&
+            t.gemm_pair_tile_n == 256 || t.gemm_pair_tile_n == 512) &&
            (t.gemm_stage_k == 0 || t.gemm_stage_k == 64 || t.gemm_stage_k == 128) &&
            (t.gemm_ring_stages == 0 ||
             (t.gemm_ring_stages >= 2 && t.gemm_ring_stages <= (t.gemm_stage_k == 64 ? 6 : 3))) &&

@@ -33,6 +33,7 @@
 #include <cuda_fp16.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <atomic>
 #include <mutex>
 #include <unordered_map>
@@ -249,17 +250,20 @@ constexpr int EPI_BYTES = 4 * 2 * EPI_BUF_BYTES; // 4 epilogue warps x 2 buffers
 constexpr int TMEM_COLS = 2 * BN;                // two 128-lane x 256-column accumulators
 constexpr int GROUP_M = 8;                       // pair-tile rows per raster group (see raster_group)
 constexpr int EPI_WARPS = 4;
-// A stage holds KSUB K sub-blocks (KSUB x 64 of K): 6 stages of 32 KiB or 3
-// of 64 KiB.  Fewer, deeper stages issue 8 MMAs per barrier wait and commit
-// instead of 4 (each commit costs the tensor pipe a few percent).
-template <int KSUB>
+// A stage holds KSUB K sub-blocks (KSUB x 64 of K) of A and of NCH 256-column
+// chunks of B: 6 stages of 32 KiB or 3 of 64 KiB for pair tiles up to 256
+// wide (NCH 1), 4 stages of 48 KiB for pair tiles of 256 x 512 (NCH 2).
+// Fewer, deeper stages issue 8 MMAs per barrier wait and commit instead of 4
+// (each commit costs the tensor pipe a few percent).
+template <int KSUB, int NCH = 1>
 struct Cfg {
-    static constexpr int STAGES = 6 / KSUB;
     static constexpr int A_STAGE_BYTES = KSUB * A_SUB_BYTES;
-    static constexpr int B_STAGE_BYTES = KSUB * B_SUB_BYTES;
+    static constexpr int B_STAGE_BYTES = KSUB * NCH * B_SUB_BYTES;
+    static constexpr int STAGES = RING_BYTES / (A_STAGE_BYTES + B_STAGE_BYTES);
     static constexpr int NUM_BARS = 2 * STAGES + 4 + 1;
     static constexpr size_t SMEM_BYTES = 1024 + (size_t)RING_BYTES + EPI_BYTES + NUM_BARS * 8 + 48;
 };
+static_assert(Cfg<1>::STAGES == 6 && Cfg<2>::STAGES == 3 && Cfg<1, 2>::STAGES == 4, "ring layout");
 // kind::f16, D fp32, A/B bf16, A K-major, B MN-major, M = 256 (pair); N is
 // added at run time in bits 17-22
 constexpr uint32_t IDESC_NO_N = (1u << 4) | (1u << 7) | (1u << 10) | (0u << 15) | (1u << 16) |
@@ -456,10 +460,12 @@ __device__ __forceinline__ void spin_ns(uint64_t ns) {
     }
 }
 
-// Pair tiles are 256 x bn (bn a multiple of 64, 128 <= bn <= 256); tiles_m,
-// tiles_n count them.  The host picks bn so the tiles fill whole waves.
-// F16: IEEE binary16 A, B and C (instruction-descriptor formats 0); else bf16.
-template <int KSUB, bool F16>
+// Pair tiles are 256 x bn (NCH 1: bn a multiple of 64, 128 <= bn <= 256;
+// NCH 2: bn = 512, two MMAs of N = 256 per K step into the two halves of one
+// 512-column accumulator); tiles_m, tiles_n count them.  The host picks bn so
+// the tiles fill whole waves.  F16: IEEE binary16 A, B and C
+// (instruction-descriptor formats 0); else bf16.
+template <int KSUB, bool F16, int NCH>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                       const __grid_constant__ CUtensorMap tmC, uint16_t *__restrict__ C, int64_t ldc, int M,
@@ -468,7 +474,8 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                       float *ws_partial, uint32_t *ws_count, uint32_t *ws_flag, uint32_t launch_id,
                       uint32_t wait_tag, int k_alternate) {
     // the pair kernel's tile constants (the file-level BM, BK serve the host's tensor maps)
-    using CF = v2::Cfg<KSUB>;
+    using CF = v2::Cfg<KSUB, NCH>;
+    static_assert(NCH == 1 || (NCH == 2 && KSUB == 1), "wide pair tiles use 64-deep stages");
     constexpr int BM = v2::BM, BN = v2::BN, BK = v2::BK, STAGES = CF::STAGES;
     constexpr int A_STAGE_BYTES = CF::A_STAGE_BYTES, B_STAGE_BYTES = CF::B_STAGE_BYTES;
     constexpr int A_SUB_BYTES = v2::A_SUB_BYTES, B_SUB_BYTES = v2::B_SUB_BYTES;
@@ -539,19 +546,23 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             const WorkItem it = work_item(w, full_items, tiles_m, tiles_n, group_m, bn, num_kb, split_k);
             const int mb = it.mb, nb = it.nb, col0 = it.col0, width = it.width;
             (void)nb;
-            const int b_half = width >> 1;                            // B columns per CTA
-            const int b_boxes = (b_half + B_BOX_N - 1) / B_BOX_N;     // TMA boxes per CTA and stage
+            const int cw = width / NCH;                               // columns of one MMA (a chunk)
+            const int b_half = cw >> 1;                               // B columns per CTA and chunk
+            const int b_boxes = (b_half + B_BOX_N - 1) / B_BOX_N;     // TMA boxes per CTA, chunk and stage
             // what each CTA of the pair loads (boxes wholly outside the matrix are skipped)
-            int a_ok[2], nbox[2];
+            int a_ok[2], nbox[2][NCH], nbox_all = 0;
             for (int r = 0; r < 2; ++r) {
                 a_ok[r] = (mb * 2 * BM + r * BM) < M;
-                const int n0r = col0 + r * b_half;
-                nbox[r] = n0r < N ? min(b_boxes, (N - n0r + B_BOX_N - 1) / B_BOX_N) : 0;
+                for (int ch = 0; ch < NCH; ++ch) {
+                    const int n0r = col0 + ch * cw + r * b_half;
+                    nbox[r][ch] = n0r < N ? min(b_boxes, (N - n0r + B_BOX_N - 1) / B_BOX_N) : 0;
+                    nbox_all += nbox[r][ch];
+                }
             }
             const uint32_t sub_bytes = (uint32_t)((a_ok[0] + a_ok[1]) * A_SUB_BYTES +
-                                                  (nbox[0] + nbox[1]) * B_BOX_BYTES);  // per K sub-block
+                                                  nbox_all * B_BOX_BYTES);  // per K sub-block
             const int m0 = mb * 2 * BM + (int)rank * BM;
-            const int n0 = col0 + (int)rank * b_half;
+            const int n0 = col0 + (int)rank * b_half;                 // this CTA's columns of chunk 0
             abort_flag[1] = (uint32_t)w;
             const bool rev = k_reversed(w, nclusters, full_items, k_alternate);
             for (int i = it.kb0; i < it.kb1; ++i) {
@@ -574,9 +585,12 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                     const int k0 = (kb * KSUB + h) * BK;
                     if (a_ok[rank])
                         tma_load_2d_pair(smem_u32(sA + stage * A_STAGE_BYTES + h * A_SUB_BYTES), &tmA, fb, k0, m0);
-                    for (int j = 0; j < nbox[rank]; ++j)
-                        tma_load_2d_pair(smem_u32(sB + stage * B_STAGE_BYTES + h * B_SUB_BYTES + j * B_BOX_BYTES),
-                                         &tmB, fb, n0 + j * B_BOX_N, k0);
+#pragma unroll
+                    for (int ch = 0; ch < NCH; ++ch)
+                        for (int j = 0; j < nbox[rank][ch]; ++j)
+                            tma_load_2d_pair(smem_u32(sB + stage * B_STAGE_BYTES + (h * NCH + ch) * B_SUB_BYTES +
+                                                      j * B_BOX_BYTES),
+                                             &tmB, fb, n0 + ch * cw + j * B_BOX_N, k0);
                 }
                 if (++stage == stages) {
                     stage = 0;
@@ -594,9 +608,10 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
         for (int w = cluster_id; ok && w < num_items; w += nclusters, ++local) {
             const WorkItem it = work_item(w, full_items, tiles_m, tiles_n, group_m, bn, num_kb, split_k);
             constexpr uint32_t idesc_ab = F16 ? (v2::IDESC_NO_N & ~((7u << 7) | (7u << 10))) : v2::IDESC_NO_N;
-            const uint32_t idesc = idesc_ab | ((uint32_t)(it.width >> 3) << 17);
-            const int acc = local & 1;
-            const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
+            const uint32_t idesc = idesc_ab | ((uint32_t)((it.width / NCH) >> 3) << 17);
+            // NCH 1: two accumulators used in turn; NCH 2: one of 512 columns
+            const int acc = NCH == 1 ? (local & 1) : 0;
+            const uint32_t acc_phase = (uint32_t)(NCH == 1 ? ((local >> 1) & 1) : (local & 1));
             abort_flag[3] = (uint32_t)w;
             abort_flag[4] = 0xFFFFFFFFu;  // waiting for the accumulator
             if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, timeout_ns, 0x41)) {
@@ -620,12 +635,18 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                     if (h < nsub) {
                         const uint64_t adesc =
                             sdesc_sw128(smem_u32(sA + stage * A_STAGE_BYTES + h * A_SUB_BYTES), 16, 1024);
-                        const uint64_t bdesc =
-                            sdesc_sw128(smem_u32(sB + stage * B_STAGE_BYTES + h * B_SUB_BYTES), B_BOX_BYTES, 1024);
 #pragma unroll
-                        for (int k = 0; k < BK / 16; ++k)
-                            mma_bf16_pair(d_tmem, adesc + (uint64_t)(2 * k), bdesc + (uint64_t)(128 * k), idesc,
-                                          ((i - it.kb0) | h | k) != 0 ? 1u : 0u);
+                        for (int k = 0; k < BK / 16; ++k) {
+#pragma unroll
+                            for (int ch = 0; ch < NCH; ++ch) {
+                                const uint64_t bdesc = sdesc_sw128(
+                                    smem_u32(sB + stage * B_STAGE_BYTES + (h * NCH + ch) * B_SUB_BYTES),
+                                    B_BOX_BYTES, 1024);
+                                mma_bf16_pair(d_tmem + (uint32_t)(ch * BN), adesc + (uint64_t)(2 * k),
+                                              bdesc + (uint64_t)(128 * k), idesc,
+                                              ((i - it.kb0) | h | k) != 0 ? 1u : 0u);
+                            }
+                        }
                     }
                 }
                 mma_commit_pair(empty_bar(stage));
@@ -649,8 +670,8 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             const WorkItem it = work_item(w, full_items, tiles_m, tiles_n, group_m, bn, num_kb, split_k);
             const int mb = it.mb, nb = it.nb, col0 = it.col0, width = it.width;
             (void)nb;
-            const int acc = local & 1;
-            const uint32_t acc_phase = (uint32_t)((local >> 1) & 1);
+            const int acc = NCH == 1 ? (local & 1) : 0;
+            const uint32_t acc_phase = (uint32_t)(NCH == 1 ? ((local >> 1) & 1) : (local & 1));
             if (ew == 0 && lane == 0) {
                 abort_flag[5] = (uint32_t)w;
                 abort_flag[6] = 1u;  // waiting for the accumulator
@@ -888,10 +909,32 @@ krex_status make_map(const void *ptr, uint64_t inner, uint64_t outer, uint64_t l
 // (krex_get_tuning_internal); a field at its default takes the measured
 // choice documented beside it.
 //
-// Pair-tile width: measured on GB300, a tcgen05.mma of N = 224 or 192 costs
-// about as much time as N = 256, so narrower tiles only add waves: 256
-// unless set (128, 192 or 256: the epilogue stores 64-column boxes).
-int pick_pair_tile_n(const krex_tuning &t) { return t.gemm_pair_tile_n ? t.gemm_pair_tile_n : 256; }
+// Pair-tile width.  Measured on GB300, a tcgen05.mma of N = 224 or 192 costs
+// about as much time as N = 256, so narrower tiles only add waves.  Wide pair
+// tiles of 256 x 512 (two MMAs of N = 256 per K step into one 512-column
+// accumulator) load a quarter fewer bytes per flop into each SM, whose load
+// rate (about 100 GB/s per SM) holds 256-wide tiles near 87 % of the tensor
+// pipe; but with one accumulator the epilogue no longer overlaps the next
+// tile's MMAs, and the tail split into column halves does not apply.  So 512
+// when K is long enough for the exposed epilogue not to matter and the wide
+// tiles fill their waves about as well (within kWideGain) as 256-wide tiles
+// with their split tail; else 256.  The tuning record fixes it (128, 192,
+// 256 or 512: the epilogue stores 64-column boxes).
+constexpr int64_t kWideMinK = 8192;
+constexpr double kWideGain = 1.04;
+
+int pick_pair_tile_n(const krex_tuning &t, int64_t M, int64_t N, int64_t K, int max_clusters) {
+    if (t.gemm_pair_tile_n) return t.gemm_pair_tile_n;
+    if (K < kWideMinK || max_clusters <= 0) return 256;
+    const int64_t tm = (M + 2 * v2::BM - 1) / (2 * v2::BM);
+    const int64_t t512 = tm * ((N + 511) / 512), t256 = tm * ((N + 255) / 256);
+    const double c = (double)max_clusters;
+    const double eff512 = (double)t512 / (c * (double)((t512 + max_clusters - 1) / max_clusters));
+    const int64_t rem = t256 % max_clusters;
+    const double waves256 = (double)(t256 / max_clusters) + (rem == 0 ? 0.0 : (2 * rem <= max_clusters ? 0.5 : 1.0));
+    const double eff256 = (double)t256 / (c * waves256);
+    return eff512 * kWideGain >= eff256 ? 512 : 256;
+}
 
 // Pair-tile rows per raster group.  Measured on GB300 (TFLOP/s, group 4 vs
 // 8, L2 flushed): 3072^3 1381 vs 1325, 4096^3 1561 vs 1525, 4608^3 1579 vs
@@ -976,21 +1019,25 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
     int dev = 0;
     KREX_CUDA_TRY(cudaGetDevice(&dev));
     if (attr_dev != dev) {
-        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<1, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)v2::Cfg<1>::SMEM_BYTES));
-        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<2, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)v2::Cfg<2>::SMEM_BYTES));
-        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<1, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)v2::Cfg<1>::SMEM_BYTES));
-        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<2, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                           (int)v2::Cfg<2>::SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<1, false, 1>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)v2::Cfg<1>::SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<2, false, 1>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)v2::Cfg<2>::SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<1, true, 1>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)v2::Cfg<1>::SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<2, true, 1>,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize, (int)v2::Cfg<2>::SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<1, false, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)v2::Cfg<1, 2>::SMEM_BYTES));
+        KREX_CUDA_TRY(cudaFuncSetAttribute(gemm_tcgen05_2sm<1, true, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)v2::Cfg<1, 2>::SMEM_BYTES));
         // co-resident CTA pairs; a persistent grid larger than this would only queue
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * (unsigned)(sm_count() / 2), 1, 1);
         cfg.blockDim = dim3(THREADS, 1, 1);
         cfg.dynamicSmemBytes = v2::Cfg<2>::SMEM_BYTES;
         int n = 0;
-        if (cudaOccupancyMaxActiveClusters(&n, gemm_tcgen05_2sm<2, false>, &cfg) != cudaSuccess || n <= 0) {
+        if (cudaOccupancyMaxActiveClusters(&n, gemm_tcgen05_2sm<2, false, 1>, &cfg) != cudaSuccess || n <= 0) {
             cudaGetLastError();
             n = sm_count() / 2;
         }
@@ -1009,7 +1056,7 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
             mc = ma;  // unused
         }
         const int tiles_m = (int)((M + 2 * v2::BM - 1) / (2 * v2::BM));
-        const int bn = pick_pair_tile_n(tun);
+        const int bn = pick_pair_tile_n(tun, M, N, K, max_clusters);
         const int tiles_n = (int)((N + bn - 1) / bn);
         const int64_t tiles = (int64_t)tiles_m * tiles_n;
         // Split the tiles of a final partial wave into column halves when that
@@ -1029,7 +1076,7 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
         // written, then read) sits on the last wave's critical path: at 4096^3
         // the K halves end their MMAs 6.8 us earlier and spend about as long
         // exchanging partials, so the multi-wave case gains nothing.
-        const int ksub = stage_ksub(tun);
+        const int ksub = bn == 512 ? 1 : stage_ksub(tun);
         const int64_t num_kb = (((K + 63) / 64) + ksub - 1) / ksub;
         const int sk_mode = tun.gemm_split_k;
         const bool k_worth_it = sk_mode == 1 || (sk_mode < 0 && K >= kSplitKMinK);
@@ -1054,14 +1101,19 @@ krex_status launch_gemm_tcgen05(const uint16_t *a, int64_t lda, const uint16_t *
                                                        tun.gemm_k_alternate == 0 ? 0 : 1);
         };
         const int st2 = ring_stages(tun, v2::Cfg<2>::STAGES), st1 = ring_stages(tun, v2::Cfg<1>::STAGES);
-        if (ksub == 2 && f16)
-            go(gemm_tcgen05_2sm<2, true>, v2::Cfg<2>::SMEM_BYTES, st2);
+        const int stw = std::min(ring_stages(tun, v2::Cfg<1, 2>::STAGES), v2::Cfg<1, 2>::STAGES);
+        if (bn == 512 && f16)
+            go(gemm_tcgen05_2sm<1, true, 2>, v2::Cfg<1, 2>::SMEM_BYTES, stw);
+        else if (bn == 512)
+            go(gemm_tcgen05_2sm<1, false, 2>, v2::Cfg<1, 2>::SMEM_BYTES, stw);
+        else if (ksub == 2 && f16)
+            go(gemm_tcgen05_2sm<2, true, 1>, v2::Cfg<2>::SMEM_BYTES, st2);
         else if (ksub == 2)
-            go(gemm_tcgen05_2sm<2, false>, v2::Cfg<2>::SMEM_BYTES, st2);
+            go(gemm_tcgen05_2sm<2, false, 1>, v2::Cfg<2>::SMEM_BYTES, st2);
         else if (f16)
-            go(gemm_tcgen05_2sm<1, true>, v2::Cfg<1>::SMEM_BYTES, st1);
+            go(gemm_tcgen05_2sm<1, true, 1>, v2::Cfg<1>::SMEM_BYTES, st1);
         else
-            go(gemm_tcgen05_2sm<1, false>, v2::Cfg<1>::SMEM_BYTES, st1);
+            go(gemm_tcgen05_2sm<1, false, 1>, v2::Cfg<1>::SMEM_BYTES, st1);
     }
     KREX_CUDA_TRY(cudaGetLastError());
     return KREX_OK;

@@ -105,7 +105,7 @@ def test_seeded_gemm_within_tolerance(M, N, K, variant):
     assert ok, worst
 
 
-@pytest.mark.parametrize("bn", [128, 192, 256])
+@pytest.mark.parametrize("bn", [128, 192, 256, 512])
 @pytest.mark.parametrize("M,N,K", [(300, 1000, 520), (512, 1792, 256), (256, 192, 64), (260, 328, 72)])
 def test_2sm_every_pair_tile_width(M, N, K, bn):
     krex.krex_set_tuning(gemm_pair_tile_n=bn)
@@ -114,6 +114,49 @@ def test_2sm_every_pair_tile_width(M, N, K, bn):
     c = _candidate(a, b)
     want = ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N))
     ok, worst = _within_tol(bits16(c), want, K)
+    assert ok, worst
+
+
+@pytest.mark.parametrize("M,N,K", [(2048, 4096, 4096), (1000, 3000 - 8, 1032), (4096, 4096, 4096)])
+def test_wide_pair_tiles_several_waves(M, N, K):
+    # pair tiles of 256 x 512 (two MMAs of N = 256 per K step into one
+    # 512-column accumulator, the epilogue draining it before the next tile):
+    # several tiles per pair, a ragged last column chunk, full output; and the
+    # same GEMM through the workspace form, both K orders
+    krex.krex_set_tuning(gemm_pair_tile_n=512)
+    seed = 3500 + M + N + K
+    a, b = _gen(seed, M, N, K)
+    want = ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N))
+    c = _candidate(a, b)
+    ok, worst = _within_tol(bits16(c), want, K)
+    assert ok, worst
+    for alt in (0, 1):
+        krex.krex_set_tuning(gemm_pair_tile_n=512, gemm_k_alternate=alt)
+        g = Guarded(M, N, torch.bfloat16)
+        krex.krex_run_candidate_ws(krex.KREX_OP_GEMM_BF16, [a, b], g.view, krex.gemm_workspace())
+        torch.cuda.synchronize()
+        assert krex.krex_device_status() == 0 and g.canaries_intact()
+        ok, worst = _within_tol(bits16(g.view), want, K)
+        assert ok, worst
+
+
+def test_wide_pair_tiles_f16_and_large_sampled():
+    krex.krex_set_tuning(gemm_pair_tile_n=512)
+    M, N, K = 1536, 2560, 2048
+    ah, bh = gen.uniform_f16(71, 0, M, K), gen.uniform_f16(71, 1, K, N)
+    c = Guarded(M, N, torch.float16)
+    krex.krex_run_candidate(krex.KREX_OP_GEMM_F16, [to_f16_tensor(ah), to_f16_tensor(bh)], c.view)
+    torch.cuda.synchronize()
+    assert krex.krex_device_status() == 0 and c.canaries_intact()
+    want = ref.gemm_f64(ah, bh, dtype="f16")
+    got = gen.f16_to_f32(bits16(c.view)).astype(np.float64)
+    assert np.all(np.abs(got - want) <= ref.gemm_tolerance(want, K, dtype="f16"))
+    n = 16384
+    a, b = _gen(5, n, n, n)
+    out = _candidate(a, b, guard=False)
+    i, j = ref.sample_indices(5, 2, 4096, n, n)
+    got = bits16(out[torch.from_numpy(i).cuda(), torch.from_numpy(j).cuda()])
+    ok, worst = _within_tol(got, ref.gemm_sampled_f64(5, n, n, n, i, j), n)
     assert ok, worst
 
 
