@@ -614,33 +614,23 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             const uint32_t acc_phase = (uint32_t)(NCH == 1 ? ((local >> 1) & 1) : (local & 1));
             abort_flag[3] = (uint32_t)w;
             abort_flag[4] = 0xFFFFFFFFu;  // waiting for the accumulator
-            if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, timeout_ns, 0x41)) {
-                ok = false;
-                break;
-            }
-            tc_fence_after();
             const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
             const bool rev = k_reversed(w, nclusters, full_items, k_alternate);
-            for (int i = it.kb0; i < it.kb1; ++i) {
-                const int kb = rev ? it.kb0 + it.kb1 - 1 - i : i;  // the stage the producer loaded
-                abort_flag[4] = (uint32_t)kb;
-                if (!mbar_wait(full_bar(stage), phase, abort_flag, timeout_ns, 0x42)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
+            // the MMAs of chunks [c0, c1) of ring stage st, which holds K stage kb (item step i)
+            auto issue = [&](int st, int kb, int i, int c0, int c1) {
                 const int nsub = min(KSUB, num_ksub - kb * KSUB);
 #pragma unroll
                 for (int h = 0; h < KSUB; ++h) {
                     if (h < nsub) {
                         const uint64_t adesc =
-                            sdesc_sw128(smem_u32(sA + stage * A_STAGE_BYTES + h * A_SUB_BYTES), 16, 1024);
+                            sdesc_sw128(smem_u32(sA + st * A_STAGE_BYTES + h * A_SUB_BYTES), 16, 1024);
 #pragma unroll
                         for (int k = 0; k < BK / 16; ++k) {
 #pragma unroll
                             for (int ch = 0; ch < NCH; ++ch) {
+                                if (ch < c0 || ch >= c1) continue;
                                 const uint64_t bdesc = sdesc_sw128(
-                                    smem_u32(sB + stage * B_STAGE_BYTES + (h * NCH + ch) * B_SUB_BYTES),
+                                    smem_u32(sB + st * B_STAGE_BYTES + (h * NCH + ch) * B_SUB_BYTES),
                                     B_BOX_BYTES, 1024);
                                 mma_bf16_pair(d_tmem + (uint32_t)(ch * BN), adesc + (uint64_t)(2 * k),
                                               bdesc + (uint64_t)(128 * k), idesc,
@@ -649,6 +639,64 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                         }
                     }
                 }
+            };
+            int i = it.kb0;
+            if constexpr (NCH == 2) {
+                // One accumulator whose halves the epilogue releases in turn: the
+                // chunk-0 MMAs of the first ring's worth of stages run as soon as
+                // half 0 is drained, while the epilogue still drains half 1; then
+                // their chunk-1 MMAs, and the stages are released.
+                if (!mbar_wait(tempty_bar(0), acc_phase ^ 1u, abort_flag, timeout_ns, 0x41)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const int pre = min(stages, it.kb1 - it.kb0);
+                int st = stage;
+                uint32_t ph = phase;
+                for (int q = 0; q < pre && ok; ++q) {
+                    const int kb = rev ? it.kb0 + it.kb1 - 1 - (i + q) : i + q;
+                    abort_flag[4] = (uint32_t)kb;
+                    if (!mbar_wait(full_bar(st), ph, abort_flag, timeout_ns, 0x42)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    issue(st, kb, i + q, 0, 1);
+                    if (++st == stages) {
+                        st = 0;
+                        ph ^= 1u;
+                    }
+                }
+                if (ok && !mbar_wait(tempty_bar(1), acc_phase ^ 1u, abort_flag, timeout_ns, 0x45)) ok = false;
+                if (!ok) break;
+                tc_fence_after();
+                for (int q = 0; q < pre; ++q) {
+                    const int kb = rev ? it.kb0 + it.kb1 - 1 - (i + q) : i + q;
+                    issue(stage, kb, i + q, 1, 2);
+                    mma_commit_pair(empty_bar(stage));
+                    if (++stage == stages) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+                i += pre;
+            } else {
+                if (!mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, timeout_ns, 0x41)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+            }
+            for (; i < it.kb1; ++i) {
+                const int kb = rev ? it.kb0 + it.kb1 - 1 - i : i;  // the stage the producer loaded
+                abort_flag[4] = (uint32_t)kb;
+                if (!mbar_wait(full_bar(stage), phase, abort_flag, timeout_ns, 0x42)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                issue(stage, kb, i, 0, NCH);
                 mma_commit_pair(empty_bar(stage));
                 if (++stage == stages) {
                     stage = 0;
@@ -723,6 +771,15 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                     }
                 }
             }
+            // NCH 2: the first half of the accumulator goes back to the MMA
+            // issuer as soon as it is read, the second at the end
+            bool half0_released = false;
+            auto release_half0 = [&]() {
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_remote(tempty_leader0);
+                half0_released = true;
+            };
             if (!store_c) {
                 // nothing to store for this item
             } else if (c_tma) {
@@ -741,6 +798,9 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                     }
 #pragma unroll 1
                     for (int c = 0; c < width / v2::EPI_BOX_COLS; ++c) {
+                        if constexpr (NCH == 2) {
+                            if (c == width / (2 * v2::EPI_BOX_COLS)) release_half0();
+                        }
                         const int col0 = n0 + c * v2::EPI_BOX_COLS;
                         if (col0 >= N) break;  // warp-uniform
                         float pcur[PC];
@@ -788,6 +848,9 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                 uint16_t *crow = C + (int64_t)row * ldc;
 #pragma unroll 1
                 for (int c = 0; c < width / 32; ++c) {
+                    if constexpr (NCH == 2) {
+                        if (c == width / 64) release_half0();
+                    }
                     const int col0 = n0 + c * 32;
                     if (col0 >= N) break;  // warp-uniform
                     uint32_t v[32];
@@ -815,9 +878,12 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                     }
                 }
             }
+            if constexpr (NCH == 2) {
+                if (!half0_released) release_half0();
+            }
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive_remote(acc ? tempty_leader1 : tempty_leader0);
+            if (lane == 0) mbar_arrive_remote((NCH == 2 || acc) ? tempty_leader1 : tempty_leader0);
             if (ew == 0 && lane == 0) abort_flag[6] = 3u;  // released
         }
         if (lane == 0) bulk_wait_group_all();  // stores complete before shared memory goes away
