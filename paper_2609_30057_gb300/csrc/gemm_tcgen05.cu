@@ -203,6 +203,22 @@ __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
+// 32 consecutive fp32 columns of this warp's 32 TMEM lanes, without waiting
+// for them (tmem_wait_ld makes them usable).
+__device__ __forceinline__ void tmem_ld32_async(uint32_t taddr, uint32_t *v) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
+          "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
+          "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
+          "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait_ld() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
 // 32 consecutive fp32 columns of this warp's 32 TMEM lanes (thread t <-> lane base+t).
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
     asm volatile(
@@ -786,7 +802,45 @@ gemm_tcgen05_2sm(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                 // 64-column chunks: TMEM -> registers -> bf16 -> 128B-swizzled staging
                 // buffer (row = lane, 16-byte chunk j at j ^ (lane % 8)) -> one TMA store of
                 // the 32 x 64 box; two buffers per warp alternate.
-                if (row0 < M) {
+                // one 64-column chunk from registers to its staging buffer and the TMA store
+                auto store_chunk = [&](int c, const uint32_t *v) {
+                    uint8_t *buf = sEpi + (ew * 2 + (epi_buf & 1)) * v2::EPI_BUF_BYTES;
+                    if (lane == 0) bulk_wait_group_read<1>();  // the store that used `buf` has read it
+                    __syncwarp();
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {  // 16-byte chunk j of the 128-byte row
+                        uint32_t w[4];
+#pragma unroll
+                        for (int i = 0; i < 4; ++i)
+                            w[i] = pack2<F16>(__uint_as_float(v[8 * j + 2 * i]), __uint_as_float(v[8 * j + 2 * i + 1]));
+                        *reinterpret_cast<uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                            make_uint4(w[0], w[1], w[2], w[3]);
+                    }
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_2d(&tmC, smem_u32(buf), n0 + c * v2::EPI_BOX_COLS, row0);
+                        bulk_commit_group();
+                    }
+                    ++epi_buf;
+                };
+                if (row0 < M && !add) {
+                    // No partial to add: both 32-column loads of a chunk in flight
+                    // at once, one wait per chunk.
+                    const int nc = min(width, N - n0) <= 0 ? 0
+                                   : (min(width, N - n0) + v2::EPI_BOX_COLS - 1) / v2::EPI_BOX_COLS;
+#pragma unroll 1
+                    for (int c = 0; c < nc; ++c) {
+                        if constexpr (NCH == 2) {
+                            if (c == width / (2 * v2::EPI_BOX_COLS)) release_half0();
+                        }
+                        uint32_t va[64];
+                        tmem_ld32_async(tbase + (uint32_t)(c * v2::EPI_BOX_COLS), va);
+                        tmem_ld32_async(tbase + (uint32_t)(c * v2::EPI_BOX_COLS + 32), va + 32);
+                        tmem_wait_ld();
+                        store_chunk(c, va);
+                    }
+                } else if (row0 < M) {
                     // The other K half's partials (split-K) are read one 64-column
                     // chunk ahead, so their L2 round trips overlap this chunk's work
                     // instead of adding one per 32 columns.
