@@ -1034,26 +1034,30 @@ krex_status make_map(const void *ptr, uint64_t inner, uint64_t outer, uint64_t l
 // tiles of 256 x 512 (two MMAs of N = 256 per K step into one 512-column
 // accumulator) load a quarter fewer bytes per flop into each SM, whose load
 // rate (about 100 GB/s per SM) holds 256-wide tiles near 87 % of the tensor
-// pipe; but with one accumulator the epilogue no longer overlaps the next
-// tile's MMAs, and the tail split into column halves does not apply.  So 512
-// when K is long enough for the exposed epilogue not to matter and the wide
-// tiles fill their waves about as well (within kWideGain) as 256-wide tiles
-// with their split tail; else 256.  The tuning record fixes it (128, 192,
-// 256 or 512: the epilogue stores 64-column boxes).
-constexpr int64_t kWideMinK = 8192;
-constexpr double kWideGain = 1.04;
+// pipe (wide ones: 96 %); but with one accumulator the epilogue overlaps the
+// next tile's MMAs only in part, and the tail split into column halves does
+// not apply.  So the choice weighs how well each width fills its waves (a
+// split tail's half-width items cost about 0.8 of a whole tile) against the
+// wide tiles' per-tile gain, measured (L2 flushed, 256 vs 512, ratio of
+// times): 1.01 at K = 2048 (8192^2), 0.95-0.97 at K = 4096 (8192^2, 16384^2;
+// a tie at 4096^3, whose wide tiles fill 1.7 waves), 0.92-0.96 from K = 6144
+// on (6144^3 to 16384^3), and 1.05 for 4096 x 8192 x 16384, where the wide
+// tiles fill 3.4 waves against the 256-wide tiles' 6.7.  The tuning record
+// fixes the width (128, 192, 256 or 512: the epilogue stores 64-column boxes).
+constexpr int64_t kWideMinK = 4096;
 
 int pick_pair_tile_n(const krex_tuning &t, int64_t M, int64_t N, int64_t K, int max_clusters) {
     if (t.gemm_pair_tile_n) return t.gemm_pair_tile_n;
     if (K < kWideMinK || max_clusters <= 0) return 256;
+    const double gain = K < 6144 ? 1.04 : 1.08;  // the wide tiles' per-tile gain at this K
     const int64_t tm = (M + 2 * v2::BM - 1) / (2 * v2::BM);
     const int64_t t512 = tm * ((N + 511) / 512), t256 = tm * ((N + 255) / 256);
     const double c = (double)max_clusters;
     const double eff512 = (double)t512 / (c * (double)((t512 + max_clusters - 1) / max_clusters));
     const int64_t rem = t256 % max_clusters;
-    const double waves256 = (double)(t256 / max_clusters) + (rem == 0 ? 0.0 : (2 * rem <= max_clusters ? 0.5 : 1.0));
+    const double waves256 = (double)(t256 / max_clusters) + (rem == 0 ? 0.0 : (2 * rem <= max_clusters ? 0.8 : 1.0));
     const double eff256 = (double)t256 / (c * waves256);
-    return eff512 * kWideGain >= eff256 ? 512 : 256;
+    return eff512 * gain >= eff256 ? 512 : 256;
 }
 
 // Pair-tile rows per raster group.  Measured on GB300 (TFLOP/s, group 4 vs

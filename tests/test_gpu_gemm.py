@@ -501,13 +501,14 @@ def test_reference_unchecked_form_equals_checked_form(f16):
     assert torch.equal(r_chk.view.contiguous().view(torch.int32), r_in.view(torch.int32))
 
 
+@pytest.mark.parametrize("bn", [256, 512])
 @pytest.mark.parametrize("alternate", [0, 1], ids=["forward", "alternating"])
-@pytest.mark.parametrize("M,N,K", [(3072, 3072, 4104), (3072, 2560, 200), (4608, 4608, 1032)])
-def test_k_direction_alternating_by_wave(M, N, K, alternate):
-    # several waves of pair tiles, every other one walking K from its end
-    # (a partial last K stage first); forward and alternating orders are both
-    # within tolerance, and equal in most elements
-    krex.krex_set_tuning(gemm_k_alternate=alternate)
+@pytest.mark.parametrize("M,N,K", [(3072, 3072, 4104), (3072, 2560, 200), (4608, 4608, 1032), (4608, 8192, 1032)])
+def test_k_direction_alternating_by_wave(M, N, K, alternate, bn):
+    # several waves of pair tiles (256 or 512 wide), every other one walking K
+    # from its end (a partial last K stage first); forward and alternating
+    # orders are both within tolerance, and equal in most elements
+    krex.krex_set_tuning(gemm_k_alternate=alternate, gemm_pair_tile_n=bn)
     seed = 8000 + M + N + K
     a, b = _gen(seed, M, N, K)
     c = _candidate(a, b)
@@ -515,7 +516,7 @@ def test_k_direction_alternating_by_wave(M, N, K, alternate):
     ok, worst = _within_tol(bits16(c), want, K)
     assert ok, worst
     if alternate:
-        krex.krex_set_tuning(gemm_k_alternate=0)
+        krex.krex_set_tuning(gemm_k_alternate=0, gemm_pair_tile_n=bn)
         c0 = _candidate(a, b)
         same = (c0.view(torch.int16) == c.view(torch.int16)).float().mean().item()
         assert same > 0.5
