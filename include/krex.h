@@ -134,8 +134,10 @@ krex_status krex_gen_inputs(uint64_t seed, uint32_t tensor_id, int32_t dist, flo
 /* The timed candidate (Section 2.1, Figure 1a's GEMM benchmarking command).
  * KREX_OP_GEMM_BF16: in[0] = A (M x K, bf16), in[1] = B (K x N, bf16), out = C
  *   (M x N, bf16, RNE from the fp32 accumulator).  tcgen05 tensor cores with
- *   TMEM accumulators, TMA loads.  Needs K, N, lda, ldb multiples of 8 and
- *   16-byte aligned A, B (TMA), else UNSUPPORTED.  K = 0 gives C = 0.
+ *   TMEM accumulators, TMA loads; pair tiles of 256 x 256, or 256 x 512 for
+ *   long-K GEMMs (krex_tuning.gemm_pair_tile_n).  Needs K, N, lda, ldb
+ *   multiples of 8 and 16-byte aligned A, B (TMA), else UNSUPPORTED.  K = 0
+ *   gives C = 0.
  * KREX_OP_GEMM_F16: the same with IEEE binary16 A, B and C (RNE out).
  * KREX_OP_SOFTMAX_F32: in[0] = X (rows x cols, fp32), out = Y (same shape,
  *   fp32); y = exp(x - max) / sum exp(x - max) per row, one HBM pass.
@@ -150,10 +152,11 @@ size_t krex_gemm_workspace_bytes(void);
 
 /* krex_run_candidate with an optional GEMM workspace (device memory of >=
  * krex_gemm_workspace_bytes(), 16-byte aligned, zero-filled before its first
- * use; may be NULL).  With it, the tiles of the GEMM's final partial wave are
- * split into two K halves whose fp32 partial sums meet in the workspace (the
- * kernel leaves it ready for the next call); without it they are split into
- * column halves.  One workspace per GEMM in flight: calls that overlap on the
+ * use; may be NULL).  With it, the 256-wide tiles of a GEMM that is one
+ * partial wave are split into two K halves whose fp32 partial sums meet in
+ * the workspace (the kernel leaves it ready for the next call); otherwise the
+ * tiles of a final partial wave are split into column halves (256-wide tiles
+ * only).  One workspace per GEMM in flight: calls that overlap on the
  * GPU must not share it.  After a KREX_ERR_DEVICE status, zero it again.
  * Other ops ignore the workspace.  Asynchronous. */
 krex_status krex_run_candidate_ws(int32_t op, const krex_buf *in, int32_t n_in, krex_buf out,
@@ -518,7 +521,8 @@ krex_status krex_probe_fma(int32_t iters, int32_t blocks, void *dev_sink, krex_s
  * paper: the knobs of this implementation's kernels.  Changing it affects
  * launches issued after the call (it is read once per launch). */
 typedef struct {
-    int32_t gemm_pair_tile_n;  /* columns of a 2-SM pair tile: 0 = 256; else 128, 192, 256 or 512 (two MMAs
+    int32_t gemm_pair_tile_n;  /* columns of a 2-SM pair tile: 0 = by shape (512 for long-K GEMMs whose wide
+                                  tiles fill their waves, else 256); else 128, 192, 256 or 512 (two MMAs
                                   of N = 256 per K step into one 512-column accumulator) */
     int32_t gemm_stage_k;      /* K depth of a shared-memory ring stage: 0 = 128; else 64 or 128 */
     int32_t gemm_ring_stages;  /* stages of the ring in use: 0 = all that fit (3 of K 128, 6 of K 64); else
