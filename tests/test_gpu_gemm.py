@@ -177,6 +177,25 @@ def test_output_row_stride(ldc_pad, variant):
     assert ok, worst
 
 
+@pytest.mark.parametrize("ldc_pad", [0, 8, 3])
+def test_wide_tiles_output_row_stride(ldc_pad):
+    # wide pair tiles (one 512-column accumulator, handed back in halves) with
+    # the TMA-store epilogue and, for rows not on 16 bytes, direct stores;
+    # several tiles per pair, a ragged last chunk; sentinels intact
+    krex.krex_set_tuning(gemm_pair_tile_n=512)
+    M, N, K = 2304, 4104, 520
+    seed = 4100 + ldc_pad
+    a, b = _gen(seed, M, N, K)
+    c = Guarded(M, N, torch.bfloat16, ld=N + ldc_pad)
+    krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [a, b], c.view)
+    torch.cuda.synchronize()
+    assert krex.krex_device_status() == 0
+    assert c.canaries_intact()
+    want = ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N))
+    ok, worst = _within_tol(bits16(c.view), want, K)
+    assert ok, worst
+
+
 @pytest.mark.parametrize("split", ["0", "1"])
 @pytest.mark.parametrize("M,N,K", [(1024, 2048, 512), (4096, 1024, 256), (256, 256, 4096)])
 def test_2sm_tail_split_on_and_off(M, N, K, split):
