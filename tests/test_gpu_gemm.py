@@ -380,6 +380,33 @@ def test_2sm_ragged_edge_items_under_contention():
     assert ok, worst
 
 
+def test_wide_tiles_ragged_edges_under_contention():
+    # the same ragged edges (last row of pair tiles 16 rows high, the last
+    # column chunk partly and wholly outside the matrix) with wide tiles,
+    # whose accumulator halves change hands on every tile, beside a softmax
+    # stream: no wait runs out, and the product is right
+    krex.krex_set_tuning(gemm_pair_tile_n=512)
+    M, N, K = 2064, 2312, 4128
+    a, b = _gen(2065, M, N, K)
+    c = torch.empty(M, N, dtype=torch.bfloat16, device="cuda")
+    x = torch.empty(16384, 8192, dtype=torch.float32, device="cuda")
+    y = torch.empty_like(x)
+    krex.krex_gen_inputs(7, 0, krex.KREX_DIST_NORMAL, 2.0, x)
+    side = torch.cuda.Stream()
+    for _ in range(40):
+        krex.krex_run_candidate(krex.KREX_OP_SOFTMAX_F32, [x], y, stream=side)
+        krex.krex_run_candidate(krex.KREX_OP_GEMM_BF16, [a, b], c)
+    torch.cuda.synchronize()
+    detail = krex.krex_device_status_detail()
+    try:
+        krex.krex_device_status()
+    except krex.KrexError as e:
+        pytest.fail(f"{e}: {detail}")
+    want = ref.gemm_f64(gen.uniform_bf16(2065, 0, M, K), gen.uniform_bf16(2065, 1, K, N))
+    ok, worst = _within_tol(bits16(c), want, K)
+    assert ok, worst
+
+
 # ------------------------------------------------------------- fp16 GEMM ----
 
 def _gen16(seed, M, N, K):
