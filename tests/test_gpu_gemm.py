@@ -177,6 +177,32 @@ def test_output_row_stride(ldc_pad, variant):
     assert ok, worst
 
 
+@pytest.mark.parametrize("tun", [{}, {"gemm_pair_tile_n": 512}, {"gemm_pair_tile_n": 256, "gemm_stage_k": 64},
+                                 {"gemm_pair_tile_n": 192}], ids=["auto", "wide", "k64", "n192"])
+def test_seeded_random_shapes(tun):
+    # twelve shapes drawn from a seeded generator (M, N, K multiples of 8 up
+    # to 2.5k, some tiny), each within tolerance of the oracle, through the
+    # workspace form (K halves where they apply)
+    rng = np.random.default_rng(20261202)
+    krex.krex_set_tuning(**tun)
+    ws = krex.gemm_workspace()
+    for t in range(12):
+        M = int(rng.integers(1, 320)) * 8
+        N = int(rng.integers(1, 320)) * 8
+        K = int(rng.integers(1, 320)) * 8
+        if t < 3:
+            M, N, K = int(rng.integers(1, 9)) * 8, int(rng.integers(1, 9)) * 8, int(rng.integers(1, 9)) * 8
+        seed = 9000 + t
+        a, b = _gen(seed, M, N, K)
+        c = Guarded(M, N, torch.bfloat16)
+        krex.krex_run_candidate_ws(krex.KREX_OP_GEMM_BF16, [a, b], c.view, ws)
+        torch.cuda.synchronize()
+        assert krex.krex_device_status() == 0 and c.canaries_intact(), (M, N, K)
+        want = ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N))
+        ok, worst = _within_tol(bits16(c.view), want, K)
+        assert ok, (M, N, K, worst)
+
+
 @pytest.mark.parametrize("ldc_pad", [0, 8, 3])
 def test_wide_tiles_output_row_stride(ldc_pad):
     # wide pair tiles (one 512-column accumulator, handed back in halves) with
