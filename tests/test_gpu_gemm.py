@@ -198,9 +198,18 @@ def test_seeded_random_shapes(tun):
         krex.krex_run_candidate_ws(krex.KREX_OP_GEMM_BF16, [a, b], c.view, ws)
         torch.cuda.synchronize()
         assert krex.krex_device_status() == 0 and c.canaries_intact(), (M, N, K)
-        want = ref.gemm_f64(gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N))
+        ah, bh = gen.uniform_bf16(seed, 0, M, K), gen.uniform_bf16(seed, 1, K, N)
+        want = ref.gemm_f64(ah, bh)
         ok, worst = _within_tol(bits16(c.view), want, K)
         assert ok, (M, N, K, worst)
+        if not tun:
+            # the reference on the same shape: within the fp32 summation bound
+            r = Guarded(M, N, torch.float32)
+            krex.krex_run_reference(krex.KREX_OP_GEMM_BF16, [a, b], r.view)
+            torch.cuda.synchronize()
+            assert r.canaries_intact()
+            absab = np.abs(gen.bf16_to_f32(ah).astype(np.float64)) @ np.abs(gen.bf16_to_f32(bh).astype(np.float64))
+            assert np.all(np.abs(r.view.cpu().numpy() - want) <= (K + 2) * 2.0 ** -24 * absab + 1e-30), (M, N, K)
 
 
 @pytest.mark.parametrize("ldc_pad", [0, 8, 3])
