@@ -171,3 +171,19 @@ def test_consecutive_checks_alternate_slots_and_stay_exact():
         r = inputs.perturbed(o, 200 + i, 0.05 * (i + 1), 10.0 ** -(i % 4 + 2))
         for sc in (s1, s2) if i % 2 else (s1,):
             _run(o, r, 1e-4, 1e-3, sc)
+
+
+def test_check_seeded_random_shapes(scratch):
+    # ten 2-D shapes from a seeded generator (rows x cols up to ~1.5 M
+    # elements, odd widths), random tolerances and planted violations: count
+    # and max bits equal the oracle's, for the bf16/fp32 and fp32/fp32 pairs
+    rng = np.random.default_rng(20261203)
+    for t in range(10):
+        rows, cols = int(rng.integers(1, 700)), int(rng.integers(1, 2200))
+        n = rows * cols
+        r32 = inputs.normal_f32(500 + t, (rows, cols))
+        o32 = inputs.perturbed(r32, 600 + t, float(rng.uniform(0.01, 0.5)), float(rng.uniform(0.0, 0.2)))
+        atol, rtol = float(rng.choice([0.0, 2.0 ** -8, 1e-3, 0.05])), float(rng.choice([0.0, 2.0 ** -7, 0.01]))
+        for pair in ("bf16_f32", "f32_f32"):
+            o = inputs.bf16_bits_from_f32(o32) if pair.startswith("bf16") else o32
+            _run(o, r32, atol, rtol, scratch)

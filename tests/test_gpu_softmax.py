@@ -138,3 +138,16 @@ def test_softmax_empty_is_noop(rows, cols):
     krex.krex_run_reference(krex.KREX_OP_SOFTMAX_F32, [x.view], y.view)
     torch.cuda.synchronize()
     assert x.canaries_intact() and y.canaries_intact()
+
+
+def test_softmax_seeded_random_shapes():
+    # ten shapes from a seeded generator (widths from 1 to 20000, across every
+    # register-tile size and the online fallback), both kernels within 1e-6
+    rng = np.random.default_rng(20261204)
+    for t in range(10):
+        rows, cols = int(rng.integers(1, 40)), int(rng.integers(1, 20000))
+        x = gen.normal_f32(700 + t, 0, rows, cols, 2.0)
+        y, r = _softmax_both(x)
+        want = ref.softmax_rows_f64(x.astype(np.float64))
+        assert np.max(np.abs(y - want)) <= ATOL, (rows, cols)
+        assert np.max(np.abs(r - want)) <= ATOL, (rows, cols)
