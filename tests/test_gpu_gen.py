@@ -146,3 +146,22 @@ def test_generator_probe_runs_and_leaves_the_context_clean(dist):
     krex.krex_probe_generator(dist, 1 << 20, n_sm, sink)
     torch.cuda.synchronize()
     assert krex.krex_device_status() == 0
+
+
+def test_fills_seeded_random_shapes_and_strides():
+    # twelve shapes and row strides from a seeded generator, seeds and tensor
+    # ids drawn too: every fill bit-identical to the oracle, padding untouched
+    rng = np.random.default_rng(20261205)
+    for t in range(12):
+        rows, cols = int(rng.integers(1, 300)), int(rng.integers(1, 3000))
+        pad = int(rng.choice([0, 0, 1, 3, 8, 17]))
+        seed, tid = int(rng.integers(0, 2 ** 63)), int(rng.integers(0, 4))
+        g = Guarded(rows, cols, torch.bfloat16, ld=cols + pad if pad else None)
+        krex.krex_gen_inputs(seed, tid, krex.KREX_DIST_UNIFORM_PM1, 0.0, g.view)
+        f = Guarded(rows, cols, torch.float32, ld=cols + pad if pad else None)
+        krex.krex_gen_inputs(seed, tid, krex.KREX_DIST_NORMAL, 2.0, f.view)
+        torch.cuda.synchronize()
+        assert g.canaries_intact() and f.canaries_intact(), (rows, cols, pad)
+        assert np.array_equal(bits16(g.view), gen.uniform_bf16(seed, tid, rows, cols)), (rows, cols, pad)
+        got = f.view.contiguous().cpu().numpy()
+        assert np.array_equal(got.view(np.uint32), gen.normal_f32(seed, tid, rows, cols, 2.0).view(np.uint32)), (rows, cols, pad)
