@@ -124,14 +124,43 @@ class ClockSampler:
 
 # ------------------------------------------------------------ helpers -------
 
-def _src_hash(path: str) -> str:
-    with open(path, "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+def code_text(src: str) -> str:
+    """C/C++/CUDA source with its comments removed and every run of whitespace
+    made one space: what the compiler sees, so an edit of comments or layout
+    leaves it unchanged and any other edit changes it.  String and character
+    literals are kept whole (a // inside one is not a comment)."""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        c = src[i]
+        if c in "\"'":
+            j = i + 1
+            while j < n and src[j] != c:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        elif src.startswith("//", i):
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+        elif src.startswith("/*", i):
+            j = src.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+            out.append(" ")
+        else:
+            out.append(c)
+            i += 1
+    return " ".join("".join(out).split())
+
+
+def code_hash(path: str) -> str:
+    """First 16 hex digits of the sha256 of code_text(path)."""
+    with open(path, encoding="utf-8") as f:
+        return hashlib.sha256(code_text(f.read()).encode()).hexdigest()[:16]
 
 
 def _ncu_traffic(kernel: str, workload: str):
     """DRAM bytes per launch of `kernel` from the committed ncu summary, or None
-    if the kernel source changed since the capture."""
+    if the kernel's code changed since the capture (the record keeps the hash
+    of the code it was taken on; edits of comments alone keep it valid)."""
     p = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     if not os.path.exists(p):
         return None
@@ -141,7 +170,7 @@ def _ncu_traffic(kernel: str, workload: str):
     if not e:
         return None
     src = os.path.join(ROOT, e["source"])
-    if not os.path.exists(src) or _src_hash(src) != e["source_sha256_16"]:
+    if not os.path.exists(src) or code_hash(src) != e["code_sha256_16"]:
         return None
     return e["dram_bytes_per_launch"]
 

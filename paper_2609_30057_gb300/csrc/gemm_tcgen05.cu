@@ -5,15 +5,21 @@
 //
 // Default form, gemm_tcgen05_2sm: a cluster of two CTAs (a TPC) computes a
 // 256 x bn pair tile with tcgen05.mma.cta_group::2 (M = 256, K = 16); a
-// persistent grid holds one cluster per co-resident SM pair.  Per CTA:
+// persistent grid holds one cluster per co-resident SM pair.  Pair tiles are
+// up to 256 wide (one MMA of N = bn per K step) or 256 x 512 (two MMAs of
+// N = 256 per K step sharing the A operand; picked for long K, where the
+// SM's load rate rather than the tail decides).  Per CTA:
 //   warp 0      TMA producer: A (K-major) and its half of B (N-major) tiles,
-//               128-byte swizzle, into a ring of 128-deep K stages; both CTAs'
-//               loads complete on the leader's full barrier, on which the peer
-//               producer also arrives.
-//   warp 1      (leader only) MMA issuer: one thread, 8 MMAs per stage, each
-//               stage released to both producers by a multicast commit.
-//   warp 2      allocates / frees 512 TMEM columns: two accumulators, so the
-//               epilogue of one tile overlaps the MMAs of the next.
+//               128-byte swizzle, into a ring of 64- or 128-deep K stages;
+//               both CTAs' loads complete on the leader's full barrier, on
+//               which the peer producer also arrives.
+//   warp 1      (leader only) MMA issuer: one thread, 4 or 8 MMAs per stage,
+//               each stage released to both producers by a multicast commit.
+//   warp 2      allocates / frees 512 TMEM columns: two 256-column
+//               accumulators, so the epilogue of one tile overlaps the MMAs
+//               of the next, or one 512-column accumulator for 256 x 512
+//               tiles, handed back in halves so that the next tile's first
+//               MMAs start while its second half is still read.
 //   warps 4-7   epilogue: tcgen05.ld of 32 rows each, 16-bit RNE, TMA store
 //               from 128B-swizzled staging (direct stores when C's rows are
 //               not 16-byte aligned).
@@ -242,7 +248,12 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
 // A tile and columns [128r, 128r+128) of the B tile in its own shared memory,
 // and its own TMEM holds its 128 rows of the 256-column accumulator.  Per SM
 // a stage is 32 KiB (A 128x64 + half of B 64x128), so six stages fit and the
-// L2 -> SM traffic per flop is two thirds of a one-SM 128 x 256 tile's.
+// L2 -> SM traffic per flop is two thirds of a one-SM 128 x 256 tile's.  A
+// 256 x 512 tile is two such column chunks side by side: each CTA holds the
+// 128-column halves of both chunks of B (48 KiB per 64-deep stage with A),
+// the MMA thread issues one MMA per chunk and K step into columns
+// [256c, 256c + 256) of one 512-column accumulator, and each SM loads 48
+// bytes per MMA cycle instead of 64.
 //   - both CTAs' TMA loads complete on the leader CTA's (rank 0) full barrier
 //     (.cta_group::2 lets the barrier live in the peer CTA);
 //   - the leader's MMA thread releases a stage in both CTAs and publishes an
@@ -263,7 +274,7 @@ constexpr int RING_BYTES = 6 * (A_SUB_BYTES + B_SUB_BYTES);  // 192 KiB of stage
 constexpr int EPI_BOX_COLS = 64;                 // TMA-store box: 64 columns x 32 rows (4 KiB)
 constexpr int EPI_BUF_BYTES = 32 * EPI_BOX_COLS * 2;
 constexpr int EPI_BYTES = 4 * 2 * EPI_BUF_BYTES; // 4 epilogue warps x 2 buffers
-constexpr int TMEM_COLS = 2 * BN;                // two 128-lane x 256-column accumulators
+constexpr int TMEM_COLS = 2 * BN;                // two 256-column accumulators, or one of 512
 constexpr int GROUP_M = 8;                       // pair-tile rows per raster group (see raster_group)
 constexpr int EPI_WARPS = 4;
 // A stage holds KSUB K sub-blocks (KSUB x 64 of K) of A and of NCH 256-column
