@@ -33,7 +33,7 @@ def _rank_main(rank, world, port, results):
 def test_two_replicas_aggregate_over_gloo():
     world = 2
     port = _free_port()
-    with mp.Manager() as m:
+    with mp.get_context("spawn").Manager() as m:   # no fork of a threaded process
         results = m.dict()
         mp.spawn(_rank_main, args=(world, port, results), nprocs=world, join=True)
         res = dict(results)
