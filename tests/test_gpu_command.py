@@ -255,3 +255,52 @@ def test_host_buffer_sizes_round_trip(nbytes):
     back.copy_(d, non_blocking=True)
     torch.cuda.synchronize()
     assert np.array_equal(back.numpy(), g)
+
+
+def test_softmax_65536x8192_command_against_the_oracle():
+    # the softmax workload's command at its full size (two timed iterations
+    # instead of a hundred): its input on sampled rows bit for bit, the
+    # candidate and the reference on 4096 oracle-sampled rows, and the verdict
+    # over all 2^29 outputs equal to the oracle's check of the downloaded buffers
+    w = scaled(WORKLOADS["softmax_f32_65536x8192"], iters=2)
+    ws = Workspace(w)
+    res = ws.run()
+    assert res.passed == 1 and res.n_iters == 2 and krex.krex_device_status() == 0
+    rows, cols = w.M, w.N
+    sample, _ = ref.sample_indices(w.seed, 3, 4096, rows, 1)
+    sample = np.unique(sample)
+    xs = np.stack([gen.normal_f32_at(w.seed, 0, np.arange(i * cols, (i + 1) * cols), w.sigma) for i in sample])
+    st = torch.from_numpy(sample).cuda()
+    assert np.array_equal(ws.inputs[0][st].cpu().numpy().view(np.uint32), xs.view(np.uint32))
+    want = ref.softmax_rows_f64(xs.astype(np.float64))
+    assert np.max(np.abs(ws.out[st].cpu().numpy() - want)) <= ref.SOFTMAX_ATOL
+    assert np.max(np.abs(ws.ref[st].cpu().numpy() - want)) <= ref.SOFTMAX_ATOL
+    mx, nv = ref.check_f32(ws.out.cpu().numpy(), ws.ref.cpu().numpy(), w.atol, w.rtol)
+    assert nv == 0 == int(res.check.n_violations)
+    assert ref.check_bits(res.check.max_abs_err) == ref.check_bits(mx)
+
+
+def test_gemm_8192_command_against_the_oracle():
+    # the 8192^3 command (wide pair tiles by the launch code's rule; two timed
+    # iterations instead of fifty): 4096 oracle-sampled outputs of the
+    # candidate and of the reference, and the verdict over all 2^26 outputs
+    # equal to the oracle's check of the downloaded buffers
+    w = scaled(WORKLOADS["gemm_bf16_8192"], iters=2)
+    ws = Workspace(w)
+    res = ws.run()
+    assert res.passed == 1 and res.n_iters == 2 and krex.krex_device_status() == 0
+    n = w.M
+    i, j = ref.sample_indices(w.seed, 2, 4096, n, n)
+    want = ref.gemm_sampled_f64(w.seed, n, n, n, i, j)
+    ti, tj = torch.from_numpy(i).cuda(), torch.from_numpy(j).cuda()
+    got = gen.bf16_to_f32(bits16(ws.out[ti, tj])).astype(np.float64)
+    assert np.all(np.abs(got - want) <= ref.gemm_tolerance(want, n))
+    r = ws.ref[ti, tj].cpu().numpy().astype(np.float64)
+    kk = np.arange(n, dtype=np.int64)
+    for s_ in range(256):
+        ra = np.abs(gen.widen("bf16", gen.uniform_at("bf16", w.seed, 0, i[s_] * n + kk)).astype(np.float64))
+        cb = np.abs(gen.widen("bf16", gen.uniform_at("bf16", w.seed, 1, kk * n + j[s_])).astype(np.float64))
+        assert abs(r[s_] - want[s_]) <= n * 2.0 ** -24 * float(ra @ cb), s_
+    mx, nv = ref.check_f32(gen.bf16_to_f32(bits16(ws.out)), ws.ref.cpu().numpy(), w.atol, w.rtol)
+    assert nv == 0 == int(res.check.n_violations)
+    assert ref.check_bits(res.check.max_abs_err) == ref.check_bits(mx)
