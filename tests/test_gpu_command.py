@@ -304,3 +304,26 @@ def test_gemm_8192_command_against_the_oracle():
     mx, nv = ref.check_f32(gen.bf16_to_f32(bits16(ws.out)), ws.ref.cpu().numpy(), w.atol, w.rtol)
     assert nv == 0 == int(res.check.n_violations)
     assert ref.check_bits(res.check.max_abs_err) == ref.check_bits(mx)
+
+
+@pytest.mark.parametrize("name", ["gemm_bf16_4096", "gemm_f16_4096"])
+def test_gemm_4096_command_full_output_against_the_oracle(name):
+    # the 4096^3 commands (bf16 and binary16; five timed iterations instead of
+    # a hundred): the inputs bit for bit, every output of the candidate within
+    # the tolerance of the oracle's fp64 product, the reference within the
+    # fp32 summation bound, and the verdict equal to the oracle's check
+    w = scaled(WORKLOADS[name], iters=5)
+    ws = Workspace(w)
+    res = ws.run()
+    assert res.passed == 1 and res.n_iters == 5 and krex.krex_device_status() == 0
+    ah, bh = gen.uniform(w.dtype, w.seed, 0, w.M, w.K), gen.uniform(w.dtype, w.seed, 1, w.K, w.N)
+    assert np.array_equal(bits16(ws.inputs[0]), ah) and np.array_equal(bits16(ws.inputs[1]), bh)
+    want = ref.gemm_f64(ah, bh, dtype=w.dtype)
+    out = gen.widen(w.dtype, bits16(ws.out))
+    assert np.all(np.abs(out.astype(np.float64) - want) <= ref.gemm_tolerance(want, w.K, dtype=w.dtype))
+    r32 = ws.ref.cpu().numpy()
+    fa, fb = gen.widen(w.dtype, ah).astype(np.float64), gen.widen(w.dtype, bh).astype(np.float64)
+    assert np.all(np.abs(r32 - want) <= w.K * 2.0 ** -24 * (np.abs(fa) @ np.abs(fb)))
+    mx, nv = ref.check_f32(out, r32, w.atol, w.rtol)
+    assert nv == 0 == int(res.check.n_violations)
+    assert ref.check_bits(res.check.max_abs_err) == ref.check_bits(mx)
