@@ -214,3 +214,26 @@ def test_fma_probe_rejects_bad_arguments():
     assert lib.krex_probe_fma(16, 1, None, None) == krex.KREX_ERR_INVALID
     assert lib.krex_probe_fma(0, 1, 16, None) == krex.KREX_ERR_INVALID
     assert lib.krex_probe_fma(16, 0, 16, None) == krex.KREX_ERR_INVALID
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    # without libkrex.so every entry point raises: the binding has no CPU or
+    # PyTorch fallback for any step of the path
+    import subprocess
+    import sys
+    code = (
+        "import paper_2609_30057_gb300 as k, torch\n"
+        f"k.LIB_PATH = {str(tmp_path / 'absent' / 'libkrex.so')!r}\n"
+        "k._lib = None\n"
+        "calls = [lambda: k.krex_gen_inputs(1, 0, 0, 0.0, torch.empty(8, 8, dtype=torch.bfloat16)),\n"
+        "         lambda: k.krex_check_scratch_bytes(), lambda: k.krex_set_tuning()]\n"
+        "for c in calls:\n"
+        "    try:\n"
+        "        c()\n"
+        "    except RuntimeError as e:\n"
+        "        assert 'no fallback' in str(e), e\n"
+        "    else:\n"
+        "        raise SystemExit('a call ran without the library')\n"
+        "print('raised')\n")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, cwd=ROOT, timeout=300)
+    assert r.returncode == 0 and r.stdout.strip().endswith("raised"), r.stdout + r.stderr
